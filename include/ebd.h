@@ -1,0 +1,185 @@
+/*
+ * ebd.h -- C ABI of the eviction-by-design (EBD) hot path on GB300 (sm_103a).
+ *
+ * Method: "Error Certificates for KV-Cache Eviction via Randomized Design"
+ * (arXiv 2607.21475).  Per (batch row, KV head) unit the eviction step keeps
+ * a certainty set A (attention sinks, a recency window, the score top slice),
+ * draws a Poisson tail T = C \ A at known inclusion probabilities pi_i
+ * (Section 3.3, Eq. 2) and compacts the survivors with one scalar
+ * log(1/pi_i) each.  The certified decode step is Hajek-corrected attention
+ * over the compact cache (Eq. 3) plus the design-based variance estimate
+ * V_hat (Theorem 2) and the empirical-Bernstein radius r_t (Section 3.4,
+ * Eq. 4), all from one pass over the compact cache.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Every pointer argument named as "device" is a CUDA device pointer into
+ *   memory the caller owns (allocated by the caller, freed by the caller).
+ *   The library never allocates, never frees, and keeps no pointer after the
+ *   call returns.  `workspace` is caller-owned scratch of the size reported
+ *   by the matching *_workspace_bytes query.
+ * - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *   stream).  Every call only enqueues work on it and returns: results are
+ *   valid once the stream has been synchronised.
+ * - Tensors are dense, row-major, with the last dimension contiguous.
+ *   B = batch, Hkv = KV heads, G = query heads per KV head (Hq = Hkv * G),
+ *   d = head_dim, N = context length, cap = compact-cache capacity per unit.
+ * - Argument errors are detected on the host and returned synchronously;
+ *   nothing is enqueued in that case.  Data-dependent conditions found on
+ *   the device are OR-ed into the caller's `dev_status` word (device int32,
+ *   which the caller zeroes) as EBD_DEV_* bits; the call never traps,
+ *   asserts or spins without a bound.
+ * - dtype EBD_F32 or EBD_BF16 applies to K, V, Q, q_obs and the compact
+ *   K_c, V_c; scores, pi, logw and every decode output are float32.
+ */
+#ifndef EBD_H_
+#define EBD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  EBD_OK = 0,
+  EBD_ERR_INVALID = 1,     /* null pointer, non-positive or inconsistent size     */
+  EBD_ERR_CAPACITY = 2,    /* capacity or workspace smaller than the call needs  */
+  EBD_ERR_NONFINITE = 3,   /* reserved: non-finite scores are reported on device */
+  EBD_ERR_UNSUPPORTED = 4, /* valid request outside what this build implements   */
+  EBD_ERR_CUDA = 5         /* a CUDA runtime call or kernel launch failed        */
+} ebd_status;
+
+typedef enum { EBD_F32 = 0, EBD_BF16 = 1 } ebd_dtype;
+
+/* Range term b_t of Eq. (4).  BOUND (default) is the one-pass triangle
+ * inequality bound  (max sqrt(1-pi) w ||v|| + ||y_hat|| max sqrt(1-pi) w) / N_hat,
+ * never below the definition.  EXACT evaluates the definition
+ * max_{S cap T} sqrt(1-pi_i) w_i ||v_i - y_hat|| / N_hat with a second pass over
+ * the compact cache once y_hat is known. */
+typedef enum { EBD_RANGE_BOUND = 0, EBD_RANGE_EXACT = 1 } ebd_range_mode;
+
+/* Bits OR-ed into *dev_status by device code. */
+#define EBD_DEV_CAPACITY 0x1  /* a unit kept more than `capacity` tokens; rows past
+                                 capacity were dropped, n_kept holds the true count */
+#define EBD_DEV_NONFINITE 0x2 /* a score was NaN or +-inf; that unit's output is
+                                 unspecified (but every write stays in bounds)       */
+#define EBD_DEV_TIMEOUT 0x4   /* an in-kernel pipeline wait hit its bound and the
+                                 kernel returned early; outputs are unspecified      */
+
+/* Design of one layer's eviction (Section 3.3 and Appendix B of the paper). */
+typedef struct {
+  int32_t batch;         /* B                                                    */
+  int32_t n_kv_heads;    /* Hkv                                                  */
+  int32_t group;         /* G, query heads per KV head (used by scoring only)    */
+  int32_t head_dim;      /* d                                                    */
+  int32_t n_ctx;         /* N, cached tokens per unit, 1 <= N <= 2^20            */
+  int32_t layer;         /* layer index: Philox counter word 2                   */
+  uint64_t seed;         /* Philox key = (seed & 0xffffffff, seed >> 32)         */
+  int32_t n_sink;        /* protected leading positions (attention sinks), 4     */
+  int32_t n_recent;      /* protected trailing positions (recency window), 32    */
+  int32_t k_head;        /* size of the score top slice (ties to lower index)    */
+  int32_t budget_tokens; /* B_t: expected retained tokens per unit (A + tail)    */
+  int32_t bisect_iters;  /* bisection steps for the scale c of Eq. (2), 1..200   */
+  float eps;             /* probability floor, 1e-6 in the paper                 */
+} ebd_design;
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char* ebd_status_string(ebd_status status);
+
+/* ABI version of this library (increments on any signature change). */
+int32_t ebd_abi_version(void);
+
+/*
+ * Philox4x32-10 words used by the Poisson draw (Section 3.3: independent
+ * Bernoulli(pi_i) retention on the tail).  For every unit (b, kvh) and token
+ * i < N writes x0[b,kvh,i] (device uint32 [B,Hkv,N]) = the first output word
+ * of Philox4x32-10 (Salmon et al., SC'11) with key (seed_lo, seed_hi) and
+ * counter (i, kvh, layer, b).  The uniform the draw compares with pi_i is
+ * (x0 >> 8) * 2^-24.  Exposed so that the draws can be checked bit for bit.
+ */
+ebd_status ebd_philox_uniforms(uint64_t seed, int32_t layer, int32_t batch, int32_t n_kv_heads,
+                               int32_t n_ctx, uint32_t* x0, void* stream);
+
+/*
+ * Accumulated-attention importance scores (Appendix B, harness: H2O-style
+ * accumulated attention from observation queries).
+ *   q_obs  device [B,Hkv,R,d] (dtype): the R = n_obs observation query rows
+ *          of every query head of the KV head's group
+ *   K      device [B,Hkv,N,d] (dtype)
+ *   scores device [B,Hkv,N] float32 out: s_j = sum_r softmax_j(q_r . K^T / sqrt(d))
+ * Needs workspace of ebd_score_workspace_bytes(B, Hkv, R) bytes.
+ * Supports d in {64, 128}, 1 <= R <= 4096.
+ */
+size_t ebd_score_workspace_bytes(int32_t batch, int32_t n_kv_heads, int32_t n_obs);
+ebd_status ebd_score(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads, int32_t head_dim,
+                     int32_t n_ctx, int32_t n_obs, const void* q_obs, const void* K,
+                     float* scores, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Certainty set and inclusion probabilities (Section 3.3, Eq. 2).
+ *   scores       device [B,Hkv,N] float32 importance scores
+ *   pi           device [B,Hkv,N] float32 out: 1 on A; clip(c * s_i, eps, 1) on T
+ *                with c such that sum_T pi_i = m = clamp(B_t - |A|, 0, |T|)
+ *                (clip-saturated tokens join A; scores <= 0 sit at eps)
+ *   certain_mask device [B,Hkv,N] uint8 out, nullable: 1 iff token in A
+ *   dev_status   device int32, nullable: EBD_DEV_NONFINITE
+ */
+ebd_status ebd_compute_pi(const ebd_design* design, const float* scores, float* pi,
+                          uint8_t* certain_mask, int32_t* dev_status, void* stream);
+
+/*
+ * Full eviction step of one layer (Section 3.3, Appendix B): certainty set,
+ * Eq. (2) probabilities, Poisson draw, stable compaction.
+ *   K, V      device [B,Hkv,N,d] (dtype)
+ *   scores    device [B,Hkv,N] float32; or NULL together with q_obs
+ *             (device [B,Hkv,n_obs,d]), in which case the scores are computed
+ *             as by ebd_score
+ *   K_c, V_c  device [B,Hkv,cap,d] (dtype) out: kept rows in increasing token order
+ *   logw_c    device [B,Hkv,cap] float32 out: log(1/pi_i) of each kept row (0 on A)
+ *   idx_c     device [B,Hkv,cap] int32 out, nullable: token index of each kept row
+ *   n_kept    device [B,Hkv] int32 out: number of kept tokens (may exceed cap, in
+ *             which case EBD_DEV_CAPACITY is raised and rows >= cap are dropped)
+ *   dev_status device int32, required
+ * Rows [n_kept, cap) of the outputs are left untouched.  Needs workspace of
+ * ebd_evict_workspace_bytes(...) bytes (0 when scores are given).
+ */
+size_t ebd_evict_workspace_bytes(const ebd_design* design, int32_t n_obs);
+ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const void* K, const void* V,
+                     const float* scores, const void* q_obs, int32_t n_obs, void* K_c, void* V_c,
+                     float* logw_c, int32_t* idx_c, int32_t* n_kept, int32_t capacity,
+                     int32_t* dev_status, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Certified decode step (Eq. 3, Theorem 2, Eq. 4) for every query head.
+ *   Q        device [B,Hkv*G,d] (dtype): query heads kvh*G .. kvh*G+G-1 read the
+ *            compact cache of KV head kvh
+ *   K_c,V_c  device [B,Hkv,cap,d] (dtype); logw_c device [B,Hkv,cap] float32
+ *   n_kept   device [B,Hkv] int32 (values above cap are read as cap)
+ *   delta    confidence parameter (0.1 in the paper); eps0 normaliser (1e-9)
+ *   y        device [B,Hkv*G,d] float32 out: y_hat of Eq. (3)
+ *   lse      device [B,Hkv*G] float32 out: log N_hat (-inf for an empty unit)
+ *   var_hat  device [B,Hkv*G] float32 out: V_hat of Theorem 2
+ *   b_t      device [B,Hkv*G] float32 out: range term (see ebd_range_mode)
+ *   radius   device [B,Hkv*G] float32 out: r_t of Eq. (4)
+ *   dev_status device int32, nullable
+ * An empty unit (n_kept = 0) gives y = 0, lse = -inf and a zero certificate.
+ * Needs workspace of ebd_decode_workspace_bytes(...) bytes for the split-K
+ * partial records.  Supports d in {64, 128} and 1 <= G <= 8.
+ */
+size_t ebd_decode_workspace_bytes(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads,
+                                  int32_t group, int32_t head_dim, int32_t capacity);
+ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads, int32_t group,
+                                int32_t head_dim, const void* Q, const void* K_c, const void* V_c,
+                                const float* logw_c, const int32_t* n_kept, int32_t capacity,
+                                float delta, float eps0, ebd_range_mode range_mode, float* y,
+                                float* lse, float* var_hat, float* b_t, float* radius,
+                                int32_t* dev_status, void* workspace, size_t ws_bytes,
+                                void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* EBD_H_ */

@@ -1,0 +1,474 @@
+// Certified decode over the compact cache (Section 3.3 Eq. 3, Theorem 2,
+// Section 3.4 Eq. 4 of the paper), split-K over the retained tokens.
+//
+// Each split of each (batch row, KV head) unit streams its K_c, V_c, logw_c
+// rows once and keeps, per query head of the group, an online-softmax state
+// relative to its running maximum logit M:
+//   l  = sum w_i                    w_i = exp(q.k_i/sqrt(d) + log(1/pi_i) - M)
+//   o  = sum w_i v_i                (Hajek numerator, Eq. 3)
+//   U  = sum u_i,  u_i = (1 - pi_i) w_i^2   (Theorem 2 weights)
+//   A1 = sum u_i v_i,  A2 = sum u_i ||v_i||^2
+//   cmax = max sqrt(u_i) ||v_i||,  umax = max sqrt(u_i)   (range-term bound)
+// A maximum increase by D rescales the w-terms by e^-D and the u-terms by
+// e^-2D.  The reduce kernel merges the splits the same way and finishes
+//   y_hat = o / l,   lse = M + log l  (= log N_hat),
+//   V_hat = (A2 - 2 y_hat.A1 + ||y_hat||^2 U) / l^2 = sum u_i ||v_i - y_hat||^2 / l^2,
+//   b_t   = (cmax + ||y_hat|| umax) / l   (bound; >= the definition),
+//   r_t   = (sqrt(2 V_hat ln(1/delta)) + b_t ln(1/delta)) / (||y_hat|| + eps0).
+// The exact range term, max_i sqrt(u_i) ||v_i - y_hat|| / l, needs y_hat and is
+// a second pass over the tail rows (EBD_RANGE_EXACT).
+//
+// This file holds the CUDA-core path (any supported dtype, head_dim 64/128,
+// G <= 8).  Its record layout and reduce are shared with the tensor-core path.
+#include <cuda_runtime.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "decode.cuh"
+#include "internal.h"
+
+namespace ebd {
+
+constexpr int kGenThreads = 128;
+constexpr int kGenWarps = kGenThreads / 32;
+
+template <typename T, int D, int GM>
+__global__ void __launch_bounds__(kGenThreads) decode_generic_kernel(DecodeArgs a) {
+  constexpr int E = D / 32;
+  constexpr int REC = rec_floats(D);
+  __shared__ float st[kGenWarps][GM][REC];
+  const int unit = blockIdx.y, split = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = a.group;
+  const int b = unit / a.n_kv_heads, kvh = unit - b * a.n_kv_heads;
+  const int n = min(a.n_kept[unit], a.cap);
+  const int t0 = split * a.tokens_per_split;
+  const int t1 = min(n, t0 + a.tokens_per_split);
+  const float scale = rsqrtf((float)D);
+  const T* Q = (const T*)a.Q + ((size_t)b * a.n_kv_heads * G + (size_t)kvh * G) * D;
+  const T* Kc = (const T*)a.Kc + (size_t)unit * a.cap * D;
+  const T* Vc = (const T*)a.Vc + (size_t)unit * a.cap * D;
+  const float* lw = a.logw + (size_t)unit * a.cap;
+
+  float q[GM][E], o[GM][E], a1[GM][E];
+  float M[GM], l[GM], U[GM], A2[GM], cmax[GM], umax[GM];
+#pragma unroll
+  for (int g = 0; g < GM; ++g) {
+#pragma unroll
+    for (int j = 0; j < E; ++j) {
+      q[g][j] = g < G ? to_f32(Q[(size_t)g * D + lane + 32 * j]) * scale : 0.f;
+      o[g][j] = 0.f;
+      a1[g][j] = 0.f;
+    }
+    M[g] = -INFINITY;
+    l[g] = U[g] = A2[g] = cmax[g] = umax[g] = 0.f;
+  }
+  for (int t = t0 + warp; t < t1; t += kGenWarps) {
+    float k[E], v[E];
+#pragma unroll
+    for (int j = 0; j < E; ++j) {
+      k[j] = to_f32(Kc[(size_t)t * D + lane + 32 * j]);
+      v[j] = to_f32(Vc[(size_t)t * D + lane + 32 * j]);
+    }
+    const float lwt = lw[t];
+    const float omp = -expm1f(-lwt);  // 1 - pi
+    const float sq = sqrtf(omp);
+    float vn2 = 0.f;
+#pragma unroll
+    for (int j = 0; j < E; ++j) vn2 = fmaf(v[j], v[j], vn2);
+    vn2 = warp_sum(vn2);
+    const float vn = sqrtf(vn2);
+#pragma unroll
+    for (int g = 0; g < GM; ++g) {
+      if (g >= G) break;
+      float dot = 0.f;
+#pragma unroll
+      for (int j = 0; j < E; ++j) dot = fmaf(q[g][j], k[j], dot);
+      const float x = warp_sum(dot) + lwt;
+      if (x > M[g]) {
+        const float f = expf(M[g] - x), f2 = f * f;
+        l[g] *= f;
+        U[g] *= f2;
+        A2[g] *= f2;
+        cmax[g] *= f;
+        umax[g] *= f;
+#pragma unroll
+        for (int j = 0; j < E; ++j) {
+          o[g][j] *= f;
+          a1[g][j] *= f2;
+        }
+        M[g] = x;
+      }
+      const float w = expf(x - M[g]);
+      const float u = omp * w * w;
+      const float su = sq * w;
+      l[g] += w;
+      U[g] += u;
+      A2[g] = fmaf(u, vn2, A2[g]);
+      cmax[g] = fmaxf(cmax[g], su * vn);
+      umax[g] = fmaxf(umax[g], su);
+#pragma unroll
+      for (int j = 0; j < E; ++j) {
+        o[g][j] = fmaf(w, v[j], o[g][j]);
+        a1[g][j] = fmaf(u, v[j], a1[g][j]);
+      }
+    }
+  }
+  // merge the warps' states
+#pragma unroll
+  for (int g = 0; g < GM; ++g) {
+    if (lane == 0) {
+      st[warp][g][kRecM] = M[g];
+      st[warp][g][kRecL] = l[g];
+      st[warp][g][kRecU] = U[g];
+      st[warp][g][kRecA2] = A2[g];
+      st[warp][g][kRecCmax] = cmax[g];
+      st[warp][g][kRecUmax] = umax[g];
+    }
+#pragma unroll
+    for (int j = 0; j < E; ++j) {
+      st[warp][g][kRecHead + lane + 32 * j] = o[g][j];
+      st[warp][g][kRecHead + D + lane + 32 * j] = a1[g][j];
+    }
+  }
+  __syncthreads();
+  float* out = a.part + ((size_t)unit * a.splits + split) * (size_t)G * REC;
+  for (int idx = threadIdx.x; idx < G * REC; idx += kGenThreads) {
+    const int g = idx / REC, e = idx - g * REC;
+    float Mx = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < kGenWarps; ++w) Mx = fmaxf(Mx, st[w][g][kRecM]);
+    float r;
+    if (e == kRecM) {
+      r = Mx;
+    } else {
+      const bool sq2 = rec_is_squared(e, D);
+      const bool is_max = (e == kRecCmax || e == kRecUmax);
+      r = 0.f;
+#pragma unroll
+      for (int w = 0; w < kGenWarps; ++w) {
+        const float Mw = st[w][g][kRecM];
+        const float f = (Mw == -INFINITY) ? 0.f : expf(Mw - Mx);
+        const float x = st[w][g][e] * (sq2 ? f * f : f);
+        r = is_max ? fmaxf(r, x) : r + x;
+      }
+    }
+    out[idx] = r;
+  }
+}
+
+// Merge the split records of one query head and finish Eq. (3), Theorem 2, Eq. (4).
+template <int D>
+__global__ void __launch_bounds__(D) decode_reduce_kernel(ReduceArgs a) {
+  constexpr int REC = rec_floats(D);
+  __shared__ float red[2][D / 32];
+  const int hq = blockIdx.x;
+  const int G = a.group;
+  const int unit = hq / G, g = hq - unit * G;
+  const int e = threadIdx.x;
+  const float* P = a.part + ((size_t)unit * a.splits * G + g) * REC;
+  const size_t sstride = (size_t)G * REC;
+  float Mx = -INFINITY;
+  for (int s = 0; s < a.splits; ++s) Mx = fmaxf(Mx, P[s * sstride + kRecM]);
+  if (Mx == -INFINITY) {  // empty unit
+    a.y[(size_t)hq * D + e] = 0.f;
+    if (e == 0) {
+      a.lse[hq] = -INFINITY;
+      a.var[hq] = 0.f;
+      a.b_t[hq] = 0.f;
+      a.radius[hq] = 0.f;
+    }
+    return;
+  }
+  float l = 0.f, U = 0.f, A2 = 0.f, cmax = 0.f, umax = 0.f, o = 0.f, a1 = 0.f;
+  for (int s = 0; s < a.splits; ++s) {
+    const float* R = P + s * sstride;
+    const float Ms = R[kRecM];
+    if (Ms == -INFINITY) continue;
+    const float f = expf(Ms - Mx), f2 = f * f;
+    l += f * R[kRecL];
+    U += f2 * R[kRecU];
+    A2 += f2 * R[kRecA2];
+    cmax = fmaxf(cmax, f * R[kRecCmax]);
+    umax = fmaxf(umax, f * R[kRecUmax]);
+    o += f * R[kRecHead + e];
+    a1 += f2 * R[kRecHead + D + e];
+  }
+  const float y = o / l;
+  a.y[(size_t)hq * D + e] = y;
+  float yy = warp_sum(y * y), ya = warp_sum(y * a1);
+  if ((e & 31) == 0) {
+    red[0][e >> 5] = yy;
+    red[1][e >> 5] = ya;
+  }
+  __syncthreads();
+  if (e == 0) {
+    yy = 0.f;
+    ya = 0.f;
+#pragma unroll
+    for (int w = 0; w < D / 32; ++w) {
+      yy += red[0][w];
+      ya += red[1][w];
+    }
+    const float ynorm = sqrtf(yy);
+    const float var = fmaxf(0.f, (A2 - 2.f * ya + yy * U) / (l * l));
+    a.lse[hq] = Mx + logf(l);
+    a.var[hq] = var;
+    if (a.exact) {
+      a.b_t[hq] = 0.f;  // filled by the exact range pass
+    } else {
+      const float bt = (cmax + ynorm * umax) / l;
+      a.b_t[hq] = bt;
+      a.radius[hq] = (sqrtf(2.f * var * a.log_inv_delta) + bt * a.log_inv_delta) / (ynorm + a.eps0);
+    }
+  }
+}
+
+// EBD_RANGE_EXACT, pass 2: max over tail rows of sqrt(1-pi_i) w_i ||v_i - y_hat|| / N_hat.
+template <typename T, int D, int GM>
+__global__ void __launch_bounds__(kGenThreads) decode_exact_range_kernel(DecodeArgs a) {
+  constexpr int E = D / 32;
+  __shared__ float smax[kGenWarps][GM];
+  const int unit = blockIdx.y, split = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = a.group;
+  const int b = unit / a.n_kv_heads, kvh = unit - b * a.n_kv_heads;
+  const int n = min(a.n_kept[unit], a.cap);
+  const int t0 = split * a.tokens_per_split;
+  const int t1 = min(n, t0 + a.tokens_per_split);
+  const float scale = rsqrtf((float)D);
+  const size_t hq0 = (size_t)unit * G;
+  const T* Q = (const T*)a.Q + hq0 * D;
+  const T* Kc = (const T*)a.Kc + (size_t)unit * a.cap * D;
+  const T* Vc = (const T*)a.Vc + (size_t)unit * a.cap * D;
+  const float* lw = a.logw + (size_t)unit * a.cap;
+  (void)b;
+  (void)kvh;
+  float q[GM][E], yv[GM][E], lse[GM], best[GM];
+#pragma unroll
+  for (int g = 0; g < GM; ++g) {
+#pragma unroll
+    for (int j = 0; j < E; ++j) {
+      q[g][j] = g < G ? to_f32(Q[(size_t)g * D + lane + 32 * j]) * scale : 0.f;
+      yv[g][j] = g < G ? a.y[(hq0 + g) * D + lane + 32 * j] : 0.f;
+    }
+    lse[g] = g < G ? a.lse[hq0 + g] : 0.f;
+    best[g] = 0.f;
+  }
+  for (int t = t0 + warp; t < t1; t += kGenWarps) {
+    const float lwt = lw[t];
+    if (!(lwt > 0.f)) continue;  // pi = 1: not in the tail sample
+    float k[E], v[E];
+#pragma unroll
+    for (int j = 0; j < E; ++j) {
+      k[j] = to_f32(Kc[(size_t)t * D + lane + 32 * j]);
+      v[j] = to_f32(Vc[(size_t)t * D + lane + 32 * j]);
+    }
+    const float sq = sqrtf(-expm1f(-lwt));
+#pragma unroll
+    for (int g = 0; g < GM; ++g) {
+      if (g >= G) break;
+      float dot = 0.f, dist = 0.f;
+#pragma unroll
+      for (int j = 0; j < E; ++j) {
+        dot = fmaf(q[g][j], k[j], dot);
+        const float dv = v[j] - yv[g][j];
+        dist = fmaf(dv, dv, dist);
+      }
+      const float x = warp_sum(dot) + lwt;
+      dist = warp_sum(dist);
+      const float p = expf(x - lse[g]);  // w_i / N_hat
+      best[g] = fmaxf(best[g], sq * p * sqrtf(dist));
+    }
+  }
+  if (lane == 0) {
+#pragma unroll
+    for (int g = 0; g < GM; ++g) smax[warp][g] = best[g];
+  }
+  __syncthreads();
+  if (threadIdx.x < G) {
+    float m = 0.f;
+#pragma unroll
+    for (int w = 0; w < kGenWarps; ++w) m = fmaxf(m, smax[w][threadIdx.x]);
+    // non-negative floats order like their bit patterns
+    atomicMax((unsigned int*)&a.b_t[hq0 + threadIdx.x], __float_as_uint(m));
+  }
+}
+
+template <int D>
+__global__ void decode_radius_kernel(ReduceArgs a, int n_heads) {
+  const int hq = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (hq >= n_heads) return;
+  float yy = 0.f;
+  for (int e = lane; e < D; e += 32) {
+    const float y = a.y[(size_t)hq * D + e];
+    yy = fmaf(y, y, yy);
+  }
+  yy = warp_sum(yy);
+  if (lane == 0) {
+    const float bt = a.b_t[hq], var = a.var[hq];
+    a.radius[hq] = (sqrtf(2.f * var * a.log_inv_delta) + bt * a.log_inv_delta) / (sqrtf(yy) + a.eps0);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+template <typename T, int D, int GM>
+static ebd_status launch_generic_t(const DecodeArgs& a, int units, cudaStream_t s) {
+  dim3 grid(a.splits, units);
+  decode_generic_kernel<T, D, GM><<<grid, kGenThreads, 0, s>>>(a);
+  return launch_status();
+}
+
+template <typename T, int D, int GM>
+static ebd_status launch_exact_t(const DecodeArgs& a, int units, cudaStream_t s) {
+  dim3 grid(a.splits, units);
+  decode_exact_range_kernel<T, D, GM><<<grid, kGenThreads, 0, s>>>(a);
+  return launch_status();
+}
+
+template <typename T, int D>
+static ebd_status dispatch_g(bool exact, const DecodeArgs& a, int units, cudaStream_t s) {
+  const int G = a.group;
+  if (G <= 1) return exact ? launch_exact_t<T, D, 1>(a, units, s) : launch_generic_t<T, D, 1>(a, units, s);
+  if (G <= 2) return exact ? launch_exact_t<T, D, 2>(a, units, s) : launch_generic_t<T, D, 2>(a, units, s);
+  if (G <= 4) return exact ? launch_exact_t<T, D, 4>(a, units, s) : launch_generic_t<T, D, 4>(a, units, s);
+  return exact ? launch_exact_t<T, D, 8>(a, units, s) : launch_generic_t<T, D, 8>(a, units, s);
+}
+
+static ebd_status dispatch_generic(bool exact, ebd_dtype dt, int D, const DecodeArgs& a, int units,
+                                   cudaStream_t s) {
+  if (dt == EBD_F32) {
+    if (D == 64) return dispatch_g<float, 64>(exact, a, units, s);
+    if (D == 128) return dispatch_g<float, 128>(exact, a, units, s);
+  } else {
+    if (D == 64) return dispatch_g<__nv_bfloat16, 64>(exact, a, units, s);
+    if (D == 128) return dispatch_g<__nv_bfloat16, 128>(exact, a, units, s);
+  }
+  return EBD_ERR_UNSUPPORTED;
+}
+
+static DecodePlan plan_generic(long long units, int group, int head_dim, int capacity) {
+  // CUDA-core path: ~8 resident CTAs per SM, at least 32 tokens per split
+  DecodePlan p;
+  const long long target = (long long)sm_count() * 8;
+  long long splits = (target + units - 1) / units;
+  const long long max_splits = (capacity + 31) / 32;
+  if (splits > max_splits) splits = max_splits;
+  if (splits < 1) splits = 1;
+  if (splits > 65535) splits = 65535;
+  p.splits = (int)splits;
+  p.tokens_per_split = (int)((capacity + splits - 1) / splits);
+  p.ws_bytes = align_up((size_t)units * p.splits * group * rec_floats(head_dim) * sizeof(float), 256);
+  return p;
+}
+
+DecodePlan plan_generic_for_exact(int batch, int n_kv_heads, int group, int head_dim,
+                                  int capacity) {
+  return plan_generic((long long)batch * n_kv_heads, group, head_dim, capacity);
+}
+
+DecodePlan plan_decode(ebd_dtype dtype, int batch, int n_kv_heads, int group, int head_dim,
+                       int capacity) {
+  const long long units = (long long)batch * n_kv_heads;
+  if (fast_decode_supported(dtype, group, head_dim, capacity)) {
+    DecodePlan p;
+    p.fast = true;
+    fast_decode_plan(p, units, group, head_dim, capacity);
+    return p;
+  }
+  return plan_generic(units, group, head_dim, capacity);
+}
+
+}  // namespace ebd
+
+using namespace ebd;
+
+extern "C" size_t ebd_decode_workspace_bytes(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads,
+                                             int32_t group, int32_t head_dim, int32_t capacity) {
+  if (batch < 1 || n_kv_heads < 1 || group < 1 || head_dim < 1 || capacity < 1) return 0;
+  return plan_decode(dtype, batch, n_kv_heads, group, head_dim, capacity).ws_bytes;
+}
+
+extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads,
+                                           int32_t group, int32_t head_dim, const void* Q,
+                                           const void* K_c, const void* V_c, const float* logw_c,
+                                           const int32_t* n_kept, int32_t capacity, float delta,
+                                           float eps0, ebd_range_mode range_mode, float* y,
+                                           float* lse, float* var_hat, float* b_t, float* radius,
+                                           int32_t* dev_status, void* workspace, size_t ws_bytes,
+                                           void* stream) {
+  if (dtype != EBD_F32 && dtype != EBD_BF16) return EBD_ERR_INVALID;
+  if (batch < 1 || n_kv_heads < 1 || group < 1 || capacity < 1) return EBD_ERR_INVALID;
+  if (!Q || !K_c || !V_c || !logw_c || !n_kept || !y || !lse || !var_hat || !b_t || !radius)
+    return EBD_ERR_INVALID;
+  if (!(delta > 0.f && delta < 1.f) || !(eps0 >= 0.f)) return EBD_ERR_INVALID;
+  if (range_mode != EBD_RANGE_BOUND && range_mode != EBD_RANGE_EXACT) return EBD_ERR_INVALID;
+  if (head_dim != 64 && head_dim != 128) return EBD_ERR_UNSUPPORTED;
+  if (group > 8) return EBD_ERR_UNSUPPORTED;
+  const long long units = (long long)batch * n_kv_heads;
+  if (units * group > 0x7fffffffLL || units > 65535) return EBD_ERR_UNSUPPORTED;
+  const DecodePlan plan = plan_decode(dtype, batch, n_kv_heads, group, head_dim, capacity);
+  if (!workspace || ws_bytes < plan.ws_bytes) return EBD_ERR_CAPACITY;
+  cudaStream_t s = (cudaStream_t)stream;
+
+  DecodeArgs a;
+  a.Q = Q;
+  a.Kc = K_c;
+  a.Vc = V_c;
+  a.logw = logw_c;
+  a.n_kept = n_kept;
+  a.cap = capacity;
+  a.n_kv_heads = n_kv_heads;
+  a.group = group;
+  a.splits = plan.splits;
+  a.tokens_per_split = plan.tokens_per_split;
+  a.part = (float*)workspace;
+  a.y = y;
+  a.lse = lse;
+  a.dev_status = dev_status;
+
+  ebd_status st;
+  if (plan.fast)
+    st = launch_fast_decode(dtype, head_dim, plan, a, (int)units, s);
+  else
+    st = dispatch_generic(false, dtype, head_dim, a, (int)units, s);
+  if (st != EBD_OK) return st;
+
+  ReduceArgs r;
+  r.part = (const float*)workspace;
+  r.splits = plan.fast ? plan.reduce_slots : plan.splits;
+  r.group = group;
+  r.y = y;
+  r.lse = lse;
+  r.var = var_hat;
+  r.b_t = b_t;
+  r.radius = radius;
+  r.log_inv_delta = logf(1.f / delta);
+  r.eps0 = eps0;
+  r.exact = range_mode == EBD_RANGE_EXACT;
+  const int n_heads = (int)(units * group);
+  if (head_dim == 128)
+    decode_reduce_kernel<128><<<n_heads, 128, 0, s>>>(r);
+  else
+    decode_reduce_kernel<64><<<n_heads, 64, 0, s>>>(r);
+  st = launch_status();
+  if (st != EBD_OK || !r.exact) return st;
+
+  // exact range term: second pass over the tail rows, then the radius
+  DecodePlan gp = plan;
+  if (plan.fast) gp = plan_generic_for_exact(batch, n_kv_heads, group, head_dim, capacity);
+  a.splits = gp.splits;
+  a.tokens_per_split = gp.tokens_per_split;
+  a.b_t = b_t;
+  st = dispatch_generic(true, dtype, head_dim, a, (int)units, s);
+  if (st != EBD_OK) return st;
+  const int warps = 4;
+  if (head_dim == 128)
+    decode_radius_kernel<128><<<(n_heads + warps - 1) / warps, warps * 32, 0, s>>>(r, n_heads);
+  else
+    decode_radius_kernel<64><<<(n_heads + warps - 1) / warps, warps * 32, 0, s>>>(r, n_heads);
+  return launch_status();
+}

@@ -1,0 +1,565 @@
+// Eviction step of eviction-by-design on GB300 (sm_103a).
+//
+// Per (batch row b, KV head kvh) unit, one CTA of 1024 threads:
+//   E1  certainty set A: protected positions (sinks, recency window) plus the
+//       top-k_head unprotected tokens by score, equal scores to the lower index
+//       (Section 3.3 and Appendix B of the paper).  Exact selection by an
+//       MSB-first 8-bit radix select over order-preserving score keys, then an
+//       ordered scan among the tokens equal to the k-th key.
+//   E2  inclusion probabilities on the tail T (Eq. 2): pi_i = clip(c s_i, eps, 1)
+//       with c solving sum_T pi_i = m (clip-saturated tokens join A), found by
+//       a fixed number of bisection steps on log c, then one exact linear solve
+//       inside the partition (clipped-high / linear / floor) the bisection ends in.
+//   E3  Poisson draw: keep_i = (u_i < pi_i) with u_i from Philox4x32-10 keyed by
+//       the seed, counter (token, kvh, layer, b).
+//   E4  stable compaction: an ordered block scan of the keep flags writes the
+//       token index and log(1/pi_i) of every kept token; a second, HBM-bound
+//       kernel then copies the kept K and V rows with 16-byte loads.
+// The certainty set lives in shared memory as a bitmask (N/8 bytes).  Scores
+// are re-read from global memory (L2-resident) by each pass.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace ebd {
+
+constexpr int kSelThreads = 1024;
+constexpr int kSelWarps = kSelThreads / 32;
+constexpr int kMaxCtx = 1 << 20;
+
+struct SelectArgs {
+  const float* scores;  // [units, N]
+  int n_ctx;
+  int n_kv_heads;
+  int layer;
+  uint64_t seed;
+  int n_sink;
+  int n_recent;
+  int k_head;
+  int budget;
+  int iters;
+  float eps;
+  float* pi_out;        // nullable [units, N]
+  uint8_t* mask_out;    // nullable [units, N]
+  int32_t* idx_c;       // nullable [units, cap] (compaction outputs all set or all null)
+  float* logw_c;        // [units, cap]
+  int32_t* n_kept;      // [units]
+  int cap;
+  int32_t* dev_status;  // nullable
+};
+
+struct BlockScratch {
+  float f[kSelWarps];
+  double d[kSelWarps];
+  int i[kSelWarps];
+};
+
+__device__ __forceinline__ float block_sum_f2d(float v, BlockScratch& sh) {
+  // per-thread float partials, combined across the block in double
+  v = warp_sum(v);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) sh.d[threadIdx.x >> 5] = (double)v;
+  __syncthreads();
+  double r = 0.0;
+#pragma unroll 8
+  for (int w = 0; w < kSelWarps; ++w) r += sh.d[w];
+  return (float)r;
+}
+__device__ __forceinline__ double block_sum_d(double v, BlockScratch& sh) {
+  v = warp_sum(v);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) sh.d[threadIdx.x >> 5] = v;
+  __syncthreads();
+  double r = 0.0;
+#pragma unroll 8
+  for (int w = 0; w < kSelWarps; ++w) r += sh.d[w];
+  return r;
+}
+__device__ __forceinline__ int block_sum_i(int v, BlockScratch& sh) {
+  v = warp_sum(v);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) sh.i[threadIdx.x >> 5] = v;
+  __syncthreads();
+  int r = 0;
+#pragma unroll 8
+  for (int w = 0; w < kSelWarps; ++w) r += sh.i[w];
+  return r;
+}
+__device__ __forceinline__ float block_max_f(float v, BlockScratch& sh) {
+  v = warp_max(v);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) sh.f[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float r = sh.f[0];
+#pragma unroll 8
+  for (int w = 1; w < kSelWarps; ++w) r = fmaxf(r, sh.f[w]);
+  return r;
+}
+__device__ __forceinline__ float block_min_f(float v, BlockScratch& sh) {
+  v = warp_min(v);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) sh.f[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float r = sh.f[0];
+#pragma unroll 8
+  for (int w = 1; w < kSelWarps; ++w) r = fminf(r, sh.f[w]);
+  return r;
+}
+
+// Ordered count: exclusive prefix of `flag` over the block in thread order and
+// the block total.  Two barriers.
+__device__ __forceinline__ int block_rank(bool flag, int& total, BlockScratch& sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const unsigned bal = __ballot_sync(0xffffffffu, flag);
+  __syncthreads();
+  if (lane == 0) sh.i[warp] = __popc(bal);
+  __syncthreads();
+  int before = 0, tot = 0;
+#pragma unroll 8
+  for (int w = 0; w < kSelWarps; ++w) {
+    const int c = sh.i[w];
+    before += (w < warp) ? c : 0;
+    tot += c;
+  }
+  total = tot;
+  return before + __popc(bal & ((1u << lane) - 1u));
+}
+
+enum PiMode : int { kPiFloor = 0, kPiAll = 1, kPiLinear = 2 };
+
+__device__ __forceinline__ float tail_pi(float s, int mode, float c, float eps) {
+  if (mode == kPiFloor) return eps;
+  if (mode == kPiAll) return s > 0.f ? 1.f : eps;
+  return fminf(1.f, fmaxf(eps, c * s));
+}
+
+__global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs a) {
+  extern __shared__ uint32_t cert_bits[];  // bit i set <=> token i in A
+  __shared__ BlockScratch sh;
+  __shared__ unsigned hist[256];
+  __shared__ unsigned sh_prefix, sh_remaining;
+  __shared__ int sh_bad;
+
+  const int unit = blockIdx.x;
+  const int b = unit / a.n_kv_heads;
+  const int kvh = unit - b * a.n_kv_heads;
+  const int N = a.n_ctx;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int words = (N + 31) >> 5;
+  const float* s = a.scores + (size_t)unit * N;
+
+  const int ns = min(a.n_sink, N);
+  const int rs = max(N - a.n_recent, 0);  // first protected trailing position
+
+  if (tid == 0) sh_bad = 0;
+  bool bad = false;
+  // protected positions
+  for (int base = 0; base < N; base += kSelThreads) {
+    const int i = base + tid;
+    const bool prot = (i < N) && (i < ns || i >= rs);
+    const unsigned bits = __ballot_sync(0xffffffffu, prot);
+    const int wd = (base >> 5) + warp;
+    if (lane == 0 && wd < words) cert_bits[wd] = bits;
+  }
+  const int n_prot = ns + (N - rs) - max(0, ns - rs);
+  const int n_cand = N - n_prot;
+  const int k = min(max(a.k_head, 0), n_cand);
+  __syncthreads();
+
+  // ---- E1: top-k among unprotected tokens ---------------------------------
+  if (k > 0 && k < n_cand) {
+    unsigned prefix = 0u, maskbits = 0u, remaining = (unsigned)k;
+    for (int shift = 24; shift >= 0; shift -= 8) {
+      for (int j = tid; j < 256; j += kSelThreads) hist[j] = 0u;
+      __syncthreads();
+      for (int i = tid; i < N; i += kSelThreads) {
+        if (i < ns || i >= rs) continue;
+        float v = __ldg(s + i);
+        if (!isfinite(v)) { bad = true; v = 0.f; }
+        const uint32_t key = orderable_key(v);
+        if ((key & maskbits) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+      }
+      __syncthreads();
+      if (warp == 0) {
+        // lane L owns bins 255-8L .. 248-8L (descending key order)
+        unsigned c[8];
+        unsigned tot = 0;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          c[q] = hist[255 - 8 * lane - q];
+          tot += c[q];
+        }
+        unsigned incl = tot;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const unsigned n = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += n;
+        }
+        const unsigned excl = incl - tot;
+        if (excl < remaining && incl >= remaining) {
+          unsigned cum = excl;
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            if (cum + c[q] >= remaining) {
+              sh_prefix = prefix | ((unsigned)(255 - 8 * lane - q) << shift);
+              sh_remaining = remaining - cum;
+              break;
+            }
+            cum += c[q];
+          }
+        }
+      }
+      __syncthreads();
+      prefix = sh_prefix;
+      remaining = sh_remaining;
+      maskbits |= 255u << shift;
+    }
+    // prefix = k-th largest key; take every key above it and the `remaining`
+    // lowest-index tokens equal to it.
+    int taken = 0;
+    for (int base = 0; base < N; base += kSelThreads) {
+      const int i = base + tid;
+      bool eq = false, gt = false;
+      if (i < N && !(i < ns || i >= rs)) {
+        float v = __ldg(s + i);
+        if (!isfinite(v)) v = 0.f;
+        const uint32_t key = orderable_key(v);
+        eq = key == prefix;
+        gt = key > prefix;
+      }
+      int total;
+      const int rank = block_rank(eq, total, sh);
+      const bool sel = gt || (eq && taken + rank < (int)remaining);
+      const unsigned bits = __ballot_sync(0xffffffffu, sel);
+      const int wd = (base >> 5) + warp;
+      if (lane == 0 && wd < words) cert_bits[wd] |= bits;
+      taken += total;
+    }
+  } else if (k > 0) {  // every unprotected token is in the top slice
+    for (int wd = tid; wd < words; wd += kSelThreads) {
+      unsigned m = 0xffffffffu;
+      if (wd == words - 1 && (N & 31)) m = (1u << (N & 31)) - 1u;
+      cert_bits[wd] = m;
+    }
+  }
+  __syncthreads();
+
+  // ---- E2: inclusion probabilities on the tail -----------------------------
+  const int n_cert = n_prot + k;
+  const int nT = N - n_cert;
+  const int m = min(max(a.budget - n_cert, 0), nT);
+  float smax = -INFINITY, sminpos = INFINITY;
+  int npos = 0;
+  for (int i = tid; i < N; i += kSelThreads) {
+    if ((cert_bits[i >> 5] >> (i & 31)) & 1u) continue;
+    float v = __ldg(s + i);
+    if (!isfinite(v)) { bad = true; v = 0.f; }
+    smax = fmaxf(smax, v);
+    if (v > 0.f) {
+      sminpos = fminf(sminpos, v);
+      ++npos;
+    }
+  }
+  smax = block_max_f(smax, sh);
+  sminpos = block_min_f(sminpos, sh);
+  npos = block_sum_i(npos, sh);
+
+  const float eps = a.eps;
+  int mode = kPiLinear;
+  float c = 0.f;
+  if (nT == 0 || (float)m <= eps * (float)nT) {
+    mode = kPiFloor;
+  } else if ((float)m >= (float)npos + eps * (float)(nT - npos)) {
+    mode = kPiAll;
+  } else {
+    float lo = logf(eps / smax), hi = logf(1.f / sminpos);
+    for (int it = 0; it < a.iters; ++it) {
+      const float mid = 0.5f * (lo + hi);
+      const float cm = expf(mid);
+      float g = 0.f;
+      for (int i = tid; i < N; i += kSelThreads) {
+        if ((cert_bits[i >> 5] >> (i & 31)) & 1u) continue;
+        float v = __ldg(s + i);
+        if (!isfinite(v)) v = 0.f;
+        g += fminf(1.f, fmaxf(eps, cm * v));
+      }
+      g = block_sum_f2d(g, sh);
+      if (g < (float)m) lo = mid; else hi = mid;
+    }
+    // exact solve inside the partition found at the upper end of the bracket
+    const float cb = expf(hi);
+    int n_hi = 0, n_lo = 0;
+    double smid = 0.0;
+    for (int i = tid; i < N; i += kSelThreads) {
+      if ((cert_bits[i >> 5] >> (i & 31)) & 1u) continue;
+      float v = __ldg(s + i);
+      if (!isfinite(v)) v = 0.f;
+      const float t = cb * v;
+      if (t >= 1.f) ++n_hi;
+      else if (t <= eps) ++n_lo;
+      else smid += (double)v;
+    }
+    n_hi = block_sum_i(n_hi, sh);
+    n_lo = block_sum_i(n_lo, sh);
+    smid = block_sum_d(smid, sh);
+    const double cstar = ((double)m - n_hi - (double)eps * n_lo) / smid;
+    const double clo = exp((double)lo), chi = exp((double)hi);
+    if (smid > 0.0 && cstar >= clo * (1.0 - 1e-6) && cstar <= chi * (1.0 + 1e-6))
+      c = (float)cstar;
+    else
+      c = expf(0.5f * (lo + hi));
+  }
+
+  // ---- E3 + E4a: draws, stable compaction of (index, log 1/pi) -------------
+  const bool compact = a.n_kept != nullptr;
+  int kept = 0;
+  for (int base = 0; base < N; base += kSelThreads) {
+    const int i = base + tid;
+    bool keep = false;
+    float pi = 1.f;
+    bool cert = false;
+    if (i < N) {
+      cert = (cert_bits[i >> 5] >> (i & 31)) & 1u;
+      if (!cert) {
+        float v = __ldg(s + i);
+        if (!isfinite(v)) { bad = true; v = 0.f; }
+        pi = tail_pi(v, mode, c, eps);
+      }
+      if (a.pi_out) a.pi_out[(size_t)unit * N + i] = pi;
+      if (a.mask_out) a.mask_out[(size_t)unit * N + i] = cert ? 1 : 0;
+      if (compact) {
+        const float u = word_to_uniform(draw_word(a.seed, a.layer, b, kvh, i));
+        keep = cert || (u < pi);
+      }
+    }
+    if (compact) {
+      int total;
+      const int rank = block_rank(keep, total, sh);
+      const int p = kept + rank;
+      if (keep && p < a.cap) {
+        a.idx_c[(size_t)unit * a.cap + p] = i;
+        a.logw_c[(size_t)unit * a.cap + p] = (cert || pi >= 1.f) ? 0.f : -logf(pi);
+      }
+      kept += total;
+    }
+  }
+  if (bad) sh_bad = 1;
+  __syncthreads();
+  if (tid == 0) {
+    if (compact) {
+      a.n_kept[unit] = kept;
+      if (kept > a.cap) raise_status(a.dev_status, EBD_DEV_CAPACITY);
+    }
+    if (sh_bad) raise_status(a.dev_status, EBD_DEV_NONFINITE);
+  }
+}
+
+// E4b: copy kept K and V rows (16-byte chunks, `cpr` chunks per row).
+constexpr int kGatherThreads = 256;
+constexpr int kGatherUnroll = 4;
+
+__global__ void __launch_bounds__(kGatherThreads) gather_rows_kernel(
+    const uint4* __restrict__ K, const uint4* __restrict__ V, uint4* __restrict__ Kc,
+    uint4* __restrict__ Vc, const int32_t* __restrict__ idx_c, const int32_t* __restrict__ n_kept,
+    int n_ctx, int cap, int cpr) {
+  const int unit = blockIdx.y;
+  const int n = min(n_kept[unit], cap);
+  const long long items = (long long)n * cpr;
+  const long long stride = (long long)gridDim.x * kGatherThreads;
+  const int32_t* idx = idx_c + (size_t)unit * cap;
+  const size_t src_base = (size_t)unit * n_ctx * cpr;
+  const size_t dst_base = (size_t)unit * cap * cpr;
+  for (long long it0 = (long long)blockIdx.x * kGatherThreads + threadIdx.x; it0 < items;
+       it0 += stride * kGatherUnroll) {
+    uint4 kv[kGatherUnroll], vv[kGatherUnroll];
+    size_t dst[kGatherUnroll];
+    bool ok[kGatherUnroll];
+#pragma unroll
+    for (int u = 0; u < kGatherUnroll; ++u) {
+      const long long it = it0 + u * stride;
+      ok[u] = it < items;
+      if (ok[u]) {
+        const int p = (int)(it / cpr);
+        const int ch = (int)(it - (long long)p * cpr);
+        const size_t src = src_base + (size_t)idx[p] * cpr + ch;
+        dst[u] = dst_base + (size_t)p * cpr + ch;
+        kv[u] = __ldg(K + src);
+        vv[u] = __ldg(V + src);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kGatherUnroll; ++u) {
+      if (ok[u]) {
+        Kc[dst[u]] = kv[u];
+        Vc[dst[u]] = vv[u];
+      }
+    }
+  }
+}
+
+__global__ void philox_words_kernel(uint64_t seed, int layer, int n_kv_heads, int n_ctx,
+                                    long long total, uint32_t* out) {
+  for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+       t += (long long)gridDim.x * blockDim.x) {
+    const long long unit = t / n_ctx;
+    const int i = (int)(t - unit * n_ctx);
+    const int b = (int)(unit / n_kv_heads);
+    const int kvh = (int)(unit - (long long)b * n_kv_heads);
+    out[t] = draw_word(seed, layer, b, kvh, i);
+  }
+}
+
+int sm_count() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (dev < 0 || dev >= 64) return 148;
+  if (!cached[dev]) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 148;
+    cached[dev] = n;
+  }
+  return cached[dev];
+}
+
+static ebd_status check_design(const ebd_design* d) {
+  if (!d) return EBD_ERR_INVALID;
+  if (d->batch < 1 || d->n_kv_heads < 1 || d->n_ctx < 1 || d->n_ctx > kMaxCtx) return EBD_ERR_INVALID;
+  if ((long long)d->batch * d->n_kv_heads > 0x7fffffffLL) return EBD_ERR_INVALID;
+  if (d->n_sink < 0 || d->n_recent < 0 || d->k_head < 0 || d->budget_tokens < 0) return EBD_ERR_INVALID;
+  if (d->bisect_iters < 1 || d->bisect_iters > 200) return EBD_ERR_INVALID;
+  if (!(d->eps > 0.f && d->eps <= 1.f)) return EBD_ERR_INVALID;
+  return EBD_OK;
+}
+
+static ebd_status launch_select(const ebd_design* d, const float* scores, float* pi,
+                                uint8_t* mask, int32_t* idx_c, float* logw_c, int32_t* n_kept,
+                                int cap, int32_t* dev_status, cudaStream_t stream) {
+  SelectArgs a;
+  a.scores = scores;
+  a.n_ctx = d->n_ctx;
+  a.n_kv_heads = d->n_kv_heads;
+  a.layer = d->layer;
+  a.seed = d->seed;
+  a.n_sink = d->n_sink;
+  a.n_recent = d->n_recent;
+  a.k_head = d->k_head;
+  a.budget = d->budget_tokens;
+  a.iters = d->bisect_iters;
+  a.eps = d->eps;
+  a.pi_out = pi;
+  a.mask_out = mask;
+  a.idx_c = idx_c;
+  a.logw_c = logw_c;
+  a.n_kept = n_kept;
+  a.cap = cap;
+  a.dev_status = dev_status;
+  const size_t smem = (size_t)((d->n_ctx + 31) / 32) * 4;
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(evict_select_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return EBD_ERR_CUDA;
+  }
+  const int units = d->batch * d->n_kv_heads;
+  evict_select_kernel<<<units, kSelThreads, smem, stream>>>(a);
+  return launch_status();
+}
+
+static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+}  // namespace ebd
+
+using namespace ebd;
+
+extern "C" const char* ebd_status_string(ebd_status s) {
+  switch (s) {
+    case EBD_OK: return "EBD_OK";
+    case EBD_ERR_INVALID: return "EBD_ERR_INVALID: invalid argument";
+    case EBD_ERR_CAPACITY: return "EBD_ERR_CAPACITY: capacity or workspace too small";
+    case EBD_ERR_NONFINITE: return "EBD_ERR_NONFINITE: non-finite input";
+    case EBD_ERR_UNSUPPORTED: return "EBD_ERR_UNSUPPORTED: not supported by this build";
+    case EBD_ERR_CUDA: return "EBD_ERR_CUDA: CUDA runtime error";
+  }
+  return "EBD_ERR_UNKNOWN";
+}
+
+extern "C" int32_t ebd_abi_version(void) { return 1; }
+
+extern "C" ebd_status ebd_philox_uniforms(uint64_t seed, int32_t layer, int32_t batch,
+                                          int32_t n_kv_heads, int32_t n_ctx, uint32_t* x0,
+                                          void* stream) {
+  if (!x0 || batch < 1 || n_kv_heads < 1 || n_ctx < 1) return EBD_ERR_INVALID;
+  const long long total = (long long)batch * n_kv_heads * n_ctx;
+  const int threads = 256;
+  long long blocks = (total + threads - 1) / threads;
+  if (blocks > (long long)sm_count() * 64) blocks = (long long)sm_count() * 64;
+  philox_words_kernel<<<(unsigned)blocks, threads, 0, (cudaStream_t)stream>>>(
+      seed, layer, n_kv_heads, n_ctx, total, x0);
+  return launch_status();
+}
+
+extern "C" ebd_status ebd_compute_pi(const ebd_design* design, const float* scores, float* pi,
+                                     uint8_t* certain_mask, int32_t* dev_status, void* stream) {
+  ebd_status st = check_design(design);
+  if (st != EBD_OK) return st;
+  if (!scores || !pi) return EBD_ERR_INVALID;
+  return launch_select(design, scores, pi, certain_mask, nullptr, nullptr, nullptr, 0,
+                       dev_status, (cudaStream_t)stream);
+}
+
+extern "C" size_t ebd_evict_workspace_bytes(const ebd_design* design, int32_t n_obs) {
+  if (!design || n_obs <= 0) return 0;
+  const size_t units = (size_t)design->batch * design->n_kv_heads;
+  return align_up(units * design->n_ctx * sizeof(float), 256) +
+         align_up(units * (size_t)n_obs * sizeof(float), 256);
+}
+
+extern "C" ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const void* K,
+                                const void* V, const float* scores, const void* q_obs,
+                                int32_t n_obs, void* K_c, void* V_c, float* logw_c,
+                                int32_t* idx_c, int32_t* n_kept, int32_t capacity,
+                                int32_t* dev_status, void* workspace, size_t ws_bytes,
+                                void* stream) {
+  ebd_status st = check_design(design);
+  if (st != EBD_OK) return st;
+  if (dtype != EBD_F32 && dtype != EBD_BF16) return EBD_ERR_INVALID;
+  if (!K || !V || !K_c || !V_c || !logw_c || !idx_c || !n_kept || !dev_status) return EBD_ERR_INVALID;
+  if (capacity < 1) return EBD_ERR_INVALID;
+  const int d = design->head_dim;
+  const int eb = dtype == EBD_F32 ? 4 : 2;
+  if (d < 1 || (d * eb) % 16 != 0) return EBD_ERR_UNSUPPORTED;
+  if (!aligned16(K) || !aligned16(V) || !aligned16(K_c) || !aligned16(V_c)) return EBD_ERR_INVALID;
+  cudaStream_t s = (cudaStream_t)stream;
+  const float* sc = scores;
+  if (!sc) {
+    if (!q_obs || n_obs < 1) return EBD_ERR_INVALID;
+    const size_t need = ebd_evict_workspace_bytes(design, n_obs);
+    if (!workspace || ws_bytes < need) return EBD_ERR_CAPACITY;
+    const size_t units = (size_t)design->batch * design->n_kv_heads;
+    float* ws_scores = (float*)workspace;
+    float* ws_lse = (float*)((char*)workspace + align_up(units * design->n_ctx * sizeof(float), 256));
+    st = launch_score(dtype, design->batch, design->n_kv_heads, d, design->n_ctx, n_obs, q_obs, K,
+                      ws_scores, ws_lse, s);
+    if (st != EBD_OK) return st;
+    sc = ws_scores;
+  }
+  st = launch_select(design, sc, nullptr, nullptr, idx_c, logw_c, n_kept, capacity, dev_status, s);
+  if (st != EBD_OK) return st;
+  const int cpr = d * eb / 16;
+  const int units = design->batch * design->n_kv_heads;
+  const long long items = (long long)capacity * cpr;
+  long long bx = (items + (long long)kGatherThreads * kGatherUnroll - 1) /
+                 ((long long)kGatherThreads * kGatherUnroll);
+  if (bx < 1) bx = 1;
+  if (bx > 65535) bx = 65535;
+  if (units > 65535) return EBD_ERR_UNSUPPORTED;
+  dim3 grid((unsigned)bx, (unsigned)units);
+  gather_rows_kernel<<<grid, kGatherThreads, 0, s>>>((const uint4*)K, (const uint4*)V, (uint4*)K_c,
+                                                     (uint4*)V_c, idx_c, n_kept, design->n_ctx,
+                                                     capacity, cpr);
+  return launch_status();
+}

@@ -1,0 +1,28 @@
+// Host-side declarations shared by the translation units of libebd.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/ebd.h"
+
+namespace ebd {
+
+inline ebd_status cuda_status(cudaError_t e) { return e == cudaSuccess ? EBD_OK : EBD_ERR_CUDA; }
+
+// Last launch error of this thread, mapped to a status (clears the error).
+inline ebd_status launch_status() { return cuda_status(cudaGetLastError()); }
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Number of SMs of the current device (cached per device).
+int sm_count();
+
+// E0: accumulated attention scores into `scores` using `workspace` for the
+// per-row log-sum-exp.  Arguments validated by the caller.
+ebd_status launch_score(ebd_dtype dtype, int batch, int n_kv_heads, int head_dim, int n_ctx,
+                        int n_obs, const void* q_obs, const void* K, float* scores,
+                        float* lse_ws, cudaStream_t stream);
+
+}  // namespace ebd
