@@ -1,0 +1,527 @@
+#!/usr/bin/env python
+"""Benchmark of the eviction-by-design hot path on one or more GB300s.
+
+One step = one pass of the whole path over one batch: (scoring, for the
+attention-scored workload) -> select (certainty set, pi, Poisson draw, index
+compaction) -> gather (kept K/V rows) -> certified decode, for every layer of
+the workload.  Each phase runs every layer back to back (a CUDA graph when
+there is more than one layer) between two CUDA events on the launching
+stream; L2 is flushed (256 MB write) before every phase, outside the events.
+
+Prints ONE JSON line (rank 0).  `value` is the certified decode-step HBM
+throughput in GB/s: algorithmic bytes (compact K/V rows, one log(1/pi) per
+row, queries and outputs) over the decode phase's device time, summed over
+ranks and divided by the slowest rank's time.
+
+  --impl reference   times the float64 CPU oracle on a bounded sample of the
+                     same workload instead (rank 0 only).
+"""
+from __future__ import annotations
+
+import os
+
+# The oracle legs are timed on one host core; set before numpy is imported.
+for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, "1")
+
+import argparse  # noqa: E402
+import hashlib  # noqa: E402
+import json  # noqa: E402
+import statistics  # noqa: E402
+import subprocess  # noqa: E402
+import sys  # noqa: E402
+import tempfile  # noqa: E402
+import time  # noqa: E402
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2607_21475_gb300.workloads import WORKLOADS, Workload, make_layer_inputs  # noqa: E402
+
+METRIC = "certified decode-step HBM GB/s (% of GB300 peak) and eviction Mtokens/s"
+NORTH_STAR_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+L2_FLUSH_BYTES = 256 << 20
+
+
+# ----------------------------------------------------------------------------- utils
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="dialogue_32k", choices=sorted(WORKLOADS))
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=12.0)
+    p.add_argument("--no-graph", action="store_true")
+    return p.parse_args()
+
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1 and args.impl == "ours":
+        torch.cuda.set_device(local)
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            pk = json.load(f)
+        return float(pk["hbm_gbs"]), "measured", pk
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback", {}
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, local_rank):
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        self.gpu = vis.split(",")[local_rank] if vis else str(local_rank)
+        self.proc = None
+        self.file = None
+
+    def start(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", self.gpu, f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.file, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.file.flush()
+        self.file.seek(0)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.file.read().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        self.file.close()
+        os.unlink(self.file.name)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def source_sha(relpath):
+    with open(os.path.join(ROOT, relpath), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def traffic_for(kernel, workload):
+    """DRAM bytes per launch from a committed ncu capture, if its kernel source
+    is unchanged since the capture (else null)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            entries = json.load(f)
+    except (OSError, ValueError):
+        return None
+    for e in entries:
+        if e.get("kernel") == kernel and e.get("workload") == workload:
+            if e.get("source_sha") == source_sha(e["source"]):
+                return float(e["dram_bytes_per_launch"])
+    return None
+
+
+# ------------------------------------------------------------------ algorithmic bytes
+def decode_bytes(w: Workload, n_kept_layers):
+    """Compact K/V rows + one float32 log(1/pi) per row, the queries and the outputs."""
+    e = w.elem_bytes
+    d = w.head_dim
+    Hq = w.n_q_heads
+    tot = 0
+    for nk in n_kept_layers:
+        tot += int(nk.sum()) * (2 * d * e + 4)
+        tot += w.batch * Hq * d * e          # Q
+        tot += w.batch * Hq * (d + 4) * 4    # y, lse, var, b, radius
+    return tot
+
+
+def gather_bytes(w: Workload, n_kept_layers):
+    e, d = w.elem_bytes, w.head_dim
+    return sum(int(nk.sum()) * (4 * d * e + 4) for nk in n_kept_layers)  # read + write, idx
+
+
+def select_bytes(w: Workload, n_kept_layers):
+    units = w.batch * w.n_kv_heads
+    return sum(units * w.n_ctx * 4 + int(nk.sum()) * 8 + units * 4 for nk in n_kept_layers)
+
+
+def score_flops(w: Workload):
+    units = w.batch * w.n_kv_heads
+    return w.n_layers * units * 2 * (2 * w.n_obs * w.group * w.n_ctx * w.head_dim)
+
+
+# ------------------------------------------------------------------------- our path
+class Path:
+    """All device buffers of one rank's workload, plus one callable per phase."""
+
+    def __init__(self, w: Workload, dev, use_graph: bool):
+        from paper_2607_21475_gb300 import ebd
+        self.ebd = ebd
+        self.w = w
+        self.dev = dev
+        L, B, H, N, d, G = w.n_layers, w.batch, w.n_kv_heads, w.n_ctx, w.head_dim, w.group
+        self.inputs = [make_layer_inputs(w, l, dev) for l in range(L)]
+        self.designs = [ebd.design_for(batch=B, n_kv_heads=H, group=G, head_dim=d, n_ctx=N,
+                                       layer=l, seed=w.philox_seed, n_sink=w.n_sink,
+                                       n_recent=w.n_recent, k_head=w.k_head,
+                                       budget_tokens=w.budget_tokens,
+                                       bisect_iters=w.bisect_iters, eps=w.eps)
+                        for l in range(L)]
+        self.cc = [ebd.alloc_compact(B, H, w.capacity, d, w.torch_dtype, dev) for _ in range(L)]
+        self.scored = w.score_kind == "attention"
+        if self.scored:
+            self.scores = [torch.empty((B, H, N), dtype=torch.float32, device=dev) for _ in range(L)]
+            self.score_ws = torch.empty(ebd.ebd_score_workspace_bytes(B, H, w.n_obs * G),
+                                        dtype=torch.uint8, device=dev)
+        else:
+            self.scores = [inp["scores"] for inp in self.inputs]
+        Hq = w.n_q_heads
+        self.out = [dict(y=torch.empty((B, Hq, d), dtype=torch.float32, device=dev),
+                         **{k: torch.empty((B, Hq), dtype=torch.float32, device=dev)
+                            for k in ("lse", "var", "b", "r")}) for _ in range(L)]
+        dt = ebd.EBD_BF16 if w.dtype == "bf16" else ebd.EBD_F32
+        self.dec_ws = torch.empty(max(1, ebd.ebd_decode_workspace_bytes(dt, B, H, G, d, w.capacity)),
+                                  dtype=torch.uint8, device=dev)
+        self.phases = (["score"] if self.scored else []) + ["select", "gather", "decode"]
+        self.launches = {"score": 2, "select": 1, "gather": 1, "decode": 2}
+        self.use_graph = use_graph and L > 1
+        self.graphs = {}
+
+    # one phase over every layer
+    def _run(self, phase):
+        ebd, w = self.ebd, self.w
+        for l in range(w.n_layers):
+            inp, cc, o = self.inputs[l], self.cc[l], self.out[l]
+            if phase == "score":
+                ebd.ebd_score(inp["q_obs"], inp["K"], self.scores[l], workspace=self.score_ws)
+            elif phase == "select":
+                ebd.ebd_select(self.designs[l], self.scores[l], cc)
+            elif phase == "gather":
+                ebd.ebd_gather(self.designs[l], inp["K"], inp["V"], cc)
+            else:
+                ebd.ebd_certified_decode(inp["Q"], cc.K_c, cc.V_c, cc.logw_c, cc.n_kept, o["y"],
+                                         o["lse"], o["var"], o["b"], o["r"],
+                                         workspace=self.dec_ws)
+
+    def capture(self):
+        if not self.use_graph:
+            return
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            for ph in self.phases:
+                self._run(ph)
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        for ph in self.phases:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                self._run(ph)
+            self.graphs[ph] = g
+        torch.cuda.synchronize()
+
+    def run(self, phase):
+        if phase in self.graphs:
+            self.graphs[phase].replay()
+        else:
+            self._run(phase)
+
+    def status(self):
+        return [int(cc.dev_status.item()) for cc in self.cc]
+
+    def n_kept(self):
+        return [torch.clamp(cc.n_kept, max=self.w.capacity).cpu().numpy() for cc in self.cc]
+
+
+def e2e_run(path: Path, steps: int):
+    """Public-API end to end: pinned host inputs -> H2D -> ebd_evict + ebd_certified_decode
+    for every layer -> D2H of the outputs, all inside the timed region."""
+    ebd, w, dev = path.ebd, path.w, path.dev
+    keys = ["K", "V", "Q"] + (["q_obs"] if path.scored else ["scores"])
+    host_in = [{k: inp[k].cpu().pin_memory() for k in keys} for inp in path.inputs]
+    host_out = [{k: v.cpu().pin_memory() for k, v in o.items()} for o in path.out]
+    h2d = sum(t.numel() * t.element_size() for hi in host_in for t in hi.values())
+    d2h = sum(t.numel() * t.element_size() for ho in host_out for t in ho.values())
+    ev_ws = None
+    if path.scored:
+        ev_ws = torch.empty(ebd.ebd_evict_workspace_bytes(path.designs[0], w.n_obs * w.group),
+                            dtype=torch.uint8, device=dev)
+
+    def one():
+        for l in range(w.n_layers):
+            inp, hi = path.inputs[l], host_in[l]
+            for k in keys:
+                inp[k].copy_(hi[k], non_blocking=True)
+            cc, o = path.cc[l], path.out[l]
+            ebd.ebd_evict(path.designs[l], inp["K"], inp["V"],
+                          None if path.scored else inp["scores"],
+                          inp["q_obs"] if path.scored else None, cc, workspace=ev_ws)
+            ebd.ebd_certified_decode(inp["Q"], cc.K_c, cc.V_c, cc.logw_c, cc.n_kept, o["y"],
+                                     o["lse"], o["var"], o["b"], o["r"], workspace=path.dec_ws)
+            for k, t in o.items():
+                host_out[l][k].copy_(t, non_blocking=True)
+
+    one()
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(steps):
+        one()
+    t1.record()
+    torch.cuda.synchronize()
+    return t0.elapsed_time(t1) / steps, h2d, d2h
+
+
+# --------------------------------------------------------------------------- oracle
+def oracle_sample(w: Workload, inputs, seconds: float, max_units=None):
+    """Run the float64 oracle on units of layer 0 until `seconds` of CPU time.
+    Returns (units, evict_s, decode_s, decode_bytes)."""
+    from oracle import ebd_oracle as O
+    B, H, G, d = w.batch, w.n_kv_heads, w.group, w.head_dim
+    units = 0
+    t_ev = t_dec = 0.0
+    dbytes = 0
+    total_units = B * H if max_units is None else min(max_units, B * H)
+    for u in range(total_units):
+        b, h = divmod(u, H)
+        K = inputs["K"][b, h].double().cpu().numpy()
+        V = inputs["V"][b, h].double().cpu().numpy()
+        Q = inputs["Q"][b, h * G:(h + 1) * G].double().cpu().numpy()
+        if w.score_kind == "attention":
+            qo = inputs["q_obs"][b, h].double().cpu().numpy()
+            t = time.perf_counter()
+            s = O.accumulated_attention_scores(qo, K).astype(np.float32)
+            t_ev += time.perf_counter() - t
+        else:
+            s = inputs["scores"][b, h].cpu().numpy()
+        t = time.perf_counter()
+        r = O.evict_unit(K, V, s, n_sink=w.n_sink, n_recent=w.n_recent, k_head=w.k_head,
+                         budget_tokens=w.budget_tokens, eps=w.eps, seed=w.philox_seed, layer=0,
+                         b=b, kvh=h, capacity=w.capacity)
+        t_ev += time.perf_counter() - t
+        t = time.perf_counter()
+        O.hajek_decode(Q, r.K_c, r.V_c, r.logw)
+        t_dec += time.perf_counter() - t
+        n = min(r.n_kept, w.capacity)
+        dbytes += n * (2 * d * w.elem_bytes + 4) + G * d * w.elem_bytes + G * (d + 4) * 4
+        units += 1
+        if t_ev + t_dec >= seconds:
+            break
+    return units, t_ev, t_dec, dbytes
+
+
+def config_of(w: Workload):
+    return {"workload": w.name, "layers": w.n_layers, "batch": w.batch, "n_ctx": w.n_ctx,
+            "q_heads": w.n_q_heads, "kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
+            "kv_dtype": w.dtype, "budget": w.budget, "budget_tokens": w.budget_tokens,
+            "k_head": w.k_head, "capacity": w.capacity, "scores": w.score_kind,
+            "l2": "flushed (256 MiB write) before every timed phase; inputs > L2"}
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return
+    w = WORKLOADS[args.workload]
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    inputs = make_layer_inputs(w, 0, dev)
+    per_step = max(2.0, 150.0 / max(1, args.steps + args.warmup))
+    vals, times = [], []
+    units = 0
+    for i in range(args.warmup + args.steps):
+        t = time.perf_counter()
+        u, t_ev, t_dec, db = oracle_sample(w, inputs, per_step)
+        dt = time.perf_counter() - t
+        if i >= args.warmup:
+            vals.append(db / t_dec / 1e9)
+            times.append(dt * 1e3)
+            units = u
+    v = statistics.mean(vals)
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": v, "unit": "GB/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": statistics.mean(times),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": config_of(w),
+        "cpu_baseline": {"value": v, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{units} of {w.batch * w.n_kv_heads} (batch row, kv head) "
+                                   f"units of layer 0 per step: eviction + certified decode"},
+        "e2e": {"value": v, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def run_ours(args, world, rank, local):
+    w = WORKLOADS[args.workload]
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    hbm_peak, peak_kind, peaks = measured_peaks()
+    path = Path(w, dev, use_graph=not args.no_graph)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+
+    for ph in path.phases:       # first eager pass (also sets kernel attributes)
+        path.run(ph)
+    torch.cuda.synchronize()
+    path.capture()
+    for _ in range(args.warmup):
+        for ph in path.phases:
+            flush.fill_(1.0)
+            path.run(ph)
+    torch.cuda.synchronize()
+    st = path.status()
+    if any(st):
+        raise RuntimeError(f"device status flags raised during warm-up: {st}")
+    n_kept = path.n_kept()
+
+    ev = {ph: [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)] for ph in path.phases}
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    for i in range(args.steps):
+        for ph in path.phases:
+            flush.fill_(float(i))
+            a, b = ev[ph][i]
+            a.record()
+            path.run(ph)
+            b.record()
+    torch.cuda.synchronize()
+    barrier(world)
+    clk = clocks.stop()
+    ph_ms = {ph: statistics.mean(a.elapsed_time(b) for a, b in ev[ph]) for ph in path.phases}
+    ph_ms = {ph: max_over_ranks(v, world) for ph, v in ph_ms.items()}
+    ms_step = sum(ph_ms.values())
+
+    L = w.n_layers
+    dbytes = decode_bytes(w, n_kept)
+    value = world * dbytes / (ph_ms["decode"] * 1e-3) / 1e9
+    evict_ms = sum(ph_ms[p] for p in path.phases if p != "decode")
+    evict_mtok = world * w.batch * w.n_ctx * L / (evict_ms * 1e-3) / 1e6
+    kern = {
+        "select": {"ms_per_launch": ph_ms["select"] / L,
+                   "alg_bytes_per_launch": select_bytes(w, n_kept) / L},
+        "gather": {"ms_per_launch": ph_ms["gather"] / L,
+                   "alg_bytes_per_launch": gather_bytes(w, n_kept) / L},
+        "decode": {"ms_per_launch": ph_ms["decode"] / L, "alg_bytes_per_launch": dbytes / L},
+    }
+    if path.scored:
+        kern["score"] = {"ms_per_launch": ph_ms["score"] / L,
+                         "alg_flops_per_launch": score_flops(w) / L}
+    for k, v in kern.items():
+        if "alg_bytes_per_launch" in v:
+            v["gbs"] = v["alg_bytes_per_launch"] / (v["ms_per_launch"] * 1e-3) / 1e9
+    dom = max(kern, key=lambda k: kern[k]["ms_per_launch"])
+    kname = {"select": "evict_select_kernel", "gather": "gather_rows_kernel",
+             "decode": "certified decode (split kernel + reduce)", "score": "score kernels"}[dom]
+    if dom == "score":
+        sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+        alu_peak = torch.cuda.get_device_properties(dev).multi_processor_count * 128 * 2 * sm_max * 1e6 / 1e12
+        ach = kern[dom]["alg_flops_per_launch"] / (kern[dom]["ms_per_launch"] * 1e-3) / 1e12
+        roof = {"bound": "alu", "achieved": ach, "peak": alu_peak, "unit": "TFLOP/s",
+                "frac": ach / alu_peak, "traffic": None, "kernel": kname,
+                "peak_source": "fp32 FMA: SMs x 128 lanes x 2 x max SM clock"}
+    else:
+        ach = kern[dom]["gbs"]
+        roof = {"bound": "hbm", "achieved": ach, "peak": hbm_peak, "unit": "GB/s",
+                "frac": ach / hbm_peak, "traffic": traffic_for(dom, w.name), "kernel": kname,
+                "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"}
+
+    e2e = None
+    if not args.no_e2e:
+        e2e_ms, h2d, d2h = e2e_run(path, args.steps)
+        e2e_ms = max_over_ranks(e2e_ms, world)
+        e2e = {"value": world * dbytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        u, t_ev, t_dec, db = oracle_sample(w, path.inputs[0], args.cpu_seconds)
+        cpu = {"value": db / t_dec / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+               "sample": f"{u} of {w.batch * w.n_kv_heads} (batch row, kv head) units of "
+                         f"layer 0: eviction + certified decode ({t_ev + t_dec:.1f} s)",
+               "evict_mtok_s": u * w.n_ctx / t_ev / 1e6}
+
+    launches = args.steps * sum(path.launches[p] * L for p in path.phases)
+    line = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+        "data": "synthetic (seeded torch generators; shapes of the paper's GQA decode workloads)",
+        "config": config_of(w),
+        "decode_pct_of_8tbs": 100.0 * value / world / NORTH_STAR_HBM_GBS,
+        "decode_pct_of_measured_hbm": 100.0 * value / world / hbm_peak,
+        "evict_mtok_s": evict_mtok,
+        "phases_ms": ph_ms, "kernels": kern,
+        "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+        "clocks": clk,
+    }
+    if rank == 0:
+        print(json.dumps(line))
+
+
+def main():
+    args = parse_args()
+    world, rank, local = dist_setup(args)
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+    else:
+        run_ours(args, world, rank, local)
+    if world > 1 and args.impl == "ours":
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -138,7 +138,7 @@ ebd_status ebd_compute_pi(const ebd_design* design, const float* scores, float* 
  *             as by ebd_score
  *   K_c, V_c  device [B,Hkv,cap,d] (dtype) out: kept rows in increasing token order
  *   logw_c    device [B,Hkv,cap] float32 out: log(1/pi_i) of each kept row (0 on A)
- *   idx_c     device [B,Hkv,cap] int32 out, nullable: token index of each kept row
+ *   idx_c     device [B,Hkv,cap] int32 out: token index of each kept row
  *   n_kept    device [B,Hkv] int32 out: number of kept tokens (may exceed cap, in
  *             which case EBD_DEV_CAPACITY is raised and rows >= cap are dropped)
  *   dev_status device int32, required
@@ -150,6 +150,31 @@ ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const void* K, c
                      const float* scores, const void* q_obs, int32_t n_obs, void* K_c, void* V_c,
                      float* logw_c, int32_t* idx_c, int32_t* n_kept, int32_t capacity,
                      int32_t* dev_status, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * The two halves of ebd_evict, for callers that keep their own cache layout
+ * (and for per-kernel timing).  ebd_evict(scores given) == ebd_select then
+ * ebd_gather on the same stream.
+ *
+ * ebd_select: certainty set, Eq. (2) probabilities, Poisson draw and the
+ * stable compaction of indices (Section 3.3, Appendix B) -- everything but
+ * the row copy.
+ *   scores  device [B,Hkv,N] float32
+ *   idx_c   device [B,Hkv,cap] int32 out: kept token indices, increasing
+ *   logw_c  device [B,Hkv,cap] float32 out: log(1/pi) of each kept token
+ *   n_kept  device [B,Hkv] int32 out (may exceed cap: EBD_DEV_CAPACITY)
+ *   dev_status device int32, required
+ *
+ * ebd_gather: copies rows K[idx_c[p]], V[idx_c[p]] to K_c[p], V_c[p] for
+ * p < min(n_kept, cap) of every unit (16-byte loads; d * elem must be a
+ * multiple of 16 bytes and the four tensors 16-byte aligned).
+ */
+ebd_status ebd_select(const ebd_design* design, const float* scores, int32_t* idx_c,
+                      float* logw_c, int32_t* n_kept, int32_t capacity, int32_t* dev_status,
+                      void* stream);
+ebd_status ebd_gather(const ebd_design* design, ebd_dtype dtype, const void* K, const void* V,
+                      const int32_t* idx_c, const int32_t* n_kept, int32_t capacity, void* K_c,
+                      void* V_c, void* stream);
 
 /*
  * Certified decode step (Eq. 3, Theorem 2, Eq. 4) for every query head.

@@ -471,6 +471,25 @@ static ebd_status launch_select(const ebd_design* d, const float* scores, float*
 
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
+static ebd_status launch_gather(const ebd_design* d, ebd_dtype dtype, const void* K,
+                                const void* V, const int32_t* idx_c, const int32_t* n_kept,
+                                int cap, void* K_c, void* V_c, cudaStream_t s) {
+  const int eb = dtype == EBD_F32 ? 4 : 2;
+  const int cpr = d->head_dim * eb / 16;
+  const int units = d->batch * d->n_kv_heads;
+  if (units > 65535) return EBD_ERR_UNSUPPORTED;
+  const long long items = (long long)cap * cpr;
+  long long bx = (items + (long long)kGatherThreads * kGatherUnroll - 1) /
+                 ((long long)kGatherThreads * kGatherUnroll);
+  if (bx < 1) bx = 1;
+  if (bx > 65535) bx = 65535;
+  dim3 grid((unsigned)bx, (unsigned)units);
+  gather_rows_kernel<<<grid, kGatherThreads, 0, s>>>((const uint4*)K, (const uint4*)V,
+                                                     (uint4*)K_c, (uint4*)V_c, idx_c, n_kept,
+                                                     d->n_ctx, cap, cpr);
+  return launch_status();
+}
+
 }  // namespace ebd
 
 using namespace ebd;
@@ -549,17 +568,29 @@ extern "C" ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const
   }
   st = launch_select(design, sc, nullptr, nullptr, idx_c, logw_c, n_kept, capacity, dev_status, s);
   if (st != EBD_OK) return st;
-  const int cpr = d * eb / 16;
-  const int units = design->batch * design->n_kv_heads;
-  const long long items = (long long)capacity * cpr;
-  long long bx = (items + (long long)kGatherThreads * kGatherUnroll - 1) /
-                 ((long long)kGatherThreads * kGatherUnroll);
-  if (bx < 1) bx = 1;
-  if (bx > 65535) bx = 65535;
-  if (units > 65535) return EBD_ERR_UNSUPPORTED;
-  dim3 grid((unsigned)bx, (unsigned)units);
-  gather_rows_kernel<<<grid, kGatherThreads, 0, s>>>((const uint4*)K, (const uint4*)V, (uint4*)K_c,
-                                                     (uint4*)V_c, idx_c, n_kept, design->n_ctx,
-                                                     capacity, cpr);
-  return launch_status();
+  return launch_gather(design, dtype, K, V, idx_c, n_kept, capacity, K_c, V_c, s);
+}
+
+extern "C" ebd_status ebd_select(const ebd_design* design, const float* scores, int32_t* idx_c,
+                                 float* logw_c, int32_t* n_kept, int32_t capacity,
+                                 int32_t* dev_status, void* stream) {
+  ebd_status st = check_design(design);
+  if (st != EBD_OK) return st;
+  if (!scores || !idx_c || !logw_c || !n_kept || !dev_status || capacity < 1) return EBD_ERR_INVALID;
+  return launch_select(design, scores, nullptr, nullptr, idx_c, logw_c, n_kept, capacity,
+                       dev_status, (cudaStream_t)stream);
+}
+
+extern "C" ebd_status ebd_gather(const ebd_design* design, ebd_dtype dtype, const void* K,
+                                 const void* V, const int32_t* idx_c, const int32_t* n_kept,
+                                 int32_t capacity, void* K_c, void* V_c, void* stream) {
+  ebd_status st = check_design(design);
+  if (st != EBD_OK) return st;
+  if (dtype != EBD_F32 && dtype != EBD_BF16) return EBD_ERR_INVALID;
+  if (!K || !V || !idx_c || !n_kept || !K_c || !V_c || capacity < 1) return EBD_ERR_INVALID;
+  const int eb = dtype == EBD_F32 ? 4 : 2;
+  if (design->head_dim < 1 || (design->head_dim * eb) % 16 != 0) return EBD_ERR_UNSUPPORTED;
+  if (!aligned16(K) || !aligned16(V) || !aligned16(K_c) || !aligned16(V_c)) return EBD_ERR_INVALID;
+  return launch_gather(design, dtype, K, V, idx_c, n_kept, capacity, K_c, V_c,
+                       (cudaStream_t)stream);
 }

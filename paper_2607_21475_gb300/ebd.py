@@ -23,8 +23,9 @@ __all__ = [
     "EbdError", "EbdDesign", "EBD_F32", "EBD_BF16", "EBD_RANGE_BOUND", "EBD_RANGE_EXACT",
     "EBD_DEV_CAPACITY", "EBD_DEV_NONFINITE", "EBD_DEV_TIMEOUT", "lib", "lib_path",
     "ebd_status_string", "ebd_abi_version", "ebd_philox_uniforms", "ebd_score_workspace_bytes",
-    "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict",
-    "ebd_decode_workspace_bytes", "ebd_certified_decode", "design_for", "CompactCache",
+    "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
+    "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode", "design_for",
+    "CompactCache",
     "alloc_compact", "ABI_FUNCTIONS",
 ]
 
@@ -36,8 +37,8 @@ EBD_DEV_CAPACITY, EBD_DEV_NONFINITE, EBD_DEV_TIMEOUT = 0x1, 0x2, 0x4
 # Every symbol include/ebd.h declares.
 ABI_FUNCTIONS = (
     "ebd_status_string", "ebd_abi_version", "ebd_philox_uniforms", "ebd_score_workspace_bytes",
-    "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict",
-    "ebd_decode_workspace_bytes", "ebd_certified_decode",
+    "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
+    "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
 )
 
 
@@ -88,6 +89,10 @@ def lib():
             "ebd_evict": (ctypes.c_int, [P, ctypes.c_int, c_void_p, c_void_p, c_void_p, c_void_p,
                                          i32, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, i32,
                                          c_void_p, c_void_p, sz, c_void_p]),
+            "ebd_select": (ctypes.c_int, [P, c_void_p, c_void_p, c_void_p, c_void_p, i32, c_void_p,
+                                          c_void_p]),
+            "ebd_gather": (ctypes.c_int, [P, ctypes.c_int, c_void_p, c_void_p, c_void_p, c_void_p,
+                                          i32, c_void_p, c_void_p, c_void_p]),
             "ebd_decode_workspace_bytes": (sz, [ctypes.c_int, i32, i32, i32, i32, i32]),
             "ebd_certified_decode": (ctypes.c_int, [ctypes.c_int, i32, i32, i32, i32, c_void_p,
                                                     c_void_p, c_void_p, c_void_p, c_void_p, i32,
@@ -248,6 +253,33 @@ def ebd_evict(design: EbdDesign, K: torch.Tensor, V: torch.Tensor, scores, q_obs
         _ptr(out.idx_c, torch.int32, (B, H, cap), "idx_c"),
         _ptr(out.n_kept, torch.int32, (B, H), "n_kept"), cap,
         _ptr(out.dev_status, torch.int32, (1,), "dev_status"), ws, wsb, _stream(stream)))
+    return out
+
+
+def ebd_select(design: EbdDesign, scores: torch.Tensor, out: CompactCache, stream=None):
+    """Certainty set, pi, Poisson draw and index compaction (no row copy)."""
+    B, H, N = design.batch, design.n_kv_heads, design.n_ctx
+    cap = out.capacity
+    _check("ebd_select", lib().ebd_select(
+        ctypes.byref(design), _ptr(scores, torch.float32, (B, H, N), "scores"),
+        _ptr(out.idx_c, torch.int32, (B, H, cap), "idx_c"),
+        _ptr(out.logw_c, torch.float32, (B, H, cap), "logw_c"),
+        _ptr(out.n_kept, torch.int32, (B, H), "n_kept"), cap,
+        _ptr(out.dev_status, torch.int32, (1,), "dev_status"), _stream(stream)))
+    return out
+
+
+def ebd_gather(design: EbdDesign, K: torch.Tensor, V: torch.Tensor, out: CompactCache,
+               stream=None):
+    """Copy the kept K/V rows named by out.idx_c into out.K_c / out.V_c."""
+    B, H, N, d = design.batch, design.n_kv_heads, design.n_ctx, design.head_dim
+    cap = out.capacity
+    _check("ebd_gather", lib().ebd_gather(
+        ctypes.byref(design), _dtype_code(K), _ptr(K, K.dtype, (B, H, N, d), "K"),
+        _ptr(V, K.dtype, (B, H, N, d), "V"), _ptr(out.idx_c, torch.int32, (B, H, cap), "idx_c"),
+        _ptr(out.n_kept, torch.int32, (B, H), "n_kept"), cap,
+        _ptr(out.K_c, K.dtype, (B, H, cap, d), "K_c"), _ptr(out.V_c, K.dtype, (B, H, cap, d), "V_c"),
+        _stream(stream)))
     return out
 
 
