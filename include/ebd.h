@@ -203,6 +203,36 @@ ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32_t n_kv_hea
                                 int32_t* dev_status, void* workspace, size_t ws_bytes,
                                 void* stream);
 
+/*
+ * Certified decode that allocates nothing.  The paper has no counterpart: this
+ * is a deployment variant of ebd_certified_decode for callers that cannot
+ * allocate device memory -- serving stacks that lay out all device memory at
+ * start-up and forbid cudaMalloc afterwards (an allocation can synchronise the
+ * device and break a planned pool), and plugin hosts that give an operator its
+ * inputs and outputs but no allocator.  Arguments, outputs and results are
+ * those of ebd_certified_decode, without the workspace.
+ *
+ * The split-K scratch is a 16 MiB array inside the library (a static
+ * __device__ variable, held by every GPU that loads the library until the
+ * process exits).  The call allocates nothing and calls no allocating routine.
+ * - Returns EBD_ERR_CAPACITY, before enqueueing anything, when the request
+ *   needs more scratch than that (ebd_decode_workspace_bytes(...) > 16 MiB).
+ * - The first call on each device looks up the array's device address with
+ *   that device current (cudaGetSymbolAddress) and caches it; make that first
+ *   call before any stream capture.
+ * - Every call on a device shares the one array, which keeps the previous
+ *   call's contents (nothing in it needs to start at zero).  Calls whose work
+ *   overlaps on the GPU -- unordered streams, or several host threads -- race
+ *   on it; the caller must order them.
+ */
+ebd_status ebd_certified_decode_static(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads,
+                                       int32_t group, int32_t head_dim, const void* Q,
+                                       const void* K_c, const void* V_c, const float* logw_c,
+                                       const int32_t* n_kept, int32_t capacity, float delta,
+                                       float eps0, ebd_range_mode range_mode, float* y,
+                                       float* lse, float* var_hat, float* b_t, float* radius,
+                                       int32_t* dev_status, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -24,7 +24,8 @@ __all__ = [
     "EBD_DEV_CAPACITY", "EBD_DEV_NONFINITE", "EBD_DEV_TIMEOUT", "lib", "lib_path",
     "ebd_status_string", "ebd_abi_version", "ebd_philox_uniforms", "ebd_score_workspace_bytes",
     "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
-    "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode", "design_for",
+    "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
+    "ebd_certified_decode_static", "design_for",
     "CompactCache",
     "alloc_compact", "ABI_FUNCTIONS",
 ]
@@ -39,6 +40,7 @@ ABI_FUNCTIONS = (
     "ebd_status_string", "ebd_abi_version", "ebd_philox_uniforms", "ebd_score_workspace_bytes",
     "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
     "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
+    "ebd_certified_decode_static",
 )
 
 
@@ -99,6 +101,10 @@ def lib():
                                                     f32, f32, ctypes.c_int, c_void_p, c_void_p,
                                                     c_void_p, c_void_p, c_void_p, c_void_p,
                                                     c_void_p, sz, c_void_p]),
+            "ebd_certified_decode_static": (ctypes.c_int, [
+                ctypes.c_int, i32, i32, i32, i32, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                i32, f32, f32, ctypes.c_int, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                c_void_p, c_void_p]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -310,4 +316,28 @@ def ebd_certified_decode(Q: torch.Tensor, K_c: torch.Tensor, V_c: torch.Tensor,
         _ptr(var_hat, f, (B, Hq), "var_hat"), _ptr(b_t, f, (B, Hq), "b_t"),
         _ptr(radius, f, (B, Hq), "radius"), _ptr(dev_status, torch.int32, (1,), "dev_status"),
         ws, wsb, _stream(stream)))
+    return y, lse, var_hat, b_t, radius
+
+
+def ebd_certified_decode_static(Q: torch.Tensor, K_c: torch.Tensor, V_c: torch.Tensor,
+                                logw_c: torch.Tensor, n_kept: torch.Tensor, y: torch.Tensor,
+                                lse: torch.Tensor, var_hat: torch.Tensor, b_t: torch.Tensor,
+                                radius: torch.Tensor, delta: float = 0.1, eps0: float = 1e-9,
+                                range_mode: int = EBD_RANGE_BOUND, dev_status=None, stream=None):
+    """ebd_certified_decode without a workspace: for callers that cannot allocate
+    device memory, the library uses its own fixed 16 MiB scratch array."""
+    B, H, cap, d = K_c.shape
+    Hq = Q.shape[1]
+    if Hq % H:
+        raise ValueError("query heads must be a multiple of KV heads")
+    G = Hq // H
+    f = torch.float32
+    _check("ebd_certified_decode_static", lib().ebd_certified_decode_static(
+        _dtype_code(K_c), B, H, G, d, _ptr(Q, K_c.dtype, (B, Hq, d), "Q"), _ptr(K_c, name="K_c"),
+        _ptr(V_c, K_c.dtype, (B, H, cap, d), "V_c"), _ptr(logw_c, f, (B, H, cap), "logw_c"),
+        _ptr(n_kept, torch.int32, (B, H), "n_kept"), cap, float(delta), float(eps0),
+        int(range_mode), _ptr(y, f, (B, Hq, d), "y"), _ptr(lse, f, (B, Hq), "lse"),
+        _ptr(var_hat, f, (B, Hq), "var_hat"), _ptr(b_t, f, (B, Hq), "b_t"),
+        _ptr(radius, f, (B, Hq), "radius"), _ptr(dev_status, torch.int32, (1,), "dev_status"),
+        _stream(stream)))
     return y, lse, var_hat, b_t, radius
