@@ -94,10 +94,11 @@ int32_t ebd_abi_version(void);
 /*
  * Philox4x32-10 words used by the Poisson draw (Section 3.3: independent
  * Bernoulli(pi_i) retention on the tail).  For every unit (b, kvh) and token
- * i < N writes x0[b,kvh,i] (device uint32 [B,Hkv,N]) = the first output word
- * of Philox4x32-10 (Salmon et al., SC'11) with key (seed_lo, seed_hi) and
- * counter (i, kvh, layer, b).  The uniform the draw compares with pi_i is
- * (x0 >> 8) * 2^-24.  Exposed so that the draws can be checked bit for bit.
+ * i < N writes x0[b,kvh,i] (device uint32 [B,Hkv,N]) = output word i % 4 of
+ * Philox4x32-10 (Salmon et al., SC'11) with key (seed_lo, seed_hi) and
+ * counter (i / 4, kvh, layer, b): one generator call serves four consecutive
+ * tokens.  The uniform the draw compares with pi_i is (x0 >> 8) * 2^-24.
+ * Exposed so that the draws can be checked bit for bit.
  */
 ebd_status ebd_philox_uniforms(uint64_t seed, int32_t layer, int32_t batch, int32_t n_kv_heads,
                                int32_t n_ctx, uint32_t* x0, void* stream);

@@ -24,8 +24,9 @@ the repository's design notes):
 * Grouped-query attention: eviction is per KV head; the certificate is per
   query head.
 * The Poisson draw uses Philox4x32-10 (Salmon et al., SC'11) with key
-  (seed low word, seed high word) and counter (token, kv head, layer, batch
-  row); the uniform is the top 24 bits of the first output word times 2^-24,
+  (seed low word, seed high word) and counter (token // 4, kv head, layer,
+  batch row); token i takes output word i % 4 and its uniform is the top 24
+  bits of that word times 2^-24,
   and a tail token is kept iff  u < float32(pi)  -- the comparison is taken in
   single precision on both sides because that is the precision the device
   path decides it in.
@@ -109,15 +110,17 @@ def philox_uniforms(seed: int, layer: int, b: int, kvh: int, n: int):
     """Uniforms u_i in [0, 1) for tokens i = 0..n-1 of one (layer, b, kvh) unit.
 
     Poisson sampling (Section 3.3) needs one independent Bernoulli(pi_i) draw
-    per tail token.  Key = (seed & 0xffffffff, seed >> 32); counter =
-    (i, kvh, layer, b).  u = (x0 >> 8) * 2^-24 is exact in float32 and float64.
-    Returns (u as float64, raw x0 words as uint32).
+    per tail token.  One Philox4x32-10 call serves four consecutive tokens:
+    key = (seed & 0xffffffff, seed >> 32), counter = (i // 4, kvh, layer, b),
+    and token i takes output word i % 4.  u = (word >> 8) * 2^-24 is exact in
+    float32 and float64.  Returns (u as float64, the raw words as uint32).
     """
     i = np.arange(n, dtype=np.uint64)
-    out = philox4x32_10((i, kvh, layer, b), (seed & _MASK32, (seed >> 32) & _MASK32))
-    x0 = out[0]
-    u = (x0 >> np.uint32(8)).astype(np.float64) * 2.0 ** -24
-    return u, x0
+    out = philox4x32_10((i >> np.uint64(2), kvh, layer, b),
+                        (seed & _MASK32, (seed >> 32) & _MASK32))
+    words = out[(i & np.uint64(3)).astype(np.intp), np.arange(n)]
+    u = (words >> np.uint32(8)).astype(np.float64) * 2.0 ** -24
+    return u, words
 
 
 # ---------------------------------------------------------------------------

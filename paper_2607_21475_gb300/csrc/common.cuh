@@ -68,12 +68,21 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
   return c;
 }
 
-// First Philox word of token i of unit (b, kvh) in `layer`; counter layout
-// (token, kv head, layer, batch row), key (seed low, seed high).
-__device__ __forceinline__ uint32_t draw_word(uint64_t seed, int layer, int b, int kvh, int i) {
-  const uint4 ctr = make_uint4((uint32_t)i, (uint32_t)kvh, (uint32_t)layer, (uint32_t)b);
+// The four Philox words for tokens 4q .. 4q+3 of unit (b, kvh) in `layer`:
+// counter (q, kv head, layer, batch row), key (seed low, seed high).
+__device__ __forceinline__ uint4 draw_block(uint64_t seed, int layer, int b, int kvh, int q) {
+  const uint4 ctr = make_uint4((uint32_t)q, (uint32_t)kvh, (uint32_t)layer, (uint32_t)b);
   const uint2 key = make_uint2((uint32_t)(seed & 0xffffffffu), (uint32_t)(seed >> 32));
-  return philox4x32_10(ctr, key).x;
+  return philox4x32_10(ctr, key);
+}
+
+__device__ __forceinline__ uint32_t word_of(const uint4& w, int r) {
+  return r == 0 ? w.x : (r == 1 ? w.y : (r == 2 ? w.z : w.w));
+}
+
+// Philox word of token i: word i % 4 of the call for tokens 4(i/4) .. 4(i/4)+3.
+__device__ __forceinline__ uint32_t draw_word(uint64_t seed, int layer, int b, int kvh, int i) {
+  return word_of(draw_block(seed, layer, b, kvh, i >> 2), i & 3);
 }
 
 // Uniform in [0,1) from the top 24 bits of a Philox word; exact in float32.

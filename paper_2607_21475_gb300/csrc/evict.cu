@@ -49,6 +49,7 @@ struct SelectArgs {
   int32_t* n_kept;      // [units]
   int cap;
   int32_t* dev_status;  // nullable
+  int vec4;             // scores rows start 16-byte aligned (float4 loads)
 };
 
 struct BlockScratch {
@@ -357,6 +358,372 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
   }
 }
 
+// ---------------------------------------------------------------------------
+// Register-resident variant for N <= 2048 * JG (JG <= 16, i.e. N <= 32768).
+// 512 threads; thread t owns tokens g*2048 + 4t + r (g < JG, r < 4), so the
+// four tokens that share one Philox call live in one thread and every score
+// is read from HBM once.  Membership sets are 64-bit masks (bit 4g + r).
+// The scale c of Eq. (2) is found by bisection on log c whose steps are
+// replaced by the exact linear solve inside the current partition whenever
+// that solve lands inside the bracket (water-filling); it stops once the
+// partition reproduces its own solve, after at most `iters` evaluations.
+// ---------------------------------------------------------------------------
+constexpr int kRegThreads = 512;
+constexpr int kRegWarps = kRegThreads / 32;
+constexpr int kRegMaxGroups = 16;
+
+struct RegScratch {
+  unsigned hist[256];
+  int tot[kRegMaxGroups][kRegWarps];
+  int off[kRegMaxGroups][kRegWarps];
+  float rf[2][kRegWarps];
+  double rd[kRegWarps];
+  int ri[2][kRegWarps];
+  unsigned prefix, remaining;
+  int total;
+};
+
+// Exclusive prefix, over the lanes of this warp, of the number of set bits in
+// 4-bit group g of `flags`.
+__device__ __forceinline__ int lane_prefix(uint64_t flags, int g) {
+  const int lane = threadIdx.x & 31;
+  const int c = __popc((unsigned)((flags >> (4 * g)) & 0xFull));
+  int incl = c;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int n = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += n;
+  }
+  return incl - c;
+}
+
+// Ordered count of the set bits of `flags` (bit 4g + r <-> token
+// g*2048 + 4*tid + r): afterwards sh.off[g][w] is the number of set bits at
+// tokens before warp w's slice of group g; returns the block total.  The rank
+// of a token is sh.off[g][warp] + lane_prefix(flags, g) + its rank in the thread.
+template <int JG>
+__device__ __forceinline__ int ordered_scan(uint64_t flags, RegScratch& sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  __syncthreads();  // previous readers of sh.off / sh.total are done
+#pragma unroll
+  for (int g = 0; g < JG; ++g) {
+    const int c = __popc((unsigned)((flags >> (4 * g)) & 0xFull));
+    const int tot = warp_sum(c);
+    if (lane == 0) sh.tot[g][warp] = tot;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    constexpr int E = JG * kRegWarps;
+    constexpr int PER = (E + 31) / 32;
+    int v[PER];
+    int local = 0;
+#pragma unroll
+    for (int q = 0; q < PER; ++q) {
+      const int e = lane * PER + q;
+      v[q] = e < E ? sh.tot[e / kRegWarps][e % kRegWarps] : 0;
+      local += v[q];
+    }
+    int incl = local;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int n = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += n;
+    }
+    int run = incl - local;
+#pragma unroll
+    for (int q = 0; q < PER; ++q) {
+      const int e = lane * PER + q;
+      if (e < E) sh.off[e / kRegWarps][e % kRegWarps] = run;
+      run += v[q];
+    }
+    if (lane == 31) sh.total = incl;
+  }
+  __syncthreads();
+  return sh.total;
+}
+
+template <int JG>
+__global__ void __launch_bounds__(kRegThreads, 1) evict_select_reg_kernel(SelectArgs a) {
+  __shared__ RegScratch sh;
+  const int unit = blockIdx.x;
+  const int b = unit / a.n_kv_heads;
+  const int kvh = unit - b * a.n_kv_heads;
+  const int N = a.n_ctx;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const float* sp = a.scores + (size_t)unit * N;
+  const int ns = min(a.n_sink, N);
+  const int rs = max(N - a.n_recent, 0);
+  const int n_prot = ns + (N - rs) - max(0, ns - rs);
+  const int n_cand = N - n_prot;
+  const int k = min(max(a.k_head, 0), n_cand);
+  const float eps = a.eps;
+  // token of (g, r) is g*2048 + 4*tid + r
+#define EBD_TOK(g, r) ((g) * 2048 + 4 * tid + (r))
+#define EBD_CAND(i) ((i) < N && (i) >= ns && (i) < rs)
+
+  float s[JG][4];
+  bool bad = false;
+  uint64_t cert = 0ull;
+#pragma unroll
+  for (int g = 0; g < JG; ++g) {
+    const int i0 = EBD_TOK(g, 0);
+    if (a.vec4 && i0 + 3 < N) {
+      const float4 v4 = __ldg(reinterpret_cast<const float4*>(sp + i0));
+      s[g][0] = v4.x;
+      s[g][1] = v4.y;
+      s[g][2] = v4.z;
+      s[g][3] = v4.w;
+    } else {
+#pragma unroll
+      for (int r = 0; r < 4; ++r) s[g][r] = (i0 + r < N) ? __ldg(sp + i0 + r) : 0.f;
+    }
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const int i = i0 + r;
+      float v = s[g][r];
+      if (!isfinite(v)) {
+        bad = bad || (i < N);
+        v = 0.f;
+      }
+      s[g][r] = v + 0.0f;
+      if (i < N && !EBD_CAND(i)) cert |= 1ull << (4 * g + r);  // protected
+    }
+  }
+
+  // ---- E1: top-k_head among the unprotected tokens ------------------------
+  if (k > 0 && k < n_cand) {
+    unsigned prefix = 0u, maskbits = 0u, remaining = (unsigned)k;
+    for (int shift = 24; shift >= 0; shift -= 8) {
+      for (int j = tid; j < 256; j += kRegThreads) sh.hist[j] = 0u;
+      __syncthreads();
+#pragma unroll
+      for (int g = 0; g < JG; ++g) {
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          if (!EBD_CAND(EBD_TOK(g, r))) continue;
+          const uint32_t key = orderable_key(s[g][r]);
+          if ((key & maskbits) == prefix) atomicAdd(&sh.hist[(key >> shift) & 255u], 1u);
+        }
+      }
+      __syncthreads();
+      if (warp == 0) {
+        unsigned c[8];
+        unsigned tot = 0;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          c[q] = sh.hist[255 - 8 * lane - q];
+          tot += c[q];
+        }
+        unsigned incl = tot;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const unsigned n = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += n;
+        }
+        const unsigned excl = incl - tot;
+        if (excl < remaining && incl >= remaining) {
+          unsigned cum = excl;
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            if (cum + c[q] >= remaining) {
+              sh.prefix = prefix | ((unsigned)(255 - 8 * lane - q) << shift);
+              sh.remaining = remaining - cum;
+              break;
+            }
+            cum += c[q];
+          }
+        }
+      }
+      __syncthreads();
+      prefix = sh.prefix;
+      remaining = sh.remaining;
+      maskbits |= 255u << shift;
+    }
+    uint64_t eq = 0ull;
+#pragma unroll
+    for (int g = 0; g < JG; ++g) {
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        if (!EBD_CAND(EBD_TOK(g, r))) continue;
+        const uint32_t key = orderable_key(s[g][r]);
+        if (key > prefix) cert |= 1ull << (4 * g + r);
+        else if (key == prefix) eq |= 1ull << (4 * g + r);
+      }
+    }
+    ordered_scan<JG>(eq, sh);
+#pragma unroll
+    for (int g = 0; g < JG; ++g) {
+      int run = sh.off[g][warp] + lane_prefix(eq, g);
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const uint64_t bit = 1ull << (4 * g + r);
+        if (eq & bit) {
+          if (run < (int)remaining) cert |= bit;
+          ++run;
+        }
+      }
+    }
+  } else if (k > 0) {
+#pragma unroll
+    for (int g = 0; g < JG; ++g)
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+        if (EBD_TOK(g, r) < N) cert |= 1ull << (4 * g + r);
+  }
+#define EBD_TAIL(g, r) (EBD_TOK(g, r) < N && !((cert >> (4 * (g) + (r))) & 1ull))
+
+  // ---- E2: inclusion probabilities on the tail ---------------------------
+  const int n_cert = n_prot + k;
+  const int nT = N - n_cert;
+  const int m = min(max(a.budget - n_cert, 0), nT);
+  float smax = -INFINITY, sminpos = INFINITY, spos = 0.f;
+  int npos = 0;
+#pragma unroll
+  for (int g = 0; g < JG; ++g) {
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      if (!EBD_TAIL(g, r)) continue;
+      const float v = s[g][r];
+      smax = fmaxf(smax, v);
+      if (v > 0.f) {
+        sminpos = fminf(sminpos, v);
+        spos += v;
+        ++npos;
+      }
+    }
+  }
+  smax = warp_max(smax);
+  sminpos = warp_min(sminpos);
+  npos = warp_sum(npos);
+  double spos_d = warp_sum((double)spos);
+  __syncthreads();
+  if (lane == 0) {
+    sh.rf[0][warp] = smax;
+    sh.rf[1][warp] = sminpos;
+    sh.ri[0][warp] = npos;
+    sh.rd[warp] = spos_d;
+  }
+  __syncthreads();
+  smax = sh.rf[0][0];
+  sminpos = sh.rf[1][0];
+  npos = 0;
+  spos_d = 0.0;
+#pragma unroll
+  for (int w = 0; w < kRegWarps; ++w) {
+    smax = fmaxf(smax, sh.rf[0][w]);
+    sminpos = fminf(sminpos, sh.rf[1][w]);
+    npos += sh.ri[0][w];
+    spos_d += sh.rd[w];
+  }
+
+  int mode = kPiLinear;
+  float c = 0.f;
+  if (nT == 0 || (float)m <= eps * (float)nT) {
+    mode = kPiFloor;
+  } else if ((float)m >= (float)npos + eps * (float)(nT - npos)) {
+    mode = kPiAll;
+  } else {
+    float lo = logf(eps / smax), hi = logf(1.f / sminpos);
+    c = fminf(fmaxf((float)((double)m / spos_d), expf(lo)), expf(hi));
+    for (int it = 0; it < a.iters; ++it) {
+      int nhi = 0, nlo = 0;
+      float smid = 0.f;
+#pragma unroll
+      for (int g = 0; g < JG; ++g) {
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          if (!EBD_TAIL(g, r)) continue;
+          const float t = c * s[g][r];
+          if (t >= 1.f) ++nhi;
+          else if (t <= eps) ++nlo;
+          else smid += s[g][r];
+        }
+      }
+      nhi = warp_sum(nhi);
+      nlo = warp_sum(nlo);
+      double smid_d = warp_sum((double)smid);
+      __syncthreads();
+      if (lane == 0) {
+        sh.ri[0][warp] = nhi;
+        sh.ri[1][warp] = nlo;
+        sh.rd[warp] = smid_d;
+      }
+      __syncthreads();
+      nhi = 0;
+      nlo = 0;
+      smid_d = 0.0;
+#pragma unroll
+      for (int w = 0; w < kRegWarps; ++w) {
+        nhi += sh.ri[0][w];
+        nlo += sh.ri[1][w];
+        smid_d += sh.rd[w];
+      }
+      const double gval = nhi + (double)eps * nlo + (double)c * smid_d;
+      if (gval < (double)m) lo = fmaxf(lo, logf(c));
+      else hi = fminf(hi, logf(c));
+      const double clin = smid_d > 0.0 ? ((double)m - nhi - (double)eps * nlo) / smid_d : -1.0;
+      if (clin > 0.0 && fabs(clin - (double)c) <= 1e-6 * (double)c) {
+        c = (float)clin;  // the partition at c reproduces its own solve
+        break;
+      }
+      float next;
+      const float lcl = clin > 0.0 ? logf((float)clin) : -INFINITY;
+      if (clin > 0.0 && lcl > lo && lcl < hi) next = (float)clin;
+      else next = expf(0.5f * (lo + hi));
+      if (next == c) break;
+      c = next;
+    }
+  }
+
+  // ---- E3 + E4a: draws and ordered compaction of (index, log 1/pi) --------
+  const bool compact = a.n_kept != nullptr;
+  uint64_t keep = 0ull;
+#pragma unroll
+  for (int g = 0; g < JG; ++g) {
+    bool any_tail = false;
+#pragma unroll
+    for (int r = 0; r < 4; ++r) any_tail = any_tail || EBD_TAIL(g, r);
+    uint4 w = make_uint4(0u, 0u, 0u, 0u);
+    if (compact && __any_sync(0xffffffffu, any_tail)) w = draw_block(a.seed, a.layer, b, kvh, g * 512 + tid);
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const int i = EBD_TOK(g, r);
+      if (i >= N) continue;
+      const bool ct = (cert >> (4 * g + r)) & 1ull;
+      const float pi = ct ? 1.f : tail_pi(s[g][r], mode, c, eps);
+      if (a.pi_out) a.pi_out[(size_t)unit * N + i] = pi;
+      if (a.mask_out) a.mask_out[(size_t)unit * N + i] = ct ? 1 : 0;
+      if (compact && (ct || word_to_uniform(word_of(w, r)) < pi)) keep |= 1ull << (4 * g + r);
+    }
+  }
+  if (compact) {
+    const int total = ordered_scan<JG>(keep, sh);
+#pragma unroll
+    for (int g = 0; g < JG; ++g) {
+      int p = sh.off[g][warp] + lane_prefix(keep, g);
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const uint64_t bit = 1ull << (4 * g + r);
+        if (!(keep & bit)) continue;
+        if (p < a.cap) {
+          const float pi = (cert & bit) ? 1.f : tail_pi(s[g][r], mode, c, eps);
+          a.idx_c[(size_t)unit * a.cap + p] = EBD_TOK(g, r);
+          a.logw_c[(size_t)unit * a.cap + p] = pi >= 1.f ? 0.f : -logf(pi);
+        }
+        ++p;
+      }
+    }
+    if (tid == 0) {
+      a.n_kept[unit] = total;
+      if (total > a.cap) raise_status(a.dev_status, EBD_DEV_CAPACITY);
+    }
+  }
+  if (__syncthreads_or(bad) && tid == 0) raise_status(a.dev_status, EBD_DEV_NONFINITE);
+#undef EBD_TAIL
+#undef EBD_CAND
+#undef EBD_TOK
+}
+
 // E4b: copy kept K and V rows (16-byte chunks, `cpr` chunks per row).
 constexpr int kGatherThreads = 256;
 constexpr int kGatherUnroll = 4;
@@ -458,13 +825,23 @@ static ebd_status launch_select(const ebd_design* d, const float* scores, float*
   a.n_kept = n_kept;
   a.cap = cap;
   a.dev_status = dev_status;
+  a.vec4 = (((uintptr_t)scores & 15u) == 0 && (d->n_ctx & 3) == 0) ? 1 : 0;
+  const int units = d->batch * d->n_kv_heads;
+  const int groups = (d->n_ctx + 2047) / 2048;
+  if (groups <= kRegMaxGroups) {
+    if (groups <= 1) evict_select_reg_kernel<1><<<units, kRegThreads, 0, stream>>>(a);
+    else if (groups <= 2) evict_select_reg_kernel<2><<<units, kRegThreads, 0, stream>>>(a);
+    else if (groups <= 4) evict_select_reg_kernel<4><<<units, kRegThreads, 0, stream>>>(a);
+    else if (groups <= 8) evict_select_reg_kernel<8><<<units, kRegThreads, 0, stream>>>(a);
+    else evict_select_reg_kernel<16><<<units, kRegThreads, 0, stream>>>(a);
+    return launch_status();
+  }
   const size_t smem = (size_t)((d->n_ctx + 31) / 32) * 4;
   if (smem > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(evict_select_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return EBD_ERR_CUDA;
   }
-  const int units = d->batch * d->n_kv_heads;
   evict_select_kernel<<<units, kSelThreads, smem, stream>>>(a);
   return launch_status();
 }

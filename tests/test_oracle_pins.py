@@ -73,9 +73,10 @@ def test_uniforms_grid_and_distribution():
     # seed's high word is the second key word
     hi, _ = philox_uniforms(7 + (1 << 32), 3, 2, 1, 1000)
     assert np.mean(hi == base) < 0.01
-    # token i of the unit is counter word 0 = i
-    direct = philox4x32_10((5, 1, 3, 2), (7, 0))[0]
-    assert int(direct) >> 8 == int(base[5] * 2**24)
+    # token i of the unit is word i % 4 of the call with counter word 0 = i // 4
+    for i in (0, 5, 10, 999):
+        direct = philox4x32_10((i // 4, 1, 3, 2), (7, 0))[i % 4]
+        assert int(direct) >> 8 == int(base[i] * 2**24)
 
 
 # ------------------------------------------------------------ Eq. (1) and scoring
