@@ -157,7 +157,10 @@ __global__ void __launch_bounds__(kGenThreads) decode_generic_kernel(DecodeArgs 
   }
 }
 
-// Merge the split records of one query head and finish Eq. (3), Theorem 2, Eq. (4).
+// Merge the partial records of one query head and finish Eq. (3), Theorem 2, Eq. (4).
+// CUDA-core path: records u*splits .. u*splits + splits - 1.  Tensor-core
+// path: records u + gw for every consumer warp gw whose tile range meets
+// unit u (none for an empty unit).
 template <int D>
 __global__ void __launch_bounds__(D) decode_reduce_kernel(ReduceArgs a) {
   constexpr int REC = rec_floats(D);
@@ -166,10 +169,24 @@ __global__ void __launch_bounds__(D) decode_reduce_kernel(ReduceArgs a) {
   const int G = a.group;
   const int unit = hq / G, g = hq - unit * G;
   const int e = threadIdx.x;
-  const float* P = a.part + ((size_t)unit * a.splits * G + g) * REC;
+  long long first = (long long)unit * a.splits;
+  int count = a.splits;
+  if (a.tile_off) {
+    const long long t0 = a.tile_off[unit], t1 = a.tile_off[unit + 1];
+    const long long Ta = a.tile_off[gridDim.x / G];
+    const long long W = a.warps < Ta ? a.warps : Ta;
+    count = 0;
+    if (t1 > t0) {
+      const long long gf = ((t0 + 1) * W - 1) / Ta;
+      const long long gl = (t1 * W - 1) / Ta;
+      first = unit + gf;
+      count = (int)(gl - gf + 1);
+    }
+  }
+  const float* P = a.part + ((size_t)first * G + g) * REC;
   const size_t sstride = (size_t)G * REC;
   float Mx = -INFINITY;
-  for (int s = 0; s < a.splits; ++s) Mx = fmaxf(Mx, P[s * sstride + kRecM]);
+  for (int s = 0; s < count; ++s) Mx = fmaxf(Mx, P[s * sstride + kRecM]);
   if (Mx == -INFINITY) {  // empty unit
     a.y[(size_t)hq * D + e] = 0.f;
     if (e == 0) {
@@ -181,7 +198,7 @@ __global__ void __launch_bounds__(D) decode_reduce_kernel(ReduceArgs a) {
     return;
   }
   float l = 0.f, U = 0.f, A2 = 0.f, cmax = 0.f, umax = 0.f, o = 0.f, a1 = 0.f;
-  for (int s = 0; s < a.splits; ++s) {
+  for (int s = 0; s < count; ++s) {
     const float* R = P + s * sstride;
     const float Ms = R[kRecM];
     if (Ms == -INFINITY) continue;
@@ -365,21 +382,17 @@ static DecodePlan plan_generic(long long units, int group, int head_dim, int cap
   return p;
 }
 
-DecodePlan plan_generic_for_exact(int batch, int n_kv_heads, int group, int head_dim,
-                                  int capacity) {
-  return plan_generic((long long)batch * n_kv_heads, group, head_dim, capacity);
-}
-
 DecodePlan plan_decode(ebd_dtype dtype, int batch, int n_kv_heads, int group, int head_dim,
                        int capacity) {
   const long long units = (long long)batch * n_kv_heads;
+  DecodePlan p = plan_generic(units, group, head_dim, capacity);
   if (fast_decode_supported(dtype, group, head_dim, capacity)) {
-    DecodePlan p;
+    const size_t generic_ws = p.ws_bytes;
     p.fast = true;
     fast_decode_plan(p, units, group, head_dim, capacity);
-    return p;
+    if (p.ws_bytes < generic_ws) p.ws_bytes = generic_ws;  // either path fits
   }
-  return plan_generic(units, group, head_dim, capacity);
+  return p;
 }
 
 }  // namespace ebd
@@ -430,8 +443,9 @@ extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32
   a.lse = lse;
   a.dev_status = dev_status;
 
+  const bool fast = plan.fast && fast_decode_usable(a, (int)units);
   ebd_status st;
-  if (plan.fast)
+  if (fast)
     st = launch_fast_decode(dtype, head_dim, plan, a, (int)units, s);
   else
     st = dispatch_generic(false, dtype, head_dim, a, (int)units, s);
@@ -439,7 +453,14 @@ extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32
 
   ReduceArgs r;
   r.part = (const float*)workspace;
-  r.splits = plan.fast ? plan.reduce_slots : plan.splits;
+  r.splits = plan.splits;
+  r.tile_off = nullptr;
+  r.warps = 0;
+  if (fast) {
+    r.tile_off = (const int32_t*)workspace;
+    r.part = (const float*)((const char*)workspace + fast_decode_records_offset((int)units));
+    r.warps = fast_decode_warps(plan);
+  }
   r.group = group;
   r.y = y;
   r.lse = lse;
@@ -458,10 +479,8 @@ extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32
   if (st != EBD_OK || !r.exact) return st;
 
   // exact range term: second pass over the tail rows, then the radius
-  DecodePlan gp = plan;
-  if (plan.fast) gp = plan_generic_for_exact(batch, n_kv_heads, group, head_dim, capacity);
-  a.splits = gp.splits;
-  a.tokens_per_split = gp.tokens_per_split;
+  a.splits = plan.splits;
+  a.tokens_per_split = plan.tokens_per_split;
   a.b_t = b_t;
   st = dispatch_generic(true, dtype, head_dim, a, (int)units, s);
   if (st != EBD_OK) return st;

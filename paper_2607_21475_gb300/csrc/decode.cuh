@@ -40,7 +40,9 @@ struct DecodeArgs {
 
 struct ReduceArgs {
   const float* part;
-  int splits;
+  int splits;                // CUDA-core path: records per unit
+  const int32_t* tile_off;   // tensor-core path: active-tile prefix (null otherwise)
+  long long warps;           // tensor-core path: consumer warps in the grid
   int group;
   float* y;
   float* lse;
@@ -53,21 +55,21 @@ struct ReduceArgs {
 };
 
 struct DecodePlan {
-  bool fast = false;
+  bool fast = false;         // the tensor-core path applies to this request
   int splits = 1;            // CUDA-core path: splits per unit
   int tokens_per_split = 0;  // CUDA-core path
-  int reduce_slots = 1;      // tensor-core path: record slots per unit
   int ctas = 0;              // tensor-core path: persistent grid size
-  int tiles_per_unit = 0;    // tensor-core path
   size_t ws_bytes = 0;
 };
 
 DecodePlan plan_decode(ebd_dtype dtype, int batch, int n_kv_heads, int group, int head_dim,
                        int capacity);
-DecodePlan plan_generic_for_exact(int batch, int n_kv_heads, int group, int head_dim, int capacity);
 
 // Tensor-core path (decode_mma.cu).
 bool fast_decode_supported(ebd_dtype dtype, int group, int head_dim, int capacity);
+bool fast_decode_usable(const DecodeArgs& a, int units);
+long long fast_decode_warps(const DecodePlan& p);
+size_t fast_decode_records_offset(int units);
 void fast_decode_plan(DecodePlan& p, long long units, int group, int head_dim, int capacity);
 ebd_status launch_fast_decode(ebd_dtype dtype, int head_dim, const DecodePlan& plan,
                               const DecodeArgs& a, int units, cudaStream_t stream);

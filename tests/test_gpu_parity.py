@@ -222,6 +222,9 @@ DECODE_CASES = [
     (3, 2, 4, 128, 704, torch.bfloat16, "edges"),   # 0, 1, cap, ragged
     (2, 2, 8, 64, 320, torch.float32, "edges"),
     (1, 3, 2, 128, 64, torch.bfloat16, "full"),
+    (2, 2, 8, 64, 512, torch.bfloat16, "edges"),     # tensor-core path, head_dim 64, G = 8
+    (2, 3, 5, 128, 1000, torch.bfloat16, "random"),  # capacity not a multiple of 16: CUDA cores
+    (1, 64, 4, 128, 256, torch.bfloat16, "random"),  # more warps than tiles
 ]
 
 
