@@ -60,7 +60,14 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--no-graph", action="store_true")
+    p.add_argument("--batch", type=int, default=0,
+                   help="override the workload's batch (smaller cases for profiling)")
     return p.parse_args()
+
+
+def workload_of(args) -> Workload:
+    w = WORKLOADS[args.workload]
+    return w.with_(batch=args.batch) if args.batch > 0 else w
 
 
 def dist_setup(args):
@@ -375,7 +382,7 @@ def config_of(w: Workload):
 def run_reference(args, world, rank):
     if rank != 0:
         return
-    w = WORKLOADS[args.workload]
+    w = workload_of(args)
     dev = "cuda" if torch.cuda.is_available() else "cpu"
     inputs = make_layer_inputs(w, 0, dev)
     per_step = max(2.0, 150.0 / max(1, args.steps + args.warmup))
@@ -403,7 +410,7 @@ def run_reference(args, world, rank):
 
 
 def run_ours(args, world, rank, local):
-    w = WORKLOADS[args.workload]
+    w = workload_of(args)
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     hbm_peak, peak_kind, peaks = measured_peaks()

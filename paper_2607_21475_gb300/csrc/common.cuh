@@ -98,6 +98,16 @@ __device__ __forceinline__ uint32_t orderable_key(float s) {
   return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
 }
 
+// 1 - e^-x for x >= 0 (x = log(1/pi), so the result is 1 - pi).  Below 0.25
+// the Taylor series to x^6 (truncation < 5e-8 relative) avoids the
+// cancellation of 1 - e^-x; above it, 1 - e^-x >= 0.22 and exp2 suffices.
+__device__ __forceinline__ float one_minus_exp_neg(float x) {
+  if (x < 0.25f) {
+    return x * (1.f - x * (0.5f - x * (1.f / 6.f - x * (1.f / 24.f - x * (1.f / 120.f - x * (1.f / 720.f))))));
+  }
+  return 1.f - exp2f(-x * kLog2e);
+}
+
 __device__ __forceinline__ void raise_status(int32_t* st, int32_t bits) {
   if (st) atomicOr(st, bits);
 }

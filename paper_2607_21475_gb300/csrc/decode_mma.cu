@@ -169,12 +169,13 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
 
   // copies: lane 0 walks its own cursor through the warp's tiles
   int pf_t = tb, pf_u = unit_of_tile(a.tile_off, units, tb);
+  int pf_lo = __ldg(a.tile_off + pf_u), pf_hi = __ldg(a.tile_off + pf_u + 1);
   int issued = 0;
   auto issue_next = [&]() {
     if (lane == 0 && pf_t < te) {
       const int s = issued % kMmaStagesPerWarp;
       const int stage = warp * kMmaStagesPerWarp + s;
-      const int row0 = pf_u * a.cap + (pf_t - __ldg(a.tile_off + pf_u)) * kMmaTile;
+      const int row0 = pf_u * a.cap + (pf_t - pf_lo) * kMmaTile;
       unsigned char* st = smem + (size_t)stage * L::kStageBytes;
       mbar_arrive_expect_tx(&my_full[s], L::kTxBytes);
 #pragma unroll
@@ -184,7 +185,11 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
       }
       bulk_load(lw_s + stage * kMmaTile, a.logw + row0, kMmaTile * 4, &my_full[s]);
       ++pf_t;
-      if (pf_t < te && pf_t == __ldg(a.tile_off + pf_u + 1)) pf_u = next_unit(a.tile_off, pf_u);
+      if (pf_t < te && pf_t == pf_hi) {
+        pf_u = next_unit(a.tile_off, pf_u);
+        pf_lo = pf_hi;
+        pf_hi = __ldg(a.tile_off + pf_u + 1);
+      }
     }
     ++issued;
   };
@@ -317,7 +322,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     for (int i = 0; i < 4; ++i) {
       const bool val = tk[i] < n_valid;
       wv[i] = exp2f(x[i] - M2);
-      const float omp = val ? -expm1f(-lwv[i]) : 0.f;  // 1 - pi
+      const float omp = val ? one_minus_exp_neg(lwv[i]) : 0.f;  // 1 - pi
       uv[i] = omp * wv[i] * wv[i];
       suv[i] = sqrtf(omp) * wv[i];
       umax = fmaxf(umax, suv[i]);
@@ -341,7 +346,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     // ---- acc += P V, ||v||^2 -------------------------------------------------
     const uint32_t m01 = (tk[0] < n_valid ? 0x0000ffffu : 0u) | (tk[1] < n_valid ? 0xffff0000u : 0u);
     const uint32_t m23 = (tk[2] < n_valid ? 0x0000ffffu : 0u) | (tk[3] < n_valid ? 0xffff0000u : 0u);
-    float vn[4] = {0.f, 0.f, 0.f, 0.f};
+    float2 vn01 = make_float2(0.f, 0.f), vn23 = make_float2(0.f, 0.f);
     {
       const int tok = ((lane >> 3) & 1) * 8 + (lane & 7);
       const int chunk_sel = lane >> 4;
@@ -356,10 +361,12 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
         v2 &= m01;
         v1 &= m23;
         v3 &= m23;
-        vn[0] = fmaf(bf16_lo(v0), bf16_lo(v0), fmaf(bf16_lo(v2), bf16_lo(v2), vn[0]));
-        vn[1] = fmaf(bf16_hi(v0), bf16_hi(v0), fmaf(bf16_hi(v2), bf16_hi(v2), vn[1]));
-        vn[2] = fmaf(bf16_lo(v1), bf16_lo(v1), fmaf(bf16_lo(v3), bf16_lo(v3), vn[2]));
-        vn[3] = fmaf(bf16_hi(v1), bf16_hi(v1), fmaf(bf16_hi(v3), bf16_hi(v3), vn[3]));
+        const float2 f0 = make_float2(bf16_lo(v0), bf16_hi(v0));
+        const float2 f1 = make_float2(bf16_lo(v1), bf16_hi(v1));
+        const float2 f2 = make_float2(bf16_lo(v2), bf16_hi(v2));
+        const float2 f3 = make_float2(bf16_lo(v3), bf16_hi(v3));
+        vn01 = __ffma2_rn(f0, f0, __ffma2_rn(f2, f2, vn01));
+        vn23 = __ffma2_rn(f1, f1, __ffma2_rn(f3, f3, vn23));
         mma_bf16_16816(acc[2 * jp], h0, h1, h2, h3, v0, v1);
         mma_bf16_16816(acc[2 * jp], r0, r1, r2, r3, v0, v1);
         mma_bf16_16816(acc[2 * jp + 1], h0, h1, h2, h3, v2, v3);
@@ -369,6 +376,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     // reads of this stage are done before a later copy overwrites it
     fence_proxy_async_smem();
     __syncwarp();
+    float vn[4] = {vn01.x, vn01.y, vn23.x, vn23.y};
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       vn[i] += __shfl_xor_sync(0xffffffffu, vn[i], 4);

@@ -359,29 +359,75 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
 }
 
 // ---------------------------------------------------------------------------
-// Register-resident variant for N <= 2048 * JG (JG <= 16, i.e. N <= 32768).
-// 512 threads; thread t owns tokens g*2048 + 4t + r (g < JG, r < 4), so the
-// four tokens that share one Philox call live in one thread and every score
-// is read from HBM once.  Membership sets are 64-bit masks (bit 4g + r).
+// Shared-memory variant for N <= 4096 * JG (JG <= 8, i.e. N <= 32768).
+// 1024 threads; thread t owns tokens g*4096 + 4t + r (g < JG, r < 4): the four
+// tokens that share one Philox call live in one thread, and its scores sit in
+// shared memory as one float4 per group (read once from HBM).  Membership is
+// a 64-bit mask per thread (bit 4g + r).  Loops over groups stay rolled so the
+// kernel stays small in the instruction cache.
 // The scale c of Eq. (2) is found by bisection on log c whose steps are
 // replaced by the exact linear solve inside the current partition whenever
 // that solve lands inside the bracket (water-filling); it stops once the
 // partition reproduces its own solve, after at most `iters` evaluations.
 // ---------------------------------------------------------------------------
-constexpr int kRegThreads = 512;
+constexpr int kRegThreads = 1024;
 constexpr int kRegWarps = kRegThreads / 32;
-constexpr int kRegMaxGroups = 16;
+constexpr int kRegMaxGroups = 8;
+constexpr int kGroupTokens = 4 * kRegThreads;
 
 struct RegScratch {
   unsigned hist[256];
   int tot[kRegMaxGroups][kRegWarps];
   int off[kRegMaxGroups][kRegWarps];
-  float rf[2][kRegWarps];
-  double rd[kRegWarps];
+  float rf[3][kRegWarps];
   int ri[2][kRegWarps];
+  double res_d;
+  float res_f[2];
+  int res_i[2];
+  float c, lo, hi;  // solve state, updated by thread 0 only
+  int mode, stop;
   unsigned prefix, remaining;
   int total;
 };
+
+// Cross-warp combine of per-warp partials written to sh.rf / sh.ri by lane 0
+// of every warp: warp 0 reduces the kRegWarps entries (the float sum in
+// double, so that only 32 lanes touch the slow fp64 pipe) and publishes
+// res_*.  Callers bracket it with barriers.
+__device__ __forceinline__ void combine_stats(RegScratch& sh) {
+  const int lane = threadIdx.x & 31;
+  if ((threadIdx.x >> 5) == 0) {
+    float mx = sh.rf[0][lane], mn = sh.rf[1][lane];
+    double sd = (double)sh.rf[2][lane];
+    int n = sh.ri[0][lane];
+    mx = warp_max(mx);
+    mn = warp_min(mn);
+    sd = warp_sum(sd);
+    n = warp_sum(n);
+    if (lane == 0) {
+      sh.res_f[0] = mx;
+      sh.res_f[1] = mn;
+      sh.res_d = sd;
+      sh.res_i[0] = n;
+    }
+  }
+}
+
+__device__ __forceinline__ void combine_partition(RegScratch& sh) {
+  const int lane = threadIdx.x & 31;
+  if ((threadIdx.x >> 5) == 0) {
+    double sd = (double)sh.rf[0][lane];
+    int a = sh.ri[0][lane], b = sh.ri[1][lane];
+    sd = warp_sum(sd);
+    a = warp_sum(a);
+    b = warp_sum(b);
+    if (lane == 0) {
+      sh.res_d = sd;
+      sh.res_i[0] = a;
+      sh.res_i[1] = b;
+    }
+  }
+}
 
 // Exclusive prefix, over the lanes of this warp, of the number of set bits in
 // 4-bit group g of `flags`.
@@ -398,14 +444,13 @@ __device__ __forceinline__ int lane_prefix(uint64_t flags, int g) {
 }
 
 // Ordered count of the set bits of `flags` (bit 4g + r <-> token
-// g*2048 + 4*tid + r): afterwards sh.off[g][w] is the number of set bits at
+// g*4096 + 4*tid + r): afterwards sh.off[g][w] is the number of set bits at
 // tokens before warp w's slice of group g; returns the block total.  The rank
 // of a token is sh.off[g][warp] + lane_prefix(flags, g) + its rank in the thread.
-template <int JG>
-__device__ __forceinline__ int ordered_scan(uint64_t flags, RegScratch& sh) {
+__device__ __forceinline__ int ordered_scan(uint64_t flags, int JG, RegScratch& sh) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   __syncthreads();  // previous readers of sh.off / sh.total are done
-#pragma unroll
+#pragma unroll 1
   for (int g = 0; g < JG; ++g) {
     const int c = __popc((unsigned)((flags >> (4 * g)) & 0xFull));
     const int tot = warp_sum(c);
@@ -413,15 +458,14 @@ __device__ __forceinline__ int ordered_scan(uint64_t flags, RegScratch& sh) {
   }
   __syncthreads();
   if (warp == 0) {
-    constexpr int E = JG * kRegWarps;
-    constexpr int PER = (E + 31) / 32;
-    int v[PER];
+    const int E = JG * kRegWarps;               // <= 256
+    const int PER = (E + 31) / 32;              // <= 8
+
     int local = 0;
-#pragma unroll
+#pragma unroll 1
     for (int q = 0; q < PER; ++q) {
       const int e = lane * PER + q;
-      v[q] = e < E ? sh.tot[e / kRegWarps][e % kRegWarps] : 0;
-      local += v[q];
+      if (e < E) local += sh.tot[e / kRegWarps][e % kRegWarps];
     }
     int incl = local;
 #pragma unroll
@@ -430,11 +474,14 @@ __device__ __forceinline__ int ordered_scan(uint64_t flags, RegScratch& sh) {
       if (lane >= o) incl += n;
     }
     int run = incl - local;
-#pragma unroll
+#pragma unroll 1
     for (int q = 0; q < PER; ++q) {
       const int e = lane * PER + q;
-      if (e < E) sh.off[e / kRegWarps][e % kRegWarps] = run;
-      run += v[q];
+      if (e < E) {
+        const int v = sh.tot[e / kRegWarps][e % kRegWarps];
+        sh.off[e / kRegWarps][e % kRegWarps] = run;
+        run += v;
+      }
     }
     if (lane == 31) sh.total = incl;
   }
@@ -442,8 +489,8 @@ __device__ __forceinline__ int ordered_scan(uint64_t flags, RegScratch& sh) {
   return sh.total;
 }
 
-template <int JG>
-__global__ void __launch_bounds__(kRegThreads, 1) evict_select_reg_kernel(SelectArgs a) {
+__global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(SelectArgs a, int JG) {
+  extern __shared__ float4 s4[];  // [JG][1024]: scores of thread t, group g at s4[g*1024 + t]
   __shared__ RegScratch sh;
   const int unit = blockIdx.x;
   const int b = unit / a.n_kv_heads;
@@ -457,52 +504,63 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_reg_kernel(Select
   const int n_cand = N - n_prot;
   const int k = min(max(a.k_head, 0), n_cand);
   const float eps = a.eps;
-  // token of (g, r) is g*2048 + 4*tid + r
-#define EBD_TOK(g, r) ((g) * 2048 + 4 * tid + (r))
-#define EBD_CAND(i) ((i) < N && (i) >= ns && (i) < rs)
+  auto tok = [&](int g, int r) { return g * kGroupTokens + 4 * tid + r; };
+  auto is_cand = [&](int i) { return i < N && i >= ns && i < rs; };
 
-  float s[JG][4];
+  // ---- load: sanitise, fold -0 onto +0, protected positions -------------------
   bool bad = false;
   uint64_t cert = 0ull;
+  // every group's load in flight before the first use
 #pragma unroll
-  for (int g = 0; g < JG; ++g) {
-    const int i0 = EBD_TOK(g, 0);
+  for (int g = 0; g < kRegMaxGroups; ++g) {
+    if (g >= JG) break;
+    const int i0 = tok(g, 0);
+    float v[4];
     if (a.vec4 && i0 + 3 < N) {
       const float4 v4 = __ldg(reinterpret_cast<const float4*>(sp + i0));
-      s[g][0] = v4.x;
-      s[g][1] = v4.y;
-      s[g][2] = v4.z;
-      s[g][3] = v4.w;
+      v[0] = v4.x;
+      v[1] = v4.y;
+      v[2] = v4.z;
+      v[3] = v4.w;
     } else {
 #pragma unroll
-      for (int r = 0; r < 4; ++r) s[g][r] = (i0 + r < N) ? __ldg(sp + i0 + r) : 0.f;
+      for (int r = 0; r < 4; ++r) v[r] = (i0 + r < N) ? __ldg(sp + i0 + r) : 0.f;
     }
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
       const int i = i0 + r;
-      float v = s[g][r];
-      if (!isfinite(v)) {
+      if (!isfinite(v[r])) {
         bad = bad || (i < N);
-        v = 0.f;
+        v[r] = 0.f;
       }
-      s[g][r] = v + 0.0f;
-      if (i < N && !EBD_CAND(i)) cert |= 1ull << (4 * g + r);  // protected
+      v[r] += 0.0f;
+      if (i < N && !is_cand(i)) cert |= 1ull << (4 * g + r);  // protected
     }
+    s4[g * kRegThreads + tid] = make_float4(v[0], v[1], v[2], v[3]);
   }
+
 
   // ---- E1: top-k_head among the unprotected tokens ------------------------
   if (k > 0 && k < n_cand) {
     unsigned prefix = 0u, maskbits = 0u, remaining = (unsigned)k;
+#pragma unroll 1
     for (int shift = 24; shift >= 0; shift -= 8) {
       for (int j = tid; j < 256; j += kRegThreads) sh.hist[j] = 0u;
       __syncthreads();
-#pragma unroll
+#pragma unroll 1
       for (int g = 0; g < JG; ++g) {
+        const float4 v4 = s4[g * kRegThreads + tid];
+        const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
 #pragma unroll
         for (int r = 0; r < 4; ++r) {
-          if (!EBD_CAND(EBD_TOK(g, r))) continue;
-          const uint32_t key = orderable_key(s[g][r]);
-          if ((key & maskbits) == prefix) atomicAdd(&sh.hist[(key >> shift) & 255u], 1u);
+          const uint32_t key = orderable_key(vv[r]);
+          const bool in = is_cand(tok(g, r)) && (key & maskbits) == prefix;
+          // one atomic per distinct bin per warp: the hot bins of skewed
+          // scores would otherwise serialise every lane
+          if (!__any_sync(0xffffffffu, in)) continue;
+          const uint32_t bin = in ? ((key >> shift) & 255u) : 256u;
+          const unsigned peers = __match_any_sync(0xffffffffu, bin);
+          if (in && lane == __ffs(peers) - 1) atomicAdd(&sh.hist[bin], (unsigned)__popc(peers));
         }
       }
       __syncthreads();
@@ -540,18 +598,20 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_reg_kernel(Select
       maskbits |= 255u << shift;
     }
     uint64_t eq = 0ull;
-#pragma unroll
+#pragma unroll 1
     for (int g = 0; g < JG; ++g) {
+      const float4 v4 = s4[g * kRegThreads + tid];
+      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
 #pragma unroll
       for (int r = 0; r < 4; ++r) {
-        if (!EBD_CAND(EBD_TOK(g, r))) continue;
-        const uint32_t key = orderable_key(s[g][r]);
+        if (!is_cand(tok(g, r))) continue;
+        const uint32_t key = orderable_key(vv[r]);
         if (key > prefix) cert |= 1ull << (4 * g + r);
         else if (key == prefix) eq |= 1ull << (4 * g + r);
       }
     }
-    ordered_scan<JG>(eq, sh);
-#pragma unroll
+    ordered_scan(eq, JG, sh);
+#pragma unroll 1
     for (int g = 0; g < JG; ++g) {
       int run = sh.off[g][warp] + lane_prefix(eq, g);
 #pragma unroll
@@ -564,13 +624,15 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_reg_kernel(Select
       }
     }
   } else if (k > 0) {
-#pragma unroll
+#pragma unroll 1
     for (int g = 0; g < JG; ++g)
 #pragma unroll
       for (int r = 0; r < 4; ++r)
-        if (EBD_TOK(g, r) < N) cert |= 1ull << (4 * g + r);
+        if (tok(g, r) < N) cert |= 1ull << (4 * g + r);
   }
-#define EBD_TAIL(g, r) (EBD_TOK(g, r) < N && !((cert >> (4 * (g) + (r))) & 1ull))
+  auto is_tail = [&](int g, int r) {
+    return tok(g, r) < N && !((cert >> (4 * g + r)) & 1ull);
+  };
 
   // ---- E2: inclusion probabilities on the tail ---------------------------
   const int n_cert = n_prot + k;
@@ -578,16 +640,17 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_reg_kernel(Select
   const int m = min(max(a.budget - n_cert, 0), nT);
   float smax = -INFINITY, sminpos = INFINITY, spos = 0.f;
   int npos = 0;
-#pragma unroll
+#pragma unroll 1
   for (int g = 0; g < JG; ++g) {
+    const float4 v4 = s4[g * kRegThreads + tid];
+    const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
-      if (!EBD_TAIL(g, r)) continue;
-      const float v = s[g][r];
-      smax = fmaxf(smax, v);
-      if (v > 0.f) {
-        sminpos = fminf(sminpos, v);
-        spos += v;
+      if (!is_tail(g, r)) continue;
+      smax = fmaxf(smax, vv[r]);
+      if (vv[r] > 0.f) {
+        sminpos = fminf(sminpos, vv[r]);
+        spos += vv[r];
         ++npos;
       }
     }
@@ -595,119 +658,131 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_reg_kernel(Select
   smax = warp_max(smax);
   sminpos = warp_min(sminpos);
   npos = warp_sum(npos);
-  double spos_d = warp_sum((double)spos);
+  spos = warp_sum(spos);
   __syncthreads();
   if (lane == 0) {
     sh.rf[0][warp] = smax;
     sh.rf[1][warp] = sminpos;
+    sh.rf[2][warp] = spos;
     sh.ri[0][warp] = npos;
-    sh.rd[warp] = spos_d;
   }
   __syncthreads();
-  smax = sh.rf[0][0];
-  sminpos = sh.rf[1][0];
-  npos = 0;
-  spos_d = 0.0;
-#pragma unroll
-  for (int w = 0; w < kRegWarps; ++w) {
-    smax = fmaxf(smax, sh.rf[0][w]);
-    sminpos = fminf(sminpos, sh.rf[1][w]);
-    npos += sh.ri[0][w];
-    spos_d += sh.rd[w];
+  combine_stats(sh);
+  __syncthreads();
+  // Scalar decisions are taken once, by thread 0, and broadcast: the fp64
+  // arithmetic they use would otherwise run on every thread.
+  if (tid == 0) {
+    const float smax_b = sh.res_f[0], sminpos_b = sh.res_f[1];
+    const int npos_b = sh.res_i[0];
+    int md = kPiLinear;
+    if (nT == 0 || (float)m <= eps * (float)nT) md = kPiFloor;
+    else if ((float)m >= (float)npos_b + eps * (float)(nT - npos_b)) md = kPiAll;
+    sh.mode = md;
+    sh.stop = md != kPiLinear;
+    if (md == kPiLinear) {
+      sh.lo = logf(eps / smax_b);
+      sh.hi = logf(1.f / sminpos_b);
+      sh.c = fminf(fmaxf((float)((double)m / sh.res_d), expf(sh.lo)), expf(sh.hi));
+    } else {
+      sh.c = 0.f;
+    }
   }
-
-  int mode = kPiLinear;
-  float c = 0.f;
-  if (nT == 0 || (float)m <= eps * (float)nT) {
-    mode = kPiFloor;
-  } else if ((float)m >= (float)npos + eps * (float)(nT - npos)) {
-    mode = kPiAll;
-  } else {
-    float lo = logf(eps / smax), hi = logf(1.f / sminpos);
-    c = fminf(fmaxf((float)((double)m / spos_d), expf(lo)), expf(hi));
-    for (int it = 0; it < a.iters; ++it) {
-      int nhi = 0, nlo = 0;
-      float smid = 0.f;
+  __syncthreads();
+  const int mode = sh.mode;
+  float c = sh.c;
+#pragma unroll 1
+  for (int it = 0; it < a.iters && !sh.stop; ++it) {
+    int nhi = 0, nlo = 0;
+    float smid = 0.f;
+#pragma unroll 1
+    for (int g = 0; g < JG; ++g) {
+      const float4 v4 = s4[g * kRegThreads + tid];
+      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
 #pragma unroll
-      for (int g = 0; g < JG; ++g) {
-#pragma unroll
-        for (int r = 0; r < 4; ++r) {
-          if (!EBD_TAIL(g, r)) continue;
-          const float t = c * s[g][r];
-          if (t >= 1.f) ++nhi;
-          else if (t <= eps) ++nlo;
-          else smid += s[g][r];
-        }
+      for (int r = 0; r < 4; ++r) {
+        if (!is_tail(g, r)) continue;
+        const float t = c * vv[r];
+        if (t >= 1.f) ++nhi;
+        else if (t <= eps) ++nlo;
+        else smid += vv[r];
       }
-      nhi = warp_sum(nhi);
-      nlo = warp_sum(nlo);
-      double smid_d = warp_sum((double)smid);
-      __syncthreads();
-      if (lane == 0) {
-        sh.ri[0][warp] = nhi;
-        sh.ri[1][warp] = nlo;
-        sh.rd[warp] = smid_d;
-      }
-      __syncthreads();
-      nhi = 0;
-      nlo = 0;
-      smid_d = 0.0;
-#pragma unroll
-      for (int w = 0; w < kRegWarps; ++w) {
-        nhi += sh.ri[0][w];
-        nlo += sh.ri[1][w];
-        smid_d += sh.rd[w];
-      }
-      const double gval = nhi + (double)eps * nlo + (double)c * smid_d;
+    }
+    nhi = warp_sum(nhi);
+    nlo = warp_sum(nlo);
+    smid = warp_sum(smid);
+    __syncthreads();
+    if (lane == 0) {
+      sh.ri[0][warp] = nhi;
+      sh.ri[1][warp] = nlo;
+      sh.rf[0][warp] = smid;
+    }
+    __syncthreads();
+    combine_partition(sh);
+    if (tid == 0) {
+      const int nh = sh.res_i[0], nl = sh.res_i[1];
+      const double smid_d = sh.res_d;
+      const double gval = nh + (double)eps * nl + (double)c * smid_d;
+      float lo = sh.lo, hi = sh.hi;
       if (gval < (double)m) lo = fmaxf(lo, logf(c));
       else hi = fminf(hi, logf(c));
-      const double clin = smid_d > 0.0 ? ((double)m - nhi - (double)eps * nlo) / smid_d : -1.0;
+      const double clin = smid_d > 0.0 ? ((double)m - nh - (double)eps * nl) / smid_d : -1.0;
       if (clin > 0.0 && fabs(clin - (double)c) <= 1e-6 * (double)c) {
-        c = (float)clin;  // the partition at c reproduces its own solve
-        break;
+        sh.c = (float)clin;  // the partition at c reproduces its own solve
+        sh.stop = 1;
+      } else {
+        float next;
+        const float lcl = clin > 0.0 ? logf((float)clin) : -INFINITY;
+        if (clin > 0.0 && lcl > lo && lcl < hi) next = (float)clin;
+        else next = expf(0.5f * (lo + hi));
+        if (next == c) sh.stop = 1;
+        sh.c = next;
       }
-      float next;
-      const float lcl = clin > 0.0 ? logf((float)clin) : -INFINITY;
-      if (clin > 0.0 && lcl > lo && lcl < hi) next = (float)clin;
-      else next = expf(0.5f * (lo + hi));
-      if (next == c) break;
-      c = next;
+      sh.lo = lo;
+      sh.hi = hi;
     }
+    __syncthreads();
+    c = sh.c;
   }
 
   // ---- E3 + E4a: draws and ordered compaction of (index, log 1/pi) --------
   const bool compact = a.n_kept != nullptr;
   uint64_t keep = 0ull;
-#pragma unroll
+#pragma unroll 1
   for (int g = 0; g < JG; ++g) {
+    const float4 v4 = s4[g * kRegThreads + tid];
+    const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
     bool any_tail = false;
 #pragma unroll
-    for (int r = 0; r < 4; ++r) any_tail = any_tail || EBD_TAIL(g, r);
+    for (int r = 0; r < 4; ++r) any_tail = any_tail || is_tail(g, r);
     uint4 w = make_uint4(0u, 0u, 0u, 0u);
-    if (compact && __any_sync(0xffffffffu, any_tail)) w = draw_block(a.seed, a.layer, b, kvh, g * 512 + tid);
+    if (compact && __any_sync(0xffffffffu, any_tail))
+      w = draw_block(a.seed, a.layer, b, kvh, g * kRegThreads + tid);
+    const uint32_t wr[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
-      const int i = EBD_TOK(g, r);
+      const int i = tok(g, r);
       if (i >= N) continue;
       const bool ct = (cert >> (4 * g + r)) & 1ull;
-      const float pi = ct ? 1.f : tail_pi(s[g][r], mode, c, eps);
+      const float pi = ct ? 1.f : tail_pi(vv[r], mode, c, eps);
       if (a.pi_out) a.pi_out[(size_t)unit * N + i] = pi;
       if (a.mask_out) a.mask_out[(size_t)unit * N + i] = ct ? 1 : 0;
-      if (compact && (ct || word_to_uniform(word_of(w, r)) < pi)) keep |= 1ull << (4 * g + r);
+      if (compact && (ct || word_to_uniform(wr[r]) < pi)) keep |= 1ull << (4 * g + r);
     }
   }
   if (compact) {
-    const int total = ordered_scan<JG>(keep, sh);
-#pragma unroll
+    const int total = ordered_scan(keep, JG, sh);
+#pragma unroll 1
     for (int g = 0; g < JG; ++g) {
       int p = sh.off[g][warp] + lane_prefix(keep, g);
+      const float4 v4 = s4[g * kRegThreads + tid];
+      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
 #pragma unroll
       for (int r = 0; r < 4; ++r) {
         const uint64_t bit = 1ull << (4 * g + r);
         if (!(keep & bit)) continue;
         if (p < a.cap) {
-          const float pi = (cert & bit) ? 1.f : tail_pi(s[g][r], mode, c, eps);
-          a.idx_c[(size_t)unit * a.cap + p] = EBD_TOK(g, r);
+          const float pi = (cert & bit) ? 1.f : tail_pi(vv[r], mode, c, eps);
+          a.idx_c[(size_t)unit * a.cap + p] = tok(g, r);
           a.logw_c[(size_t)unit * a.cap + p] = pi >= 1.f ? 0.f : -logf(pi);
         }
         ++p;
@@ -719,9 +794,6 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_reg_kernel(Select
     }
   }
   if (__syncthreads_or(bad) && tid == 0) raise_status(a.dev_status, EBD_DEV_NONFINITE);
-#undef EBD_TAIL
-#undef EBD_CAND
-#undef EBD_TOK
 }
 
 // E4b: copy kept K and V rows (16-byte chunks, `cpr` chunks per row).
@@ -827,13 +899,14 @@ static ebd_status launch_select(const ebd_design* d, const float* scores, float*
   a.dev_status = dev_status;
   a.vec4 = (((uintptr_t)scores & 15u) == 0 && (d->n_ctx & 3) == 0) ? 1 : 0;
   const int units = d->batch * d->n_kv_heads;
-  const int groups = (d->n_ctx + 2047) / 2048;
+  const int groups = (d->n_ctx + kGroupTokens - 1) / kGroupTokens;
   if (groups <= kRegMaxGroups) {
-    if (groups <= 1) evict_select_reg_kernel<1><<<units, kRegThreads, 0, stream>>>(a);
-    else if (groups <= 2) evict_select_reg_kernel<2><<<units, kRegThreads, 0, stream>>>(a);
-    else if (groups <= 4) evict_select_reg_kernel<4><<<units, kRegThreads, 0, stream>>>(a);
-    else if (groups <= 8) evict_select_reg_kernel<8><<<units, kRegThreads, 0, stream>>>(a);
-    else evict_select_reg_kernel<16><<<units, kRegThreads, 0, stream>>>(a);
+    const size_t smem = (size_t)groups * kRegThreads * sizeof(float4);
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(evict_select_smem_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem) != cudaSuccess)
+      return EBD_ERR_CUDA;
+    evict_select_smem_kernel<<<units, kRegThreads, smem, stream>>>(a, groups);
     return launch_status();
   }
   const size_t smem = (size_t)((d->n_ctx + 31) / 32) * 4;
