@@ -1012,7 +1012,7 @@ extern "C" ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const
     float* ws_scores = (float*)workspace;
     float* ws_lse = (float*)((char*)workspace + align_up(units * design->n_ctx * sizeof(float), 256));
     st = launch_score(dtype, design->batch, design->n_kv_heads, d, design->n_ctx, n_obs, q_obs, K,
-                      ws_scores, ws_lse, s);
+                      ws_scores, ws_lse, dev_status, s);
     if (st != EBD_OK) return st;
     sc = ws_scores;
   }

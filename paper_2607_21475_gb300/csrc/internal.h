@@ -20,9 +20,15 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 int sm_count();
 
 // E0: accumulated attention scores into `scores` using `workspace` for the
-// per-row log-sum-exp.  Arguments validated by the caller.
+// per-row log-sum-exp.  Arguments validated by the caller; dev_status nullable.
 ebd_status launch_score(ebd_dtype dtype, int batch, int n_kv_heads, int head_dim, int n_ctx,
                         int n_obs, const void* q_obs, const void* K, float* scores,
-                        float* lse_ws, cudaStream_t stream);
+                        float* lse_ws, int32_t* dev_status, cudaStream_t stream);
+
+// Tensor-core E0 (score_mma.cu): bf16, head_dim 64/128, 16-byte aligned inputs.
+bool score_mma_supported(ebd_dtype dtype, int head_dim, const void* q_obs, const void* K);
+ebd_status launch_score_mma(int units, int head_dim, int n_ctx, int n_obs, const void* q_obs,
+                            const void* K, float* scores, float* lse, int32_t* dev_status,
+                            cudaStream_t s);
 
 }  // namespace ebd

@@ -124,9 +124,12 @@ static ebd_status launch_score_t(int units, int n_ctx, int n_obs, const void* q_
 
 ebd_status launch_score(ebd_dtype dtype, int batch, int n_kv_heads, int head_dim, int n_ctx,
                         int n_obs, const void* q_obs, const void* K, float* scores,
-                        float* lse_ws, cudaStream_t s) {
+                        float* lse_ws, int32_t* dev_status, cudaStream_t s) {
   const int units = batch * n_kv_heads;
   if (units > 0x7fffffff || n_obs > 4096 || n_obs < 1) return EBD_ERR_UNSUPPORTED;
+  if (score_mma_supported(dtype, head_dim, q_obs, K) && units <= 65535 &&
+      (n_ctx + 63) / 64 <= 65535)
+    return launch_score_mma(units, head_dim, n_ctx, n_obs, q_obs, K, scores, lse_ws, dev_status, s);
   if ((n_obs + kLseWarps - 1) / kLseWarps > 65535 || (n_ctx + kColThreads - 1) / kColThreads > 65535)
     return EBD_ERR_UNSUPPORTED;
   if (dtype == EBD_BF16) {
@@ -158,5 +161,5 @@ extern "C" ebd_status ebd_score(ebd_dtype dtype, int32_t batch, int32_t n_kv_hea
   if (!workspace || ws_bytes < ebd_score_workspace_bytes(batch, n_kv_heads, n_obs))
     return EBD_ERR_CAPACITY;
   return launch_score(dtype, batch, n_kv_heads, head_dim, n_ctx, n_obs, q_obs, K, scores,
-                      (float*)workspace, (cudaStream_t)stream);
+                      (float*)workspace, nullptr, (cudaStream_t)stream);
 }
