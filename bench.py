@@ -244,7 +244,7 @@ class Path:
                                   dtype=torch.uint8, device=dev)
         self.phases = (["score"] if self.scored else []) + ["select", "gather", "decode"]
         self.launches = {"score": 2, "select": 1, "gather": 1, "decode": 2}
-        self.use_graph = use_graph and L > 1
+        self.use_graph = use_graph
         self.graphs = {}
 
     # one phase over every layer

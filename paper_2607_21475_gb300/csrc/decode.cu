@@ -157,24 +157,31 @@ __global__ void __launch_bounds__(kGenThreads) decode_generic_kernel(DecodeArgs 
   }
 }
 
-// Merge the partial records of one query head and finish Eq. (3), Theorem 2, Eq. (4).
-// CUDA-core path: records u*splits .. u*splits + splits - 1.  Tensor-core
-// path: records u + gw for every consumer warp gw whose tile range meets
-// unit u (none for an empty unit).
+// Merge the partial records of one query head and finish Eq. (3), Theorem 2,
+// Eq. (4).  One warp per query head: lanes take 32 records at a time (scale
+// factors and scalar moments), then every lane streams its D/32 columns of each
+// record.  CUDA-core path: records u*splits .. u*splits + splits - 1.
+// Tensor-core path: records u + gw for every working warp gw whose tile range
+// meets unit u (none for an empty unit).
+constexpr int kReduceWarps = 4;
+
 template <int D>
-__global__ void __launch_bounds__(D) decode_reduce_kernel(ReduceArgs a) {
+__global__ void __launch_bounds__(kReduceWarps * 32) decode_reduce_kernel(ReduceArgs a,
+                                                                          int n_heads) {
   constexpr int REC = rec_floats(D);
-  __shared__ float red[2][D / 32];
-  const int hq = blockIdx.x;
+  constexpr int PER = D / 32;
+  const int lane = threadIdx.x & 31;
+  const int hq = blockIdx.x * kReduceWarps + (threadIdx.x >> 5);
+  if (hq >= n_heads) return;
   const int G = a.group;
   const int unit = hq / G, g = hq - unit * G;
-  const int e = threadIdx.x;
   long long first = (long long)unit * a.splits;
   int count = a.splits;
   if (a.tile_off) {
     const long long t0 = a.tile_off[unit], t1 = a.tile_off[unit + 1];
-    const long long Ta = a.tile_off[gridDim.x / G];
-    const long long W = a.warps < Ta ? a.warps : Ta;
+    const long long Ta = a.tile_off[n_heads / G];
+    long long W = Ta / a.min_tiles > 0 ? Ta / a.min_tiles : 1;
+    if (a.warps < W) W = a.warps;
     count = 0;
     if (t1 > t0) {
       const long long gf = ((t0 + 1) * W - 1) / Ta;
@@ -183,13 +190,15 @@ __global__ void __launch_bounds__(D) decode_reduce_kernel(ReduceArgs a) {
       count = (int)(gl - gf + 1);
     }
   }
-  const float* P = a.part + ((size_t)first * G + g) * REC;
-  const size_t sstride = (size_t)G * REC;
+  const size_t slot = (size_t)G * REC;
+  const float* R0 = a.part + ((size_t)first * G + g) * REC;
   float Mx = -INFINITY;
-  for (int s = 0; s < count; ++s) Mx = fmaxf(Mx, P[s * sstride + kRecM]);
+  for (int s = lane; s < count; s += 32) Mx = fmaxf(Mx, R0[s * slot + kRecM]);
+  Mx = warp_max(Mx);
   if (Mx == -INFINITY) {  // empty unit
-    a.y[(size_t)hq * D + e] = 0.f;
-    if (e == 0) {
+#pragma unroll
+    for (int e = 0; e < PER; ++e) a.y[(size_t)hq * D + PER * lane + e] = 0.f;
+    if (lane == 0) {
       a.lse[hq] = -INFINITY;
       a.var[hq] = 0.f;
       a.b_t[hq] = 0.f;
@@ -197,36 +206,68 @@ __global__ void __launch_bounds__(D) decode_reduce_kernel(ReduceArgs a) {
     }
     return;
   }
-  float l = 0.f, U = 0.f, A2 = 0.f, cmax = 0.f, umax = 0.f, o = 0.f, a1 = 0.f;
-  for (int s = 0; s < count; ++s) {
-    const float* R = P + s * sstride;
-    const float Ms = R[kRecM];
-    if (Ms == -INFINITY) continue;
-    const float f = expf(Ms - Mx), f2 = f * f;
-    l += f * R[kRecL];
-    U += f2 * R[kRecU];
-    A2 += f2 * R[kRecA2];
-    cmax = fmaxf(cmax, f * R[kRecCmax]);
-    umax = fmaxf(umax, f * R[kRecUmax]);
-    o += f * R[kRecHead + e];
-    a1 += f2 * R[kRecHead + D + e];
-  }
-  const float y = o / l;
-  a.y[(size_t)hq * D + e] = y;
-  float yy = warp_sum(y * y), ya = warp_sum(y * a1);
-  if ((e & 31) == 0) {
-    red[0][e >> 5] = yy;
-    red[1][e >> 5] = ya;
-  }
-  __syncthreads();
-  if (e == 0) {
-    yy = 0.f;
-    ya = 0.f;
+  float l = 0.f, U = 0.f, A2 = 0.f, cmax = 0.f, umax = 0.f;
+  float o[PER], a1[PER];
 #pragma unroll
-    for (int w = 0; w < D / 32; ++w) {
-      yy += red[0][w];
-      ya += red[1][w];
+  for (int e = 0; e < PER; ++e) o[e] = a1[e] = 0.f;
+  for (int s0 = 0; s0 < count; s0 += 32) {
+    float f = 0.f;
+    if (s0 + lane < count) {
+      const float* R = R0 + (s0 + lane) * slot;
+      const float Ms = R[kRecM];
+      if (Ms != -INFINITY) {
+        f = expf(Ms - Mx);
+        const float f2 = f * f;
+        l = fmaf(f, R[kRecL], l);
+        U = fmaf(f2, R[kRecU], U);
+        A2 = fmaf(f2, R[kRecA2], A2);
+        cmax = fmaxf(cmax, f * R[kRecCmax]);
+        umax = fmaxf(umax, f * R[kRecUmax]);
+      }
     }
+    const int nrec = min(32, count - s0);
+#pragma unroll 4
+    for (int k = 0; k < nrec; ++k) {
+      const float fk = __shfl_sync(0xffffffffu, f, k);
+      const float f2k = fk * fk;
+      const float* Rk = R0 + (s0 + k) * slot + kRecHead + PER * lane;
+      if constexpr (PER == 4) {
+        const float4 ov = *reinterpret_cast<const float4*>(Rk);
+        const float4 av = *reinterpret_cast<const float4*>(Rk + D);
+        o[0] = fmaf(fk, ov.x, o[0]);
+        o[1] = fmaf(fk, ov.y, o[1]);
+        o[2] = fmaf(fk, ov.z, o[2]);
+        o[3] = fmaf(fk, ov.w, o[3]);
+        a1[0] = fmaf(f2k, av.x, a1[0]);
+        a1[1] = fmaf(f2k, av.y, a1[1]);
+        a1[2] = fmaf(f2k, av.z, a1[2]);
+        a1[3] = fmaf(f2k, av.w, a1[3]);
+      } else {
+        const float2 ov = *reinterpret_cast<const float2*>(Rk);
+        const float2 av = *reinterpret_cast<const float2*>(Rk + D);
+        o[0] = fmaf(fk, ov.x, o[0]);
+        o[1] = fmaf(fk, ov.y, o[1]);
+        a1[0] = fmaf(f2k, av.x, a1[0]);
+        a1[1] = fmaf(f2k, av.y, a1[1]);
+      }
+    }
+  }
+  l = warp_sum(l);
+  U = warp_sum(U);
+  A2 = warp_sum(A2);
+  cmax = warp_max(cmax);
+  umax = warp_max(umax);
+  float yy = 0.f, ya = 0.f;
+#pragma unroll
+  for (int e = 0; e < PER; ++e) {
+    const float yv = o[e] / l;
+    a.y[(size_t)hq * D + PER * lane + e] = yv;
+    yy = fmaf(yv, yv, yy);
+    ya = fmaf(yv, a1[e], ya);
+  }
+  yy = warp_sum(yy);
+  ya = warp_sum(ya);
+  if (lane == 0) {
     const float ynorm = sqrtf(yy);
     const float var = fmaxf(0.f, (A2 - 2.f * ya + yy * U) / (l * l));
     a.lse[hq] = Mx + logf(l);
@@ -444,23 +485,12 @@ extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32
   a.dev_status = dev_status;
 
   const bool fast = plan.fast && fast_decode_usable(a, (int)units);
-  ebd_status st;
-  if (fast)
-    st = launch_fast_decode(dtype, head_dim, plan, a, (int)units, s);
-  else
-    st = dispatch_generic(false, dtype, head_dim, a, (int)units, s);
-  if (st != EBD_OK) return st;
-
   ReduceArgs r;
   r.part = (const float*)workspace;
   r.splits = plan.splits;
   r.tile_off = nullptr;
   r.warps = 0;
-  if (fast) {
-    r.tile_off = (const int32_t*)workspace;
-    r.part = (const float*)((const char*)workspace + fast_decode_records_offset((int)units));
-    r.warps = fast_decode_warps(plan);
-  }
+  r.min_tiles = 1;
   r.group = group;
   r.y = y;
   r.lse = lse;
@@ -471,13 +501,25 @@ extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32
   r.eps0 = eps0;
   r.exact = range_mode == EBD_RANGE_EXACT;
   const int n_heads = (int)(units * group);
+  ebd_status st;
+  if (fast) {
+    st = launch_fast_decode(dtype, head_dim, plan, a, (int)units, s);
+    r.tile_off = (const int32_t*)workspace;
+    r.part = (const float*)((const char*)workspace + fast_decode_records_offset((int)units));
+    r.warps = fast_decode_warps(plan);
+    r.min_tiles = fast_decode_min_tiles_per_warp();
+  } else {
+    st = dispatch_generic(false, dtype, head_dim, a, (int)units, s);
+  }
+  if (st != EBD_OK) return st;
+  const int rblocks = (n_heads + kReduceWarps - 1) / kReduceWarps;
   if (head_dim == 128)
-    decode_reduce_kernel<128><<<n_heads, 128, 0, s>>>(r);
+    decode_reduce_kernel<128><<<rblocks, kReduceWarps * 32, 0, s>>>(r, n_heads);
   else
-    decode_reduce_kernel<64><<<n_heads, 64, 0, s>>>(r);
+    decode_reduce_kernel<64><<<rblocks, kReduceWarps * 32, 0, s>>>(r, n_heads);
   st = launch_status();
-  if (st != EBD_OK || !r.exact) return st;
-
+  if (st != EBD_OK) return st;
+  if (!r.exact) return EBD_OK;
   // exact range term: second pass over the tail rows, then the radius
   a.splits = plan.splits;
   a.tokens_per_split = plan.tokens_per_split;

@@ -10,10 +10,11 @@
 namespace ebd {
 
 // One partial record per (unit, split slot, query head of the group), floats:
-//   [M, l, U, A2, cmax, umax, o[0..D), A1[0..D)]
-// w-terms (l, o, cmax, umax) scale by e^(M_old - M_new) on a merge, u-terms
-// (U, A2, A1) by its square.  An empty record has M = -inf and zeros.
-enum : int { kRecM = 0, kRecL = 1, kRecU = 2, kRecA2 = 3, kRecCmax = 4, kRecUmax = 5, kRecHead = 6 };
+//   [M, l, U, A2, cmax, umax, pad, pad, o[0..D), A1[0..D)]
+// (16-byte multiple, so o and A1 can be read as float4).  w-terms (l, o,
+// cmax, umax) scale by e^(M_old - M_new) on a merge, u-terms (U, A2, A1) by
+// its square.  An empty record has M = -inf and zeros.
+enum : int { kRecM = 0, kRecL = 1, kRecU = 2, kRecA2 = 3, kRecCmax = 4, kRecUmax = 5, kRecHead = 8 };
 
 __host__ __device__ constexpr int rec_floats(int D) { return kRecHead + 2 * D; }
 __host__ __device__ constexpr bool rec_is_squared(int e, int D) {
@@ -42,7 +43,8 @@ struct ReduceArgs {
   const float* part;
   int splits;                // CUDA-core path: records per unit
   const int32_t* tile_off;   // tensor-core path: active-tile prefix (null otherwise)
-  long long warps;           // tensor-core path: consumer warps in the grid
+  long long warps;           // tensor-core path: warps in the grid
+  int min_tiles;             // tensor-core path: minimum tiles per working warp
   int group;
   float* y;
   float* lse;
@@ -71,7 +73,9 @@ bool fast_decode_usable(const DecodeArgs& a, int units);
 long long fast_decode_warps(const DecodePlan& p);
 size_t fast_decode_records_offset(int units);
 void fast_decode_plan(DecodePlan& p, long long units, int group, int head_dim, int capacity);
+// Plan + decode kernels; records for the reduce kernel.
 ebd_status launch_fast_decode(ebd_dtype dtype, int head_dim, const DecodePlan& plan,
                               const DecodeArgs& a, int units, cudaStream_t stream);
+int fast_decode_min_tiles_per_warp();
 
 }  // namespace ebd

@@ -11,7 +11,7 @@
 // split into equal contiguous ranges, one per warp.  A warp's range
 // crosses at most a few units; for each unit it meets it writes one partial
 // record, at index (unit + global warp), so records never collide and no
-// scratch needs clearing.
+// scratch needs clearing.  The reduce kernel merges the records of a unit.
 //
 // Per tile and warp:
 //   S[16 x 16]  = Qpad[16 x d] . K_tile^T       (rows 0..G-1 = query heads,
@@ -52,6 +52,7 @@ constexpr int kMmaStagesPerWarp = 3;
 constexpr int kMmaStages = kMmaConsumers * kMmaStagesPerWarp;
 constexpr int kMmaThreads = kMmaConsumers * 32;
 constexpr float kRescaleLog2 = 8.f;
+constexpr int kMinTilesPerWarp = 4;
 
 template <int D>
 struct MmaLayout {
@@ -94,6 +95,8 @@ __device__ __forceinline__ int next_unit(const int32_t* tile_off, int u) {
   return u;
 }
 
+// Exclusive prefix of active (16-token) tiles per unit: tile_off[u], with
+// tile_off[units] = the total.
 __global__ void decode_tile_plan_kernel(const int32_t* __restrict__ n_kept, int units, int cap,
                                         int32_t* __restrict__ tile_off) {
   __shared__ int warp_tot[32];
@@ -156,9 +159,12 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
   const int Ta = __ldg(a.tile_off + units);
   if (Ta == 0) return;
   const long long Wall = (long long)gridDim.x * kMmaConsumers;
-  const long long W = Wall < Ta ? Wall : Ta;  // every working warp gets >= 1 tile
+  // working warps: every one gets >= kMinTilesPerWarp tiles (bounded merge work)
+  const long long Wcap = Ta / kMinTilesPerWarp > 0 ? Ta / kMinTilesPerWarp : 1;
+  const long long W = Wall < Wcap ? Wall : Wcap;
 
-  const long long gw = (long long)blockIdx.x * kMmaConsumers + warp;
+  // global warp index, consecutive indices on different SMs
+  const long long gw = (long long)warp * gridDim.x + blockIdx.x;
   if (gw >= W) return;
   const int tb = (int)(gw * Ta / W);
   const int te = (int)((gw + 1) * Ta / W);
@@ -436,7 +442,7 @@ void fast_decode_plan(DecodePlan& p, long long units, int group, int head_dim, i
   (void)capacity;
   p.ctas = sm_count();
   const long long W = (long long)p.ctas * kMmaConsumers;
-  p.ws_bytes = align_up((size_t)(units + 1) * sizeof(int32_t), 256) +
+  p.ws_bytes = fast_decode_records_offset((int)units) +
                align_up((size_t)(units + W) * group * rec_floats(head_dim) * sizeof(float), 256);
 }
 
@@ -444,6 +450,9 @@ static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
 long long fast_decode_warps(const DecodePlan& p) { return (long long)p.ctas * kMmaConsumers; }
 
+int fast_decode_min_tiles_per_warp() { return kMinTilesPerWarp; }
+
+// Workspace: tile_off [units + 1] | records.
 size_t fast_decode_records_offset(int units) {
   return align_up((size_t)(units + 1) * sizeof(int32_t), 256);
 }
