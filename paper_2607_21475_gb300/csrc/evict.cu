@@ -431,9 +431,9 @@ __device__ __forceinline__ void combine_partition(RegScratch& sh) {
 
 // Exclusive prefix, over the lanes of this warp, of the number of set bits in
 // 4-bit group g of `flags`.
-__device__ __forceinline__ int lane_prefix(uint64_t flags, int g) {
+__device__ __forceinline__ int lane_prefix(uint32_t flags, int g) {
   const int lane = threadIdx.x & 31;
-  const int c = __popc((unsigned)((flags >> (4 * g)) & 0xFull));
+  const int c = __popc((flags >> (4 * g)) & 0xFu);
   int incl = c;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
@@ -447,12 +447,12 @@ __device__ __forceinline__ int lane_prefix(uint64_t flags, int g) {
 // g*4096 + 4*tid + r): afterwards sh.off[g][w] is the number of set bits at
 // tokens before warp w's slice of group g; returns the block total.  The rank
 // of a token is sh.off[g][warp] + lane_prefix(flags, g) + its rank in the thread.
-__device__ __forceinline__ int ordered_scan(uint64_t flags, int JG, RegScratch& sh) {
+__device__ __forceinline__ int ordered_scan(uint32_t flags, int JG, RegScratch& sh) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   __syncthreads();  // previous readers of sh.off / sh.total are done
 #pragma unroll 1
   for (int g = 0; g < JG; ++g) {
-    const int c = __popc((unsigned)((flags >> (4 * g)) & 0xFull));
+    const int c = __popc((flags >> (4 * g)) & 0xFu);
     const int tot = warp_sum(c);
     if (lane == 0) sh.tot[g][warp] = tot;
   }
@@ -491,6 +491,8 @@ __device__ __forceinline__ int ordered_scan(uint64_t flags, int JG, RegScratch& 
 
 __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(SelectArgs a, int JG) {
   extern __shared__ float4 s4[];  // [JG][1024]: scores of thread t, group g at s4[g*1024 + t]
+  // followed by the per-warp top-digit histograms [kRegWarps][256]
+  unsigned* whist = reinterpret_cast<unsigned*>(s4 + JG * kRegThreads);
   __shared__ RegScratch sh;
   const int unit = blockIdx.x;
   const int b = unit / a.n_kv_heads;
@@ -509,7 +511,7 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
 
   // ---- load: sanitise, fold -0 onto +0, protected positions -------------------
   bool bad = false;
-  uint64_t cert = 0ull;
+  uint32_t cert = 0u, valid = 0u;
   // every group's load in flight before the first use
 #pragma unroll
   for (int g = 0; g < kRegMaxGroups; ++g) {
@@ -534,33 +536,53 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
         v[r] = 0.f;
       }
       v[r] += 0.0f;
-      if (i < N && !is_cand(i)) cert |= 1ull << (4 * g + r);  // protected
+      if (i < N) valid |= 1u << (4 * g + r);
+      if (i < N && !is_cand(i)) cert |= 1u << (4 * g + r);  // protected
     }
     s4[g * kRegThreads + tid] = make_float4(v[0], v[1], v[2], v[3]);
   }
 
 
   // ---- E1: top-k_head among the unprotected tokens ------------------------
+  // MSB-first radix select over 8-bit digits of the order-preserving keys.
+  // `live` holds the tokens whose key still matches the chosen prefix; after
+  // each digit, tokens above it join the certainty set and tokens below it
+  // drop out, so later passes touch only the few tokens still in contention.
   if (k > 0 && k < n_cand) {
-    unsigned prefix = 0u, maskbits = 0u, remaining = (unsigned)k;
+    uint32_t live = valid & ~cert;  // the unprotected tokens
+    unsigned remaining = (unsigned)k;
 #pragma unroll 1
     for (int shift = 24; shift >= 0; shift -= 8) {
       for (int j = tid; j < 256; j += kRegThreads) sh.hist[j] = 0u;
       __syncthreads();
+      if (shift == 24) {
+        // every candidate takes part: per-warp private histograms keep the
+        // crowded top bins of skewed scores from serialising across warps
+        unsigned* wh = whist + warp * 256;
+        for (int j = lane; j < 256; j += 32) wh[j] = 0u;
+        __syncwarp();
 #pragma unroll 1
-      for (int g = 0; g < JG; ++g) {
-        const float4 v4 = s4[g * kRegThreads + tid];
-        const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+        for (int g = 0; g < JG; ++g) {
+          const float4 v4 = s4[g * kRegThreads + tid];
+          const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
 #pragma unroll
-        for (int r = 0; r < 4; ++r) {
-          const uint32_t key = orderable_key(vv[r]);
-          const bool in = is_cand(tok(g, r)) && (key & maskbits) == prefix;
-          // one atomic per distinct bin per warp: the hot bins of skewed
-          // scores would otherwise serialise every lane
-          if (!__any_sync(0xffffffffu, in)) continue;
-          const uint32_t bin = in ? ((key >> shift) & 255u) : 256u;
-          const unsigned peers = __match_any_sync(0xffffffffu, bin);
-          if (in && lane == __ffs(peers) - 1) atomicAdd(&sh.hist[bin], (unsigned)__popc(peers));
+          for (int r = 0; r < 4; ++r)
+            if ((live >> (4 * g + r)) & 1u) atomicAdd(&wh[orderable_key(vv[r]) >> 24], 1u);
+        }
+        __syncthreads();
+        for (int j = tid; j < 256; j += kRegThreads) {
+          unsigned t = 0u;
+#pragma unroll 8
+          for (int w = 0; w < kRegWarps; ++w) t += whist[w * 256 + j];
+          sh.hist[j] = t;
+        }
+      } else {
+        for (uint32_t m = live; m; m &= m - 1) {
+          const int bitpos = __ffs(m) - 1;
+          const float4 v4 = s4[(bitpos >> 2) * kRegThreads + tid];
+          const int r = bitpos & 3;
+          const float v = r == 0 ? v4.x : (r == 1 ? v4.y : (r == 2 ? v4.z : v4.w));
+          atomicAdd(&sh.hist[(orderable_key(v) >> shift) & 255u], 1u);
         }
       }
       __syncthreads();
@@ -584,7 +606,7 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
 #pragma unroll
           for (int q = 0; q < 8; ++q) {
             if (cum + c[q] >= remaining) {
-              sh.prefix = prefix | ((unsigned)(255 - 8 * lane - q) << shift);
+              sh.prefix = (unsigned)(255 - 8 * lane - q);  // the chosen digit
               sh.remaining = remaining - cum;
               break;
             }
@@ -593,30 +615,30 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
         }
       }
       __syncthreads();
-      prefix = sh.prefix;
+      const unsigned digit = sh.prefix;
       remaining = sh.remaining;
-      maskbits |= 255u << shift;
-    }
-    uint64_t eq = 0ull;
-#pragma unroll 1
-    for (int g = 0; g < JG; ++g) {
-      const float4 v4 = s4[g * kRegThreads + tid];
-      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
-#pragma unroll
-      for (int r = 0; r < 4; ++r) {
-        if (!is_cand(tok(g, r))) continue;
-        const uint32_t key = orderable_key(vv[r]);
-        if (key > prefix) cert |= 1ull << (4 * g + r);
-        else if (key == prefix) eq |= 1ull << (4 * g + r);
+      for (uint32_t m = live; m; m &= m - 1) {
+        const int bitpos = __ffs(m) - 1;
+        const float4 v4 = s4[(bitpos >> 2) * kRegThreads + tid];
+        const int r = bitpos & 3;
+        const float v = r == 0 ? v4.x : (r == 1 ? v4.y : (r == 2 ? v4.z : v4.w));
+        const unsigned d = (orderable_key(v) >> shift) & 255u;
+        if (d != digit) {
+          live &= ~(1u << bitpos);
+          if (d > digit) cert |= 1u << bitpos;
+        }
       }
     }
+    // `live` now holds exactly the tokens whose key equals the k-th largest;
+    // the `remaining` lowest-index ones complete the top slice
+    const uint32_t eq = live;
     ordered_scan(eq, JG, sh);
 #pragma unroll 1
     for (int g = 0; g < JG; ++g) {
       int run = sh.off[g][warp] + lane_prefix(eq, g);
 #pragma unroll
       for (int r = 0; r < 4; ++r) {
-        const uint64_t bit = 1ull << (4 * g + r);
+        const uint32_t bit = 1u << (4 * g + r);
         if (eq & bit) {
           if (run < (int)remaining) cert |= bit;
           ++run;
@@ -624,15 +646,10 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
       }
     }
   } else if (k > 0) {
-#pragma unroll 1
-    for (int g = 0; g < JG; ++g)
-#pragma unroll
-      for (int r = 0; r < 4; ++r)
-        if (tok(g, r) < N) cert |= 1ull << (4 * g + r);
+    cert = valid;  // every unprotected token is in the top slice
   }
-  auto is_tail = [&](int g, int r) {
-    return tok(g, r) < N && !((cert >> (4 * g + r)) & 1ull);
-  };
+  const uint32_t tail = valid & ~cert;
+  auto is_tail = [&](int g, int r) { return (tail >> (4 * g + r)) & 1u; };
 
   // ---- E2: inclusion probabilities on the tail ---------------------------
   const int n_cert = n_prot + k;
@@ -746,14 +763,12 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
 
   // ---- E3 + E4a: draws and ordered compaction of (index, log 1/pi) --------
   const bool compact = a.n_kept != nullptr;
-  uint64_t keep = 0ull;
+  uint32_t keep = 0u;
 #pragma unroll 1
   for (int g = 0; g < JG; ++g) {
     const float4 v4 = s4[g * kRegThreads + tid];
     const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
-    bool any_tail = false;
-#pragma unroll
-    for (int r = 0; r < 4; ++r) any_tail = any_tail || is_tail(g, r);
+    const bool any_tail = ((tail >> (4 * g)) & 0xFu) != 0u;
     uint4 w = make_uint4(0u, 0u, 0u, 0u);
     if (compact && __any_sync(0xffffffffu, any_tail))
       w = draw_block(a.seed, a.layer, b, kvh, g * kRegThreads + tid);
@@ -761,12 +776,12 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
       const int i = tok(g, r);
-      if (i >= N) continue;
-      const bool ct = (cert >> (4 * g + r)) & 1ull;
+      if (!((valid >> (4 * g + r)) & 1u)) continue;
+      const bool ct = (cert >> (4 * g + r)) & 1u;
       const float pi = ct ? 1.f : tail_pi(vv[r], mode, c, eps);
       if (a.pi_out) a.pi_out[(size_t)unit * N + i] = pi;
       if (a.mask_out) a.mask_out[(size_t)unit * N + i] = ct ? 1 : 0;
-      if (compact && (ct || word_to_uniform(wr[r]) < pi)) keep |= 1ull << (4 * g + r);
+      if (compact && (ct || word_to_uniform(wr[r]) < pi)) keep |= 1u << (4 * g + r);
     }
   }
   if (compact) {
@@ -778,7 +793,7 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
       const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
 #pragma unroll
       for (int r = 0; r < 4; ++r) {
-        const uint64_t bit = 1ull << (4 * g + r);
+        const uint32_t bit = 1u << (4 * g + r);
         if (!(keep & bit)) continue;
         if (p < a.cap) {
           const float pi = (cert & bit) ? 1.f : tail_pi(vv[r], mode, c, eps);
@@ -901,7 +916,7 @@ static ebd_status launch_select(const ebd_design* d, const float* scores, float*
   const int units = d->batch * d->n_kv_heads;
   const int groups = (d->n_ctx + kGroupTokens - 1) / kGroupTokens;
   if (groups <= kRegMaxGroups) {
-    const size_t smem = (size_t)groups * kRegThreads * sizeof(float4);
+    const size_t smem = (size_t)groups * kRegThreads * sizeof(float4) + kRegWarps * 256 * 4;
     if (smem > 48 * 1024 &&
         cudaFuncSetAttribute(evict_select_smem_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem) != cudaSuccess)
