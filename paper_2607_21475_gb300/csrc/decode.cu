@@ -158,11 +158,10 @@ __global__ void __launch_bounds__(kGenThreads) decode_generic_kernel(DecodeArgs 
 }
 
 // Merge the partial records of one query head and finish Eq. (3), Theorem 2,
-// Eq. (4).  One warp per query head: lanes take 32 records at a time (scale
-// factors and scalar moments), then every lane streams its D/32 columns of each
-// record.  CUDA-core path: records u*splits .. u*splits + splits - 1.
-// Tensor-core path: records u + gw for every working warp gw whose tile range
-// meets unit u (none for an empty unit).
+// Eq. (4) (CUDA-core path; the tensor-core kernel merges in place).  One warp
+// per query head: lanes take 32 records at a time (scale factors and scalar
+// moments), then every lane streams its D/32 columns of each record, records
+// u*splits .. u*splits + splits - 1.
 constexpr int kReduceWarps = 4;
 
 template <int D>
@@ -175,21 +174,8 @@ __global__ void __launch_bounds__(kReduceWarps * 32) decode_reduce_kernel(Reduce
   if (hq >= n_heads) return;
   const int G = a.group;
   const int unit = hq / G, g = hq - unit * G;
-  long long first = (long long)unit * a.splits;
-  int count = a.splits;
-  if (a.tile_off) {
-    const long long t0 = a.tile_off[unit], t1 = a.tile_off[unit + 1];
-    const long long Ta = a.tile_off[n_heads / G];
-    long long W = Ta / a.min_tiles > 0 ? Ta / a.min_tiles : 1;
-    if (a.warps < W) W = a.warps;
-    count = 0;
-    if (t1 > t0) {
-      const long long gf = ((t0 + 1) * W - 1) / Ta;
-      const long long gl = (t1 * W - 1) / Ta;
-      first = unit + gf;
-      count = (int)(gl - gf + 1);
-    }
-  }
+  const long long first = (long long)unit * a.splits;
+  const int count = a.splits;
   const size_t slot = (size_t)G * REC;
   const float* R0 = a.part + ((size_t)first * G + g) * REC;
   float Mx = -INFINITY;
@@ -430,7 +416,7 @@ DecodePlan plan_decode(ebd_dtype dtype, int batch, int n_kv_heads, int group, in
   if (fast_decode_supported(dtype, group, head_dim, capacity)) {
     const size_t generic_ws = p.ws_bytes;
     p.fast = true;
-    fast_decode_plan(p, units, group, head_dim, capacity);
+    fast_decode_plan(p, units, group, head_dim);
     if (p.ws_bytes < generic_ws) p.ws_bytes = generic_ws;  // either path fits
   }
   return p;
@@ -484,13 +470,9 @@ extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32
   a.lse = lse;
   a.dev_status = dev_status;
 
-  const bool fast = plan.fast && fast_decode_usable(a, (int)units);
   ReduceArgs r;
   r.part = (const float*)workspace;
   r.splits = plan.splits;
-  r.tile_off = nullptr;
-  r.warps = 0;
-  r.min_tiles = 1;
   r.group = group;
   r.y = y;
   r.lse = lse;
@@ -502,22 +484,19 @@ extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32
   r.exact = range_mode == EBD_RANGE_EXACT;
   const int n_heads = (int)(units * group);
   ebd_status st;
-  if (fast) {
-    st = launch_fast_decode(dtype, head_dim, plan, a, (int)units, s);
-    r.tile_off = (const int32_t*)workspace;
-    r.part = (const float*)((const char*)workspace + fast_decode_records_offset((int)units));
-    r.warps = fast_decode_warps(plan);
-    r.min_tiles = fast_decode_min_tiles_per_warp();
+  if (plan.fast && fast_decode_usable(a, r, (int)units)) {
+    st = launch_fast_decode(dtype, head_dim, plan, a, r, (int)units, workspace, s);
   } else {
     st = dispatch_generic(false, dtype, head_dim, a, (int)units, s);
+    if (st == EBD_OK) {
+      const int rblocks = (n_heads + kReduceWarps - 1) / kReduceWarps;
+      if (head_dim == 128)
+        decode_reduce_kernel<128><<<rblocks, kReduceWarps * 32, 0, s>>>(r, n_heads);
+      else
+        decode_reduce_kernel<64><<<rblocks, kReduceWarps * 32, 0, s>>>(r, n_heads);
+      st = launch_status();
+    }
   }
-  if (st != EBD_OK) return st;
-  const int rblocks = (n_heads + kReduceWarps - 1) / kReduceWarps;
-  if (head_dim == 128)
-    decode_reduce_kernel<128><<<rblocks, kReduceWarps * 32, 0, s>>>(r, n_heads);
-  else
-    decode_reduce_kernel<64><<<rblocks, kReduceWarps * 32, 0, s>>>(r, n_heads);
-  st = launch_status();
   if (st != EBD_OK) return st;
   if (!r.exact) return EBD_OK;
   // exact range term: second pass over the tail rows, then the radius

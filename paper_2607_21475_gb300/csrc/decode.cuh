@@ -40,11 +40,8 @@ struct DecodeArgs {
 };
 
 struct ReduceArgs {
-  const float* part;
-  int splits;                // CUDA-core path: records per unit
-  const int32_t* tile_off;   // tensor-core path: active-tile prefix (null otherwise)
-  long long warps;           // tensor-core path: warps in the grid
-  int min_tiles;             // tensor-core path: minimum tiles per working warp
+  const float* part;         // CUDA-core path: [units, splits, G, rec_floats(D)]
+  int splits;                // records per unit
   int group;
   float* y;
   float* lse;
@@ -61,21 +58,20 @@ struct DecodePlan {
   int splits = 1;            // CUDA-core path: splits per unit
   int tokens_per_split = 0;  // CUDA-core path
   int ctas = 0;              // tensor-core path: persistent grid size
-  size_t ws_bytes = 0;
+  size_t ws_bytes = 0;       // the larger of the two paths' needs
 };
 
 DecodePlan plan_decode(ebd_dtype dtype, int batch, int n_kv_heads, int group, int head_dim,
                        int capacity);
 
-// Tensor-core path (decode_mma.cu).
+// Tensor-core path (decode_mma.cu): decode kernel, then a merge kernel
+// launched as its programmatic dependent (plus a prefix kernel above 4096
+// units).  `ws`: the workspace.
 bool fast_decode_supported(ebd_dtype dtype, int group, int head_dim, int capacity);
-bool fast_decode_usable(const DecodeArgs& a, int units);
-long long fast_decode_warps(const DecodePlan& p);
-size_t fast_decode_records_offset(int units);
-void fast_decode_plan(DecodePlan& p, long long units, int group, int head_dim, int capacity);
-// Plan + decode kernels; records for the reduce kernel.
+bool fast_decode_usable(const DecodeArgs& a, const ReduceArgs& r, int units);
+void fast_decode_plan(DecodePlan& p, long long units, int group, int head_dim);
 ebd_status launch_fast_decode(ebd_dtype dtype, int head_dim, const DecodePlan& plan,
-                              const DecodeArgs& a, int units, cudaStream_t stream);
-int fast_decode_min_tiles_per_warp();
+                              const DecodeArgs& a, const ReduceArgs& r, int units, void* ws,
+                              cudaStream_t stream);
 
 }  // namespace ebd

@@ -5,13 +5,17 @@
 // l = sum w, o = sum w v, U = sum u, A1 = sum u v, A2 = sum u ||v||^2 and the
 // range-bound maxima, with u = (1 - pi) w^2.
 //
-// Layout of the work.  A persistent grid (one CTA per SM) of 8 warps.  The
-// active 16-token tiles of all units (tiles
-// below min(n_kept, cap), counted by a one-CTA plan kernel into tile_off) are
-// split into equal contiguous ranges, one per warp.  A warp's range
-// crosses at most a few units; for each unit it meets it writes one partial
-// record, at index (unit + global warp), so records never collide and no
-// scratch needs clearing.  The reduce kernel merges the records of a unit.
+// Two kernels.  The decode kernel is a persistent grid (one CTA per SM) of 8
+// warps.  Every CTA first builds the prefix of active 16-token tiles per unit
+// (tiles below min(n_kept, cap)) in shared memory (CTA 0 also stores it for
+// the merge); the active tiles of all units are then split into equal
+// contiguous ranges, one per warp.  A warp's range crosses at most a few
+// units; for each unit it meets it writes one partial record, at index
+// (unit + global warp), so records never collide and nothing needs clearing.
+// The merge kernel (one CTA per query head, launched as a programmatic
+// dependent of the decode so its launch overlaps the decode's tail) spreads
+// the head's records over its warps, combines them in shared memory and
+// writes y_hat, lse, V_hat, b_t and r_t.
 //
 // Per tile and warp:
 //   S[16 x 16]  = Qpad[16 x d] . K_tile^T       (rows 0..G-1 = query heads,
@@ -53,6 +57,7 @@ constexpr int kMmaStages = kMmaConsumers * kMmaStagesPerWarp;
 constexpr int kMmaThreads = kMmaConsumers * 32;
 constexpr float kRescaleLog2 = 8.f;
 constexpr int kMinTilesPerWarp = 4;
+constexpr int kLocalUnits = 4096;  // tile prefix kept in shared memory up to this many units
 
 template <int D>
 struct MmaLayout {
@@ -61,28 +66,62 @@ struct MmaLayout {
   static constexpr int kStageBytes = 2 * kHalves * kBoxBytes;
   static constexpr int kLogwOff = kMmaStages * kStageBytes;
   static constexpr int kBarOff = kLogwOff + kMmaStages * kMmaTile * 4;
-  static constexpr int kBytes = kBarOff + kMmaStages * 8 + 1024;  // + alignment slack
+  static constexpr int kScanOff = kBarOff + kMmaStages * 8;       // [kMmaConsumers] ints
+  static constexpr int kPlanOff = kScanOff + 64;                  // [kLocalUnits + 1] ints
+  static constexpr int kBytes = kPlanOff + (kLocalUnits + 1) * 4 + 1024;  // + alignment slack
   static constexpr uint32_t kTxBytes = 2 * kHalves * kBoxBytes + kMmaTile * 4;
 };
 
 struct FastArgs {
-  const __nv_bfloat16* Q;  // [units * G, D]
-  const float* logw;       // [units, cap]
-  const int32_t* n_kept;   // [units]
-  const int32_t* tile_off;  // [units + 1], written by the plan kernel
-  float* part;             // records [(units + W) * G, rec_floats(D)]
+  const __nv_bfloat16* Q;    // [units * G, D]
+  const float* logw;         // [units, cap]
+  const int32_t* n_kept;     // [units]
+  int32_t* tile_off;         // [units + 1]: written by CTA 0, or by the prefix kernel
+  bool plan_done;            // tile_off already holds the prefix (more than kLocalUnits units)
+  float* part;               // records [(units + W) * G, rec_floats(D)]
   int32_t* dev_status;
   int units;
   int cap;
   int group;
 };
 
+struct MergeArgs {
+  const int32_t* tile_off;   // [units + 1]
+  const float* part;         // records of the decode kernel
+  long long warps;           // warps of the decode grid
+  int units;
+  int group;
+  float* y;                  // [units * G, D]
+  float* lse;                // [units * G]
+  float* var;
+  float* b_t;
+  float* radius;
+  float log_inv_delta;
+  float eps0;
+  bool exact;                // b_t / radius come from the exact range pass
+};
+
+// Programmatic dependent launch: the decode lets the merge grid launch early;
+// the merge waits for the whole decode grid (and its memory) before reading.
+__device__ __forceinline__ void grid_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// Working warps of a decode over Ta active tiles (each gets >= kMinTilesPerWarp).
+__host__ __device__ __forceinline__ long long decode_working_warps(long long Ta, long long Wall) {
+  const long long Wcap = Ta / kMinTilesPerWarp > 0 ? Ta / kMinTilesPerWarp : 1;
+  return Wall < Wcap ? Wall : Wcap;
+}
+
 // Largest unit u with tile_off[u] <= t (a unit that holds tile t).
 __device__ __forceinline__ int unit_of_tile(const int32_t* tile_off, int units, int t) {
   int lo = 0, hi = units - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
-    if (__ldg(tile_off + mid) <= t) lo = mid;
+    if (tile_off[mid] <= t) lo = mid;
     else hi = mid - 1;
   }
   return lo;
@@ -91,7 +130,7 @@ __device__ __forceinline__ int unit_of_tile(const int32_t* tile_off, int units, 
 // Next unit after u that holds at least one tile (tile t exists beyond u).
 __device__ __forceinline__ int next_unit(const int32_t* tile_off, int u) {
   ++u;
-  while (__ldg(tile_off + u + 1) == __ldg(tile_off + u)) ++u;
+  while (tile_off[u + 1] == tile_off[u]) ++u;
   return u;
 }
 
@@ -136,6 +175,38 @@ __global__ void decode_tile_plan_kernel(const int32_t* __restrict__ n_kept, int 
   if (tid == 0) tile_off[units] = carry;
 }
 
+// The same prefix built by one CTA of the decode kernel in shared memory:
+// every thread carries the running total itself, so only the per-warp sums of
+// one block-wide step pass through `scan`.
+__device__ void block_tile_prefix(const int32_t* __restrict__ n_kept, int units, int cap,
+                                  int32_t* toff, int* scan) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  int carry = 0;
+  for (int base = 0; base < units; base += kMmaThreads) {
+    const int u = base + tid;
+    const int v = u < units ? (min(max(__ldg(n_kept + u), 0), cap) + kMmaTile - 1) / kMmaTile : 0;
+    int incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int n = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += n;
+    }
+    if (lane == 31) scan[warp] = incl;
+    __syncthreads();
+    int before = 0, total = 0;
+#pragma unroll
+    for (int w = 0; w < kMmaConsumers; ++w) {
+      const int x = scan[w];
+      before += w < warp ? x : 0;
+      total += x;
+    }
+    if (u < units) toff[u] = carry + before + incl - v;
+    carry += total;
+    __syncthreads();  // scan[] is rewritten by the next step
+  }
+  if (tid == 0) toff[units] = carry;
+}
+
 template <int D>
 __global__ void __launch_bounds__(kMmaThreads, 1)
     decode_mma_kernel(const __grid_constant__ CUtensorMap tmK,
@@ -153,16 +224,22 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     for (int s = 0; s < kMmaStages; ++s) mbar_init(&full[s], 1);
     fence_barrier_init();
   }
-  __syncthreads();
-
   const int units = a.units;
-  const int Ta = __ldg(a.tile_off + units);
-  if (Ta == 0) return;
-  const long long Wall = (long long)gridDim.x * kMmaConsumers;
-  // working warps: every one gets >= kMinTilesPerWarp tiles (bounded merge work)
-  const long long Wcap = Ta / kMinTilesPerWarp > 0 ? Ta / kMinTilesPerWarp : 1;
-  const long long W = Wall < Wcap ? Wall : Wcap;
+  const int32_t* toff = a.tile_off;
+  if (!a.plan_done) {
+    int32_t* ts = reinterpret_cast<int32_t*>(smem + L::kPlanOff);
+    block_tile_prefix(a.n_kept, units, a.cap, ts, reinterpret_cast<int*>(smem + L::kScanOff));
+    __syncthreads();
+    if (blockIdx.x == 0)
+      for (int i = threadIdx.x; i <= units; i += kMmaThreads) a.tile_off[i] = ts[i];
+    toff = ts;
+  }
+  __syncthreads();
+  grid_launch_dependents();
 
+  const int Ta = toff[units];
+  if (Ta == 0) return;
+  const long long W = decode_working_warps(Ta, (long long)gridDim.x * kMmaConsumers);
   // global warp index, consecutive indices on different SMs
   const long long gw = (long long)warp * gridDim.x + blockIdx.x;
   if (gw >= W) return;
@@ -174,8 +251,8 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
   uint64_t* my_full = full + warp * kMmaStagesPerWarp;
 
   // copies: lane 0 walks its own cursor through the warp's tiles
-  int pf_t = tb, pf_u = unit_of_tile(a.tile_off, units, tb);
-  int pf_lo = __ldg(a.tile_off + pf_u), pf_hi = __ldg(a.tile_off + pf_u + 1);
+  int pf_t = tb, pf_u = unit_of_tile(toff, units, tb);
+  int pf_lo = toff[pf_u], pf_hi = toff[pf_u + 1];
   int issued = 0;
   auto issue_next = [&]() {
     if (lane == 0 && pf_t < te) {
@@ -192,9 +269,9 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
       bulk_load(lw_s + stage * kMmaTile, a.logw + row0, kMmaTile * 4, &my_full[s]);
       ++pf_t;
       if (pf_t < te && pf_t == pf_hi) {
-        pf_u = next_unit(a.tile_off, pf_u);
+        pf_u = next_unit(toff, pf_u);
         pf_lo = pf_hi;
-        pf_hi = __ldg(a.tile_off + pf_u + 1);
+        pf_hi = toff[pf_u + 1];
       }
     }
     ++issued;
@@ -207,8 +284,8 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
   int seg_end = 0, n_u = 0, seg_start = 0;
 
   auto begin_segment = [&]() {
-    seg_start = __ldg(a.tile_off + u);
-    seg_end = __ldg(a.tile_off + u + 1);
+    seg_start = toff[u];
+    seg_end = toff[u + 1];
     n_u = min(__ldg(a.n_kept + u), a.cap);
     const uint32_t* qrow =
         reinterpret_cast<const uint32_t*>(a.Q + ((size_t)u * G + (g < G ? g : 0)) * D);
@@ -262,7 +339,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     issue_next();  // tile j + 2 into the stage tile j - 1 left
     if (t == seg_end) {
       flush_segment();
-      u = next_unit(a.tile_off, u);
+      u = next_unit(toff, u);
       begin_segment();
     }
     const int n_valid = min(kMmaTile, n_u - (t - seg_start) * kMmaTile);
@@ -403,6 +480,182 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
   }
 }
 
+// Merge the partial records of one query head (Eq. 3, Theorem 2, Eq. 4).  One
+// CTA of MW warps per query head.  Warp w takes records w, w + MW, ... four at
+// a time (all their loads in flight), keeping a running merge relative to its
+// own maximum: every lane reads the same record headers and D/32 columns of o
+// and A1.  The MW warp partials are then combined in shared memory by warp 0,
+// which writes the outputs.  Records of unit u: index u + gw for every working
+// decode warp gw whose tile range meets u.
+template <int D, int MW>
+__global__ void __launch_bounds__(MW * 32) decode_merge_kernel(MergeArgs a) {
+  constexpr int REC = rec_floats(D);
+  constexpr int PER = D / 32;
+  constexpr int BATCH = 4;
+  __shared__ float sh_s[MW][8];  // M, l, U, A2, cmax, umax per warp
+  __shared__ __align__(16) float sh_o[MW][D];
+  __shared__ __align__(16) float sh_a[MW][D];
+  grid_dependency_wait();
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = a.group;
+  const long long hq = blockIdx.x;
+  const int u = (int)(hq / G), g = (int)(hq - (long long)u * G);
+  const long long t0 = a.tile_off[u], t1 = a.tile_off[u + 1];
+  if (t1 == t0) {  // no retained row: y = 0, lse = -inf, zero certificate
+    if (warp == 0) {
+#pragma unroll
+      for (int e = 0; e < PER; ++e) a.y[hq * D + PER * lane + e] = 0.f;
+      if (lane == 0) {
+        a.lse[hq] = -INFINITY;
+        a.var[hq] = 0.f;
+        a.b_t[hq] = 0.f;
+        a.radius[hq] = 0.f;
+      }
+    }
+    return;
+  }
+  const long long Ta = a.tile_off[a.units];
+  const long long W = decode_working_warps(Ta, a.warps);
+  const long long gf = ((t0 + 1) * W - 1) / Ta;  // first decode warp meeting u
+  const long long gl = (t1 * W - 1) / Ta;        // last
+  const int count = (int)(gl - gf + 1);
+  const float* R0 = a.part + ((size_t)(u + gf) * G + g) * REC;
+  const size_t slot = (size_t)G * REC;
+
+  float Mw = -INFINITY, l = 0.f, U = 0.f, A2 = 0.f, cm = 0.f, um = 0.f;
+  float o[PER], a1[PER];
+#pragma unroll
+  for (int e = 0; e < PER; ++e) o[e] = a1[e] = 0.f;
+  for (int k0 = warp; k0 < count; k0 += BATCH * MW) {
+    float4 h[BATCH];
+    float2 c[BATCH];
+    float ov[BATCH][PER], av[BATCH][PER];
+#pragma unroll
+    for (int i = 0; i < BATCH; ++i) {
+      const int k = k0 + i * MW;
+      if (k < count) {
+        const float* R = R0 + k * slot;
+        h[i] = __ldcg(reinterpret_cast<const float4*>(R));
+        c[i] = __ldcg(reinterpret_cast<const float2*>(R + kRecCmax));
+        if constexpr (PER == 4) {
+          const float4 x = __ldcg(reinterpret_cast<const float4*>(R + kRecHead) + lane);
+          const float4 z = __ldcg(reinterpret_cast<const float4*>(R + kRecHead + D) + lane);
+          ov[i][0] = x.x; ov[i][1] = x.y; ov[i][2] = x.z; ov[i][3] = x.w;
+          av[i][0] = z.x; av[i][1] = z.y; av[i][2] = z.z; av[i][3] = z.w;
+        } else {
+          const float2 x = __ldcg(reinterpret_cast<const float2*>(R + kRecHead) + lane);
+          const float2 z = __ldcg(reinterpret_cast<const float2*>(R + kRecHead + D) + lane);
+          ov[i][0] = x.x; ov[i][1] = x.y;
+          av[i][0] = z.x; av[i][1] = z.y;
+        }
+      } else {
+        h[i] = make_float4(-INFINITY, 0.f, 0.f, 0.f);
+        c[i] = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int e = 0; e < PER; ++e) ov[i][e] = av[i][e] = 0.f;
+      }
+    }
+    float mb = Mw;
+#pragma unroll
+    for (int i = 0; i < BATCH; ++i) mb = fmaxf(mb, h[i].x);
+    if (mb > Mw) {  // rescale what this warp holds to the new maximum
+      const float s = Mw == -INFINITY ? 0.f : expf(Mw - mb), s2 = s * s;
+      l *= s;
+      U *= s2;
+      A2 *= s2;
+      cm *= s;
+      um *= s;
+#pragma unroll
+      for (int e = 0; e < PER; ++e) {
+        o[e] *= s;
+        a1[e] *= s2;
+      }
+      Mw = mb;
+    }
+#pragma unroll
+    for (int i = 0; i < BATCH; ++i) {
+      if (h[i].x == -INFINITY) continue;
+      const float f = expf(h[i].x - Mw), f2 = f * f;
+      l = fmaf(f, h[i].y, l);
+      U = fmaf(f2, h[i].z, U);
+      A2 = fmaf(f2, h[i].w, A2);
+      cm = fmaxf(cm, f * c[i].x);
+      um = fmaxf(um, f * c[i].y);
+#pragma unroll
+      for (int e = 0; e < PER; ++e) {
+        o[e] = fmaf(f, ov[i][e], o[e]);
+        a1[e] = fmaf(f2, av[i][e], a1[e]);
+      }
+    }
+  }
+  if (lane == 0) {
+    sh_s[warp][0] = Mw;
+    sh_s[warp][1] = l;
+    sh_s[warp][2] = U;
+    sh_s[warp][3] = A2;
+    sh_s[warp][4] = cm;
+    sh_s[warp][5] = um;
+  }
+#pragma unroll
+  for (int e = 0; e < PER; ++e) {
+    sh_o[warp][PER * lane + e] = o[e];
+    sh_a[warp][PER * lane + e] = a1[e];
+  }
+  __syncthreads();
+  if (warp != 0) return;
+
+  float Mx = -INFINITY;
+#pragma unroll
+  for (int w = 0; w < MW; ++w) Mx = fmaxf(Mx, sh_s[w][0]);
+  l = U = A2 = cm = um = 0.f;
+#pragma unroll
+  for (int e = 0; e < PER; ++e) o[e] = a1[e] = 0.f;
+#pragma unroll
+  for (int w = 0; w < MW; ++w) {
+    const float Ms = sh_s[w][0];
+    if (Ms == -INFINITY) continue;
+    const float f = expf(Ms - Mx), f2 = f * f;
+    l = fmaf(f, sh_s[w][1], l);
+    U = fmaf(f2, sh_s[w][2], U);
+    A2 = fmaf(f2, sh_s[w][3], A2);
+    cm = fmaxf(cm, f * sh_s[w][4]);
+    um = fmaxf(um, f * sh_s[w][5]);
+#pragma unroll
+    for (int e = 0; e < PER; ++e) {
+      o[e] = fmaf(f, sh_o[w][PER * lane + e], o[e]);
+      a1[e] = fmaf(f2, sh_a[w][PER * lane + e], a1[e]);
+    }
+  }
+  float yy = 0.f, ya = 0.f;
+  float yv[PER];
+#pragma unroll
+  for (int e = 0; e < PER; ++e) {
+    yv[e] = o[e] / l;
+    yy = fmaf(yv[e], yv[e], yy);
+    ya = fmaf(yv[e], a1[e], ya);
+  }
+  if constexpr (PER == 4)
+    *reinterpret_cast<float4*>(a.y + hq * D + 4 * lane) = make_float4(yv[0], yv[1], yv[2], yv[3]);
+  else
+    *reinterpret_cast<float2*>(a.y + hq * D + 2 * lane) = make_float2(yv[0], yv[1]);
+  yy = warp_sum(yy);
+  ya = warp_sum(ya);
+  if (lane == 0) {
+    const float ynorm = sqrtf(yy);
+    const float var = fmaxf(0.f, (A2 - 2.f * ya + yy * U) / (l * l));
+    a.lse[hq] = Mx + logf(l);
+    a.var[hq] = var;
+    if (a.exact) {
+      a.b_t[hq] = 0.f;  // filled by the exact range pass
+    } else {
+      const float bt = (cm + ynorm * um) / l;
+      a.b_t[hq] = bt;
+      a.radius[hq] = (sqrtf(2.f * var * a.log_inv_delta) + bt * a.log_inv_delta) / (ynorm + a.eps0);
+    }
+  }
+}
+
 // ---------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------
@@ -438,48 +691,47 @@ bool fast_decode_supported(ebd_dtype dtype, int group, int head_dim, int capacit
          capacity % kMmaTile == 0;
 }
 
-void fast_decode_plan(DecodePlan& p, long long units, int group, int head_dim, int capacity) {
-  (void)capacity;
+// Workspace of the tensor-core path: the tile prefix, then the records.
+static size_t fast_plan_bytes(long long units) {
+  return align_up((size_t)(units + 1) * sizeof(int32_t), 256);
+}
+
+void fast_decode_plan(DecodePlan& p, long long units, int group, int head_dim) {
   p.ctas = sm_count();
   const long long W = (long long)p.ctas * kMmaConsumers;
-  p.ws_bytes = fast_decode_records_offset((int)units) +
+  p.ws_bytes = fast_plan_bytes(units) +
                align_up((size_t)(units + W) * group * rec_floats(head_dim) * sizeof(float), 256);
 }
 
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
-long long fast_decode_warps(const DecodePlan& p) { return (long long)p.ctas * kMmaConsumers; }
-
-int fast_decode_min_tiles_per_warp() { return kMinTilesPerWarp; }
-
-// Workspace: tile_off [units + 1] | records.
-size_t fast_decode_records_offset(int units) {
-  return align_up((size_t)(units + 1) * sizeof(int32_t), 256);
-}
-
-bool fast_decode_usable(const DecodeArgs& a, int units) {
+bool fast_decode_usable(const DecodeArgs& a, const ReduceArgs& r, int units) {
   return aligned16(a.Kc) && aligned16(a.Vc) && aligned16(a.logw) && aligned16(a.Q) &&
-         (long long)units * a.cap < 0x7fffffffLL && tensor_map_encoder() != nullptr;
+         aligned16(r.y) && (long long)units * a.cap < 0x7fffffffLL &&
+         tensor_map_encoder() != nullptr;
 }
 
 template <int D>
-static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, int units,
-                                cudaStream_t s) {
+static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, const ReduceArgs& r,
+                                int units, void* ws, cudaStream_t s) {
   CUtensorMap tmK, tmV;
   const long long rows = (long long)units * a.cap;
   if (!encode_rows_map(&tmK, a.Kc, rows, D) || !encode_rows_map(&tmV, a.Vc, rows, D))
     return EBD_ERR_CUDA;
-  int32_t* tile_off = reinterpret_cast<int32_t*>(a.part);
-  float* recs = reinterpret_cast<float*>(reinterpret_cast<char*>(a.part) +
-                                         fast_decode_records_offset(units));
-  decode_tile_plan_kernel<<<1, 1024, 0, s>>>(a.n_kept, units, a.cap, tile_off);
-  ebd_status st = launch_status();
-  if (st != EBD_OK) return st;
+  int32_t* tile_off = reinterpret_cast<int32_t*>(ws);
+  float* recs = reinterpret_cast<float*>(reinterpret_cast<char*>(ws) + fast_plan_bytes(units));
+  const bool plan_done = units > kLocalUnits;
+  if (plan_done) {
+    decode_tile_plan_kernel<<<1, 1024, 0, s>>>(a.n_kept, units, a.cap, tile_off);
+    const ebd_status st = launch_status();
+    if (st != EBD_OK) return st;
+  }
   FastArgs f;
   f.Q = reinterpret_cast<const __nv_bfloat16*>(a.Q);
   f.logw = a.logw;
   f.n_kept = a.n_kept;
   f.tile_off = tile_off;
+  f.plan_done = plan_done;
   f.part = recs;
   f.dev_status = a.dev_status;
   f.units = units;
@@ -490,14 +742,45 @@ static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, int
                            smem) != cudaSuccess)
     return EBD_ERR_CUDA;
   decode_mma_kernel<D><<<plan.ctas, kMmaThreads, smem, s>>>(tmK, tmV, f);
-  return launch_status();
+  ebd_status st = launch_status();
+  if (st != EBD_OK) return st;
+
+  MergeArgs m;
+  m.tile_off = tile_off;
+  m.part = recs;
+  m.warps = (long long)plan.ctas * kMmaConsumers;
+  m.units = units;
+  m.group = a.group;
+  m.y = r.y;
+  m.lse = r.lse;
+  m.var = r.var;
+  m.b_t = r.b_t;
+  m.radius = r.radius;
+  m.log_inv_delta = r.log_inv_delta;
+  m.eps0 = r.eps0;
+  m.exact = r.exact;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)((long long)units * a.group));
+  // a few records per head: 2 warps (one wave of CTAs); many: 8 warps
+  const bool wide = (long long)plan.ctas * kMmaConsumers > 12LL * units;
+  cfg.blockDim = dim3((wide ? 8 : 2) * 32);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (wide) return cuda_status(cudaLaunchKernelEx(&cfg, decode_merge_kernel<D, 8>, m));
+  return cuda_status(cudaLaunchKernelEx(&cfg, decode_merge_kernel<D, 2>, m));
 }
 
 ebd_status launch_fast_decode(ebd_dtype dtype, int head_dim, const DecodePlan& plan,
-                              const DecodeArgs& a, int units, cudaStream_t stream) {
+                              const DecodeArgs& a, const ReduceArgs& r, int units, void* ws,
+                              cudaStream_t stream) {
   if (dtype != EBD_BF16) return EBD_ERR_UNSUPPORTED;
-  if (head_dim == 128) return launch_fast_t<128>(plan, a, units, stream);
-  if (head_dim == 64) return launch_fast_t<64>(plan, a, units, stream);
+  if (head_dim == 128) return launch_fast_t<128>(plan, a, r, units, ws, stream);
+  if (head_dim == 64) return launch_fast_t<64>(plan, a, r, units, ws, stream);
   return EBD_ERR_UNSUPPORTED;
 }
 

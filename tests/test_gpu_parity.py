@@ -225,6 +225,7 @@ DECODE_CASES = [
     (2, 2, 8, 64, 512, torch.bfloat16, "edges"),     # tensor-core path, head_dim 64, G = 8
     (2, 3, 5, 128, 1000, torch.bfloat16, "random"),  # capacity not a multiple of 16: CUDA cores
     (1, 64, 4, 128, 256, torch.bfloat16, "random"),  # more warps than tiles
+    (1, 1, 8, 128, 32768, torch.bfloat16, "full"),    # one unit, hundreds of partial records
 ]
 
 
@@ -261,6 +262,46 @@ def test_decode_matches_oracle_on_synthetic_cache(E, B, H, G, d, cap, dtype, pat
             sl = slice(h * G, (h + 1) * G)
             compare_decode_heads(dec, out[0][b, sl], out[1][b, sl], out[2][b, sl], out[3][b, sl],
                                  out[4][b, sl], exact)
+
+
+def test_decode_workspace_needs_no_clearing_and_is_deterministic(E):
+    """The decode writes every partial record before its merge reads it: a
+    workspace full of garbage gives the same bits as a fresh one, call after
+    call (both kernels of the tensor-core path reduce in a fixed order)."""
+    B, H, G, d, cap = 4, 8, 4, 128, 2048
+    Kc, Vc, logw, n = _synthetic_cache(B, H, cap, d, torch.bfloat16, "random", seed=11)
+    Q = torch.randn((B, H * G, d), generator=torch.Generator().manual_seed(3)).to(torch.bfloat16)
+    nb = E.ebd_decode_workspace_bytes(E.EBD_BF16, B, H, G, d, cap)
+    ws = torch.full((nb,), 0x7f, dtype=torch.uint8, device=DEV)
+    args = [t.to(DEV) for t in (Q, Kc, Vc, logw, n)]
+    outs = []
+    for i in range(3):
+        if i == 2:
+            ws.fill_(0xff)  # NaN patterns everywhere
+        y = torch.empty((B, H * G, d), dtype=torch.float32, device=DEV)
+        lse, var, bt, r = (torch.empty((B, H * G), dtype=torch.float32, device=DEV) for _ in range(4))
+        E.ebd_certified_decode(*args, y, lse, var, bt, r, workspace=ws)
+        torch.cuda.synchronize()
+        outs.append(torch.cat([y.flatten(), lse.flatten(), var.flatten(), bt.flatten(), r.flatten()]))
+    assert torch.isfinite(outs[0]).all()
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+
+
+def test_decode_many_units_global_tile_prefix(E):
+    """Above 4096 units the tile prefix no longer fits in shared memory and
+    comes from a separate prefix kernel; same results against the oracle."""
+    B, H, G, d, cap = 1040, 4, 2, 64, 64
+    Kc, Vc, logw, n = _synthetic_cache(B, H, cap, d, torch.bfloat16, "edges", seed=5)
+    Q = torch.randn((B, H * G, d), generator=torch.Generator().manual_seed(9)).to(torch.bfloat16)
+    out = _decode(E, Q.to(DEV), Kc.to(DEV), Vc.to(DEV), logw.to(DEV), n.to(DEV))
+    Qd, Kd, Vd, ld = Q.double().numpy(), Kc.double().numpy(), Vc.double().numpy(), logw.double().numpy()
+    for b in list(range(0, B, 37)) + [B - 1]:
+        for h in range(H):
+            k = int(n[b, h])
+            dec = O.hajek_decode(Qd[b, h * G:(h + 1) * G], Kd[b, h, :k], Vd[b, h, :k], ld[b, h, :k])
+            sl = slice(h * G, (h + 1) * G)
+            compare_decode_heads(dec, out[0][b, sl], out[1][b, sl], out[2][b, sl], out[3][b, sl],
+                                 out[4][b, sl], False)
 
 
 def test_evict_then_decode_tiny_end_to_end(E):
