@@ -25,7 +25,15 @@ ebd_status launch_score(ebd_dtype dtype, int batch, int n_kv_heads, int head_dim
                         int n_obs, const void* q_obs, const void* K, float* scores,
                         float* lse_ws, int32_t* dev_status, cudaStream_t stream);
 
-// Tensor-core E0 (score_mma.cu): bf16, head_dim 64/128, 16-byte aligned inputs.
+// E0 on tcgen05 with tensor-memory accumulators (score_tc.cu): bf16,
+// head_dim 64/128, at most 512 observation rows, 16-byte aligned inputs.
+bool score_tc_supported(ebd_dtype dtype, int head_dim, int n_obs, const void* q_obs,
+                        const void* K);
+ebd_status launch_score_tc(int units, int head_dim, int n_ctx, int n_obs, const void* q_obs,
+                           const void* K, float* scores, float* lse, int32_t* dev_status,
+                           cudaStream_t s);
+
+// E0 on mma.sync (score_mma.cu): bf16, head_dim 64/128, 16-byte aligned inputs.
 bool score_mma_supported(ebd_dtype dtype, int head_dim, const void* q_obs, const void* K);
 ebd_status launch_score_mma(int units, int head_dim, int n_ctx, int n_obs, const void* q_obs,
                             const void* K, float* scores, float* lse, int32_t* dev_status,

@@ -127,6 +127,8 @@ ebd_status launch_score(ebd_dtype dtype, int batch, int n_kv_heads, int head_dim
                         float* lse_ws, int32_t* dev_status, cudaStream_t s) {
   const int units = batch * n_kv_heads;
   if (units > 0x7fffffff || n_obs > 4096 || n_obs < 1) return EBD_ERR_UNSUPPORTED;
+  if (score_tc_supported(dtype, head_dim, n_obs, q_obs, K))
+    return launch_score_tc(units, head_dim, n_ctx, n_obs, q_obs, K, scores, lse_ws, dev_status, s);
   if (score_mma_supported(dtype, head_dim, q_obs, K) && units <= 65535 &&
       (n_ctx + 63) / 64 <= 65535)
     return launch_score_mma(units, head_dim, n_ctx, n_obs, q_obs, K, scores, lse_ws, dev_status, s);

@@ -1,0 +1,490 @@
+// E0 on the 5th-generation tensor cores: accumulated attention mass
+//     s_j = sum_r softmax_j(q_r . K^T / sqrt(d))
+// (Appendix B harness, H2O-style accumulated attention from R observation
+// query rows of a KV head's group), bf16 inputs, f32 accumulation in tensor
+// memory, head_dim 64/128, R <= 512.
+//
+// Pass 1, score_lse_tc_kernel: one CTA per (unit, 128 query rows).  The rows
+// are the MMA's M (= tensor-memory lanes), 256-key tiles its N, so the
+// accumulator S[128 x 256] = Q K^T holds one query row per lane and the
+// epilogue thread that owns a lane keeps that row's running
+// (max, sum 2^(x - max)) without any cross-thread traffic.  Two accumulators
+// (256 columns each) alternate so the MMA of tile j + 1 overlaps the epilogue
+// of tile j.  Output: the base-2 log-sum-exp of every row (workspace).
+// Pass 2, score_col_tc_kernel: the transposed product S^T = K Q^T, keys as M
+// (one key per lane), all R query rows as N (split in two halves of <= 256
+// columns, one per accumulator), so key j's thread sums 2^(x_rj - lse_r) over
+// its own row.  A persistent grid walks (unit, 128-key tile) items in order,
+// reloading Q only when the unit changes.
+//
+// Roles: warps 0-3 are the epilogue (warp w reads tensor-memory lanes
+// 32w..32w+31); warp 4 allocates tensor memory and one of its lanes issues
+// the TMA copies (128-byte swizzle) and the tcgen05.mma instructions.
+// Hand-offs use mbarriers: TMA -> MMA (transaction counts), MMA -> epilogue
+// and MMA -> smem reuse (tcgen05.commit), epilogue -> MMA (128 arrivals).
+// Every wait is bounded (~2 s); a timeout raises EBD_DEV_TIMEOUT, the roles
+// leave their loops and the tensor memory is released.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+#include <math.h>
+
+#include <mutex>
+
+#include "common.cuh"
+#include "internal.h"
+#include "ptx.cuh"
+#include "tcgen05.cuh"
+
+namespace ebd {
+
+constexpr int kTcRows1 = 128;   // pass 1: query rows per CTA (MMA M)
+constexpr int kTcKeys1 = 256;   // pass 1: keys per tile (MMA N)
+constexpr int kTcKeys2 = 128;   // pass 2: keys per tile (MMA M)
+constexpr int kTcMaxRows = 512; // pass 2: query rows held as accumulator columns
+constexpr int kTcThreads = 160; // 4 epilogue warps + 1 issue warp
+constexpr uint32_t kTmemCols = 512;
+
+template <int D>
+struct Tc1Layout {
+  static constexpr int kHalves = D / 64;             // 64-column (128-byte) boxes
+  static constexpr int kQBox = kTcRows1 * 128;       // 16 KB
+  static constexpr int kKBox = kTcKeys1 * 128;       // 32 KB
+  static constexpr int kKOff = kHalves * kQBox;
+  static constexpr int kBarOff = kKOff + 2 * kHalves * kKBox;
+  static constexpr int kBytes = kBarOff + 16 * 8 + 1024;  // + alignment slack
+};
+
+template <int D>
+struct Tc2Layout {
+  static constexpr int kHalves = D / 64;
+  static constexpr int kQBox = kTcMaxRows * 128;     // 64 KB (rows beyond R unused)
+  static constexpr int kKBox = kTcKeys2 * 128;       // 16 KB
+  static constexpr int kKOff = kHalves * kQBox;
+  static constexpr int kLseOff = kKOff + 2 * kHalves * kKBox;  // [2][kTcMaxRows] f32
+  static constexpr int kBarOff = kLseOff + 2 * kTcMaxRows * 4;
+  static constexpr int kBytes = kBarOff + 16 * 8 + 1024;
+};
+
+struct TcArgs {
+  int units;
+  int n_ctx;     // N
+  int n_obs;     // R
+  int mtiles;    // pass 1: ceil(R / 128)
+  int rows_pad;  // pass 2: R rounded up to 32
+  int n_a;       // pass 2: accumulator A columns (<= 256)
+  int n_b;       // pass 2: accumulator B columns (rows_pad - n_a)
+  int items;     // pass 2: units * ceil(N / 128)
+  float scale2;  // log2(e) / sqrt(d)
+  float* lse2;   // [units, R] base-2 log-sum-exp (pass 1 out, pass 2 in)
+  float* scores; // [units, N]
+  int32_t* dev_status;
+};
+
+__device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
+  return (unsigned char*)(((uintptr_t)p + 1023) & ~(uintptr_t)1023);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
+                        const __grid_constant__ CUtensorMap tmK, TcArgs a) {
+  using L = Tc1Layout<D>;
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem = align1024(smem_raw);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::kBarOff);
+  uint64_t* q_full = bars;
+  uint64_t* k_full = bars + 1;     // [2]
+  uint64_t* k_empty = bars + 3;    // [2]
+  uint64_t* acc_full = bars + 5;   // [2]
+  uint64_t* acc_empty = bars + 7;  // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 9);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int unit = blockIdx.x / a.mtiles, mt = blockIdx.x - unit * a.mtiles;
+  const int nk = (a.n_ctx + kTcKeys1 - 1) / kTcKeys1;
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+      mbar_init(&acc_full[s], 1);
+      mbar_init(&acc_empty[s], 128);
+    }
+    fence_barrier_init();
+  }
+  if (warp == 4) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  bool ok = true;
+
+  if (warp == 4) {
+    if (lane == 0) {
+      const int krow0 = unit * a.n_ctx;
+      mbar_arrive_expect_tx(q_full, L::kHalves * L::kQBox);
+#pragma unroll
+      for (int h = 0; h < L::kHalves; ++h)
+        tma_load_2d(smem + h * L::kQBox, &tmQ, h * 64, unit * a.n_obs + mt * kTcRows1, q_full);
+      auto load_k = [&](int j) {
+        const int s = j & 1;
+        mbar_arrive_expect_tx(&k_full[s], L::kHalves * L::kKBox);
+#pragma unroll
+        for (int h = 0; h < L::kHalves; ++h)
+          tma_load_2d(smem + L::kKOff + (s * L::kHalves + h) * L::kKBox, &tmK, h * 64,
+                      krow0 + j * kTcKeys1, &k_full[s]);
+      };
+      load_k(0);
+      ok = mbar_wait_bounded(q_full, 0);
+      const uint32_t idesc = umma_idesc_bf16_f32(128, kTcKeys1);
+      const uint32_t qbase = smem_u32(smem);
+      for (int j = 0; ok && j < nk; ++j) {
+        const int s = j & 1;
+        if (j + 1 < nk) {  // next key tile into the other stage once its MMAs are done
+          if (j >= 1 && !mbar_wait_bounded(&k_empty[s ^ 1], ((j - 1) >> 1) & 1)) {
+            ok = false;
+            break;
+          }
+          load_k(j + 1);
+        }
+        if (!mbar_wait_bounded(&k_full[s], (j >> 1) & 1) ||
+            (j >= 2 && !mbar_wait_bounded(&acc_empty[s], ((j - 2) >> 1) & 1))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t kbase = smem_u32(smem + L::kKOff + s * L::kHalves * L::kKBox);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (uint32_t)((kk & 3) * 32);
+          const uint64_t ad = umma_desc_k_sw128(qbase + (kk >> 2) * L::kQBox + off);
+          const uint64_t bd = umma_desc_k_sw128(kbase + (kk >> 2) * L::kKBox + off);
+          umma_bf16(tmem + s * kTcKeys1, ad, bd, idesc, kk > 0);
+        }
+        umma_commit(&k_empty[s]);
+        umma_commit(&acc_full[s]);
+      }
+    }
+    __syncwarp();
+  } else {
+    // epilogue: thread = query row = tensor-memory lane
+    const int row = warp * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    float m = -INFINITY, ssum = 0.f;
+    for (int j = 0; j < nk; ++j) {
+      const int b = j & 1;
+      if (!mbar_wait_bounded(&acc_full[b], (j >> 1) & 1)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const int kvalid = a.n_ctx - j * kTcKeys1;  // keys of this tile inside the unit
+#pragma unroll 1
+      for (int c = 0; c < kTcKeys1 / 32 && c * 32 < kvalid; ++c) {
+        uint32_t r[32];
+        tmem_ld32(tmem + lane_base + b * kTcKeys1 + c * 32, r);
+        tmem_ld_wait();
+        float x[32];
+        float cm = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          x[i] = (c * 32 + i < kvalid) ? __uint_as_float(r[i]) * a.scale2 : -INFINITY;
+          cm = fmaxf(cm, x[i]);
+        }
+        if (cm > m) {
+          ssum *= exp2f(m - cm);
+          m = cm;
+        }
+        float cs = 0.f;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) cs += exp2f(x[i] - m);
+        ssum += cs;
+      }
+      tc_fence_before();
+      mbar_arrive(&acc_empty[b]);
+    }
+    const int r = mt * kTcRows1 + row;
+    if (ok && r < a.n_obs) a.lse2[(size_t)unit * a.n_obs + r] = m + log2f(ssum);
+  }
+  if (!ok) raise_status(a.dev_status, EBD_DEV_TIMEOUT);
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 4) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    score_col_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
+                        const __grid_constant__ CUtensorMap tmK, TcArgs a) {
+  using L = Tc2Layout<D>;
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem = align1024(smem_raw);
+  float* lse_s = reinterpret_cast<float*>(smem + L::kLseOff);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::kBarOff);
+  uint64_t* q_full = bars;
+  uint64_t* k_full = bars + 1;     // [2] key stages
+  uint64_t* k_empty = bars + 3;    // [2]
+  uint64_t* acc_full = bars + 5;   // [2] accumulator halves
+  uint64_t* acc_empty = bars + 7;  // [2]
+  uint64_t* lse_ready = bars + 9;  // the epilogue staged a unit's row log-sum-exps
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 10);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nkt = (a.n_ctx + kTcKeys2 - 1) / kTcKeys2;
+  const int i0 = (int)((long long)blockIdx.x * a.items / gridDim.x);
+  const int i1 = (int)((long long)(blockIdx.x + 1) * a.items / gridDim.x);
+  const int n = i1 - i0;
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+      mbar_init(&acc_full[s], 1);
+      mbar_init(&acc_empty[s], 128);
+    }
+    mbar_init(lse_ready, 128);
+    fence_barrier_init();
+  }
+  if (warp == 4) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  bool ok = true;
+  const int nq_loads = (a.rows_pad + 255) / 256;  // 256-row TMA boxes of Q
+
+  if (warp == 4) {
+    if (lane == 0 && n > 0) {
+      auto load_k = [&](int i) {
+        const int item = i0 + i, u = item / nkt, kt = item - u * nkt;
+        const int s = i & 1;
+        mbar_arrive_expect_tx(&k_full[s], L::kHalves * L::kKBox);
+#pragma unroll
+        for (int h = 0; h < L::kHalves; ++h)
+          tma_load_2d(smem + L::kKOff + (s * L::kHalves + h) * L::kKBox, &tmK, h * 64,
+                      u * a.n_ctx + kt * kTcKeys2, &k_full[s]);
+      };
+      const uint32_t idesc_a = umma_idesc_bf16_f32(128, a.n_a);
+      const uint32_t idesc_b = umma_idesc_bf16_f32(128, a.n_b > 0 ? a.n_b : 16);
+      const uint32_t qbase = smem_u32(smem);
+      int cur_u = -1, qloads = 0;
+      bool qwait = false;
+      load_k(0);
+      for (int i = 0; ok && i < n; ++i) {
+        const int item = i0 + i, u = item / nkt;
+        const int s = i & 1;
+        if (u != cur_u) {  // new unit: Q once every MMA reading the old one is done
+          if (i > 0 && !mbar_wait_bounded(&k_empty[s ^ 1], ((i - 1) >> 1) & 1)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(q_full, L::kHalves * nq_loads * 256 * 128);
+#pragma unroll
+          for (int h = 0; h < L::kHalves; ++h)
+            for (int l = 0; l < nq_loads; ++l)
+              tma_load_2d(smem + h * L::kQBox + l * 256 * 128, &tmQ, h * 64,
+                          u * a.n_obs + l * 256, q_full);
+          cur_u = u;
+          qwait = true;
+        }
+        if (i + 1 < n) {
+          if (i >= 1 && !mbar_wait_bounded(&k_empty[s ^ 1], ((i - 1) >> 1) & 1)) {
+            ok = false;
+            break;
+          }
+          load_k(i + 1);
+        }
+        if (!mbar_wait_bounded(&k_full[s], (i >> 1) & 1)) {
+          ok = false;
+          break;
+        }
+        if (qwait) {
+          if (!mbar_wait_bounded(q_full, qloads & 1)) {
+            ok = false;
+            break;
+          }
+          ++qloads;
+          qwait = false;
+        }
+        const uint32_t kbase = smem_u32(smem + L::kKOff + s * L::kHalves * L::kKBox);
+        for (int hh = 0; hh < 2; ++hh) {
+          const int ncols = hh == 0 ? a.n_a : a.n_b;
+          if (ncols == 0) continue;
+          if (i >= 1 && !mbar_wait_bounded(&acc_empty[hh], (i - 1) & 1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t row_off = (uint32_t)(hh * a.n_a) * 128u;  // first query row of the half
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (uint32_t)((kk & 3) * 32);
+            const uint64_t ad = umma_desc_k_sw128(kbase + (kk >> 2) * L::kKBox + off);
+            const uint64_t bd = umma_desc_k_sw128(qbase + (kk >> 2) * L::kQBox + row_off + off);
+            umma_bf16(tmem + hh * 256, ad, bd, hh == 0 ? idesc_a : idesc_b, kk > 0);
+          }
+          umma_commit(&acc_full[hh]);
+        }
+        if (!ok) break;
+        umma_commit(&k_empty[s]);
+      }
+    }
+    __syncwarp();
+  } else {
+    // epilogue: thread = key = tensor-memory lane
+    const int row = warp * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    int cur_u = -1, par = 0, changes = 0;
+    for (int i = 0; i < n; ++i) {
+      const int item = i0 + i, u = item / nkt, kt = item - u * nkt;
+      if (u != cur_u) {  // this unit's row log-sum-exps (padding rows contribute 0)
+        par ^= 1;
+        float* ls = lse_s + par * kTcMaxRows;
+        for (int r = row; r < a.rows_pad; r += 128)
+          ls[r] = r < a.n_obs ? a.lse2[(size_t)u * a.n_obs + r] : INFINITY;
+        mbar_arrive(lse_ready);  // release: the rows this thread staged
+        if (!mbar_wait_bounded(lse_ready, changes & 1)) {
+          ok = false;
+          break;
+        }
+        ++changes;
+        cur_u = u;
+      }
+      const float* ls = lse_s + par * kTcMaxRows;
+      float sum = 0.f;
+      for (int hh = 0; hh < 2; ++hh) {
+        const int ncols = hh == 0 ? a.n_a : a.n_b;
+        if (ncols == 0) continue;
+        if (!mbar_wait_bounded(&acc_full[hh], i & 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const float* lh = ls + hh * a.n_a;
+#pragma unroll 1
+        for (int c = 0; c < ncols / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(tmem + lane_base + hh * 256 + c * 32, r);
+          tmem_ld_wait();
+          float cs = 0.f;
+#pragma unroll
+          for (int t = 0; t < 32; ++t)
+            cs += exp2f(fmaf(__uint_as_float(r[t]), a.scale2, -lh[c * 32 + t]));
+          sum += cs;
+        }
+        tc_fence_before();
+        mbar_arrive(&acc_empty[hh]);
+      }
+      if (!ok) break;
+      const int key = kt * kTcKeys2 + row;
+      if (key < a.n_ctx) a.scores[(size_t)u * a.n_ctx + key] = sum;
+    }
+  }
+  if (!ok) raise_status(a.dev_status, EBD_DEV_TIMEOUT);
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 4) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+static PFN_cuTensorMapEncodeTiled_v12000 tc_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// [rows, D] bf16 as 2D; box = 64 columns x box_rows rows, 128-byte swizzle.
+static bool encode_bf16_rows(CUtensorMap* map, const void* base, long long rows, int D,
+                             int box_rows) {
+  auto enc = tc_encoder();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)D * 2};
+  const cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool score_tc_supported(ebd_dtype dtype, int head_dim, int n_obs, const void* q_obs,
+                        const void* K) {
+  return dtype == EBD_BF16 && (head_dim == 64 || head_dim == 128) && n_obs >= 1 &&
+         n_obs <= kTcMaxRows && ((uintptr_t)q_obs & 15u) == 0 && ((uintptr_t)K & 15u) == 0 &&
+         tc_encoder() != nullptr;
+}
+
+template <int D>
+static ebd_status launch_score_tc_t(int units, int n_ctx, int n_obs, const void* q_obs,
+                                    const void* K, float* scores, float* lse2,
+                                    int32_t* dev_status, cudaStream_t s) {
+  CUtensorMap tmQ1, tmK1, tmQ2, tmK2;
+  const long long qrows = (long long)units * n_obs, krows = (long long)units * n_ctx;
+  if (!encode_bf16_rows(&tmQ1, q_obs, qrows, D, kTcRows1) ||
+      !encode_bf16_rows(&tmK1, K, krows, D, kTcKeys1) ||
+      !encode_bf16_rows(&tmQ2, q_obs, qrows, D, 256) ||
+      !encode_bf16_rows(&tmK2, K, krows, D, kTcKeys2))
+    return EBD_ERR_CUDA;
+  TcArgs a;
+  a.units = units;
+  a.n_ctx = n_ctx;
+  a.n_obs = n_obs;
+  a.mtiles = (n_obs + kTcRows1 - 1) / kTcRows1;
+  a.rows_pad = (n_obs + 31) / 32 * 32;
+  a.n_a = a.rows_pad < 256 ? a.rows_pad : 256;
+  a.n_b = a.rows_pad - a.n_a;
+  a.items = units * ((n_ctx + kTcKeys2 - 1) / kTcKeys2);
+  a.scale2 = kLog2e / sqrtf((float)D);
+  a.lse2 = lse2;
+  a.scores = scores;
+  a.dev_status = dev_status;
+  const int smem1 = Tc1Layout<D>::kBytes, smem2 = Tc2Layout<D>::kBytes;
+  if (cudaFuncSetAttribute(score_lse_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           smem1) != cudaSuccess ||
+      cudaFuncSetAttribute(score_col_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           smem2) != cudaSuccess)
+    return EBD_ERR_CUDA;
+  score_lse_tc_kernel<D><<<units * a.mtiles, kTcThreads, smem1, s>>>(tmQ1, tmK1, a);
+  ebd_status st = launch_status();
+  if (st != EBD_OK) return st;
+  const int ctas = a.items < sm_count() ? a.items : sm_count();
+  score_col_tc_kernel<D><<<ctas, kTcThreads, smem2, s>>>(tmQ2, tmK2, a);
+  return launch_status();
+}
+
+ebd_status launch_score_tc(int units, int head_dim, int n_ctx, int n_obs, const void* q_obs,
+                           const void* K, float* scores, float* lse, int32_t* dev_status,
+                           cudaStream_t s) {
+  if ((long long)units * n_ctx >= 0x7fffffffLL || (long long)units * n_obs >= 0x7fffffffLL)
+    return EBD_ERR_UNSUPPORTED;
+  if (head_dim == 128)
+    return launch_score_tc_t<128>(units, n_ctx, n_obs, q_obs, K, scores, lse, dev_status, s);
+  if (head_dim == 64)
+    return launch_score_tc_t<64>(units, n_ctx, n_obs, q_obs, K, scores, lse, dev_status, s);
+  return EBD_ERR_UNSUPPORTED;
+}
+
+}  // namespace ebd
