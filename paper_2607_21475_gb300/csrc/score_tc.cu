@@ -17,11 +17,14 @@
 // its own row.  A persistent grid walks (unit, 128-key tile) items in order,
 // reloading Q only when the unit changes.
 //
-// Roles: warps 0-3 are the epilogue (warp w reads tensor-memory lanes
-// 32w..32w+31); warp 4 allocates tensor memory and one of its lanes issues
-// the TMA copies (128-byte swizzle) and the tcgen05.mma instructions.
+// Roles: warps 0-15 are the epilogue (warps w, w + 4, w + 8, w + 12 read
+// tensor-memory lanes 32 (w % 4) .. + 31 and take every fourth 32-column chunk
+// of the accumulator); warp 16 allocates tensor memory and one of its lanes
+// issues the TMA copies (128-byte swizzle) and the tcgen05.mma instructions.
 // Hand-offs use mbarriers: TMA -> MMA (transaction counts), MMA -> epilogue
-// and MMA -> smem reuse (tcgen05.commit), epilogue -> MMA (128 arrivals).
+// and MMA -> smem reuse (tcgen05.commit), epilogue -> MMA (512 arrivals).  The
+// four warps of a lane quarter combine their parts of a row (pass 1) or of a
+// key's sum (pass 2) through shared memory, in a fixed order.
 // Every wait is bounded (~2 s); a timeout raises EBD_DEV_TIMEOUT, the roles
 // leave their loops and the tensor memory is released.
 #include <cuda.h>
@@ -42,7 +45,10 @@ constexpr int kTcRows1 = 128;   // pass 1: query rows per CTA (MMA M)
 constexpr int kTcKeys1 = 256;   // pass 1: keys per tile (MMA N)
 constexpr int kTcKeys2 = 128;   // pass 2: keys per tile (MMA M)
 constexpr int kTcMaxRows = 512; // pass 2: query rows held as accumulator columns
-constexpr int kTcThreads = 160; // 4 epilogue warps + 1 issue warp
+constexpr int kTcGroups = 4;    // epilogue warps per tensor-memory lane quarter
+constexpr int kTcEpi = 128 * kTcGroups;  // epilogue threads
+constexpr int kTcThreads = kTcEpi + 32;  // + 1 issue warp
+constexpr int kTcIssueWarp = kTcEpi / 32;
 constexpr uint32_t kTmemCols = 512;
 
 template <int D>
@@ -51,7 +57,8 @@ struct Tc1Layout {
   static constexpr int kQBox = kTcRows1 * 128;       // 16 KB
   static constexpr int kKBox = kTcKeys1 * 128;       // 32 KB
   static constexpr int kKOff = kHalves * kQBox;
-  static constexpr int kBarOff = kKOff + 2 * kHalves * kKBox;
+  static constexpr int kPartOff = kKOff + 2 * kHalves * kKBox;  // [groups][128][2] f32
+  static constexpr int kBarOff = kPartOff + kTcGroups * 128 * 2 * 4;
   static constexpr int kBytes = kBarOff + 16 * 8 + 1024;  // + alignment slack
 };
 
@@ -62,7 +69,8 @@ struct Tc2Layout {
   static constexpr int kKBox = kTcKeys2 * 128;       // 16 KB
   static constexpr int kKOff = kHalves * kQBox;
   static constexpr int kLseOff = kKOff + 2 * kHalves * kKBox;  // [2][kTcMaxRows] f32
-  static constexpr int kBarOff = kLseOff + 2 * kTcMaxRows * 4;
+  static constexpr int kPartOff = kLseOff + 2 * kTcMaxRows * 4;  // [2][groups][128] f32
+  static constexpr int kBarOff = kPartOff + 2 * kTcGroups * 128 * 4;
   static constexpr int kBytes = kBarOff + 16 * 8 + 1024;
 };
 
@@ -109,11 +117,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_init(&k_full[s], 1);
       mbar_init(&k_empty[s], 1);
       mbar_init(&acc_full[s], 1);
-      mbar_init(&acc_empty[s], 128);
+      mbar_init(&acc_empty[s], kTcEpi);
     }
     fence_barrier_init();
   }
-  if (warp == 4) {
+  if (warp == kTcIssueWarp) {
     tmem_alloc(tmem_slot, kTmemCols);
     tmem_relinquish();
   }
@@ -122,8 +130,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   bool ok = true;
+  const int quarter = warp & 3, grp = warp >> 2;  // epilogue lane quarter, chunk group
+  const int row = quarter * 32 + lane;
+  float m = -INFINITY, ssum = 0.f;  // epilogue: raw max logit and sum 2^((x - m) scale2)
 
-  if (warp == 4) {
+  if (warp == kTcIssueWarp) {
     if (lane == 0) {
       const int krow0 = unit * a.n_ctx;
       mbar_arrive_expect_tx(q_full, L::kHalves * L::kQBox);
@@ -171,10 +182,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     __syncwarp();
   } else {
-    // epilogue: thread = query row = tensor-memory lane
-    const int row = warp * 32 + lane;
-    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-    float m = -INFINITY, ssum = 0.f;
+    // epilogue: thread = query row (tensor-memory lane) x every fourth 32-key chunk
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    const float sc = a.scale2;
     for (int j = 0; j < nk; ++j) {
       const int b = j & 1;
       if (!mbar_wait_bounded(&acc_full[b], (j >> 1) & 1)) {
@@ -184,36 +194,54 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       tc_fence_after();
       const int kvalid = a.n_ctx - j * kTcKeys1;  // keys of this tile inside the unit
 #pragma unroll 1
-      for (int c = 0; c < kTcKeys1 / 32 && c * 32 < kvalid; ++c) {
+      for (int c = grp; c < kTcKeys1 / 32 && c * 32 < kvalid; c += kTcGroups) {
         uint32_t r[32];
         tmem_ld32(tmem + lane_base + b * kTcKeys1 + c * 32, r);
         tmem_ld_wait();
         float x[32];
-        float cm = -INFINITY;
+        const int nv = kvalid - c * 32;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          x[i] = (c * 32 + i < kvalid) ? __uint_as_float(r[i]) * a.scale2 : -INFINITY;
-          cm = fmaxf(cm, x[i]);
-        }
+        for (int i = 0; i < 32; ++i) x[i] = (nv >= 32 || i < nv) ? __uint_as_float(r[i]) : -INFINITY;
+        float m4[4] = {x[0], x[1], x[2], x[3]};
+#pragma unroll
+        for (int i = 4; i < 32; ++i) m4[i & 3] = fmaxf(m4[i & 3], x[i]);
+        const float cm = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
         if (cm > m) {
-          ssum *= exp2f(m - cm);
+          ssum *= exp2f((m - cm) * sc);
           m = cm;
         }
-        float cs = 0.f;
+        const float mc = m * sc;
+        float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int i = 0; i < 32; ++i) cs += exp2f(x[i] - m);
-        ssum += cs;
+        for (int i = 0; i < 32; ++i) s4[i & 3] += exp2f(fmaf(x[i], sc, -mc));
+        ssum += (s4[0] + s4[1]) + (s4[2] + s4[3]);
       }
       tc_fence_before();
       mbar_arrive(&acc_empty[b]);
     }
+  }
+  // the four parts of each row meet in shared memory
+  float* part = reinterpret_cast<float*>(smem + L::kPartOff);
+  if (warp < kTcIssueWarp) {
+    part[(grp * 128 + row) * 2] = m;
+    part[(grp * 128 + row) * 2 + 1] = ssum;
+  }
+  __syncthreads();
+  if (warp < kTcIssueWarp && grp == 0) {
+    float M = -INFINITY;
+#pragma unroll
+    for (int q = 0; q < kTcGroups; ++q) M = fmaxf(M, part[(q * 128 + row) * 2]);
+    float tot = 0.f;
+#pragma unroll
+    for (int q = 0; q < kTcGroups; ++q)
+      tot += part[(q * 128 + row) * 2 + 1] * exp2f((part[(q * 128 + row) * 2] - M) * a.scale2);
     const int r = mt * kTcRows1 + row;
-    if (ok && r < a.n_obs) a.lse2[(size_t)unit * a.n_obs + r] = m + log2f(ssum);
+    if (ok && r < a.n_obs) a.lse2[(size_t)unit * a.n_obs + r] = M * a.scale2 + log2f(tot);
   }
   if (!ok) raise_status(a.dev_status, EBD_DEV_TIMEOUT);
   tc_fence_before();
   __syncthreads();
-  if (warp == 4) {
+  if (warp == kTcIssueWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
@@ -233,8 +261,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   uint64_t* k_empty = bars + 3;    // [2]
   uint64_t* acc_full = bars + 5;   // [2] accumulator halves
   uint64_t* acc_empty = bars + 7;  // [2]
-  uint64_t* lse_ready = bars + 9;  // the epilogue staged a unit's row log-sum-exps
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 10);
+  uint64_t* lse_ready = bars + 9;   // the epilogue staged a unit's row log-sum-exps
+  uint64_t* part_ready = bars + 10;  // warps 4-15 left their partial key sums
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 11);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nkt = (a.n_ctx + kTcKeys2 - 1) / kTcKeys2;
@@ -247,12 +276,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_init(&k_full[s], 1);
       mbar_init(&k_empty[s], 1);
       mbar_init(&acc_full[s], 1);
-      mbar_init(&acc_empty[s], 128);
+      mbar_init(&acc_empty[s], kTcEpi);
     }
-    mbar_init(lse_ready, 128);
+    mbar_init(lse_ready, kTcEpi);
+    mbar_init(part_ready, kTcEpi - 128);
     fence_barrier_init();
   }
-  if (warp == 4) {
+  if (warp == kTcIssueWarp) {
     tmem_alloc(tmem_slot, kTmemCols);
     tmem_relinquish();
   }
@@ -263,7 +293,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   bool ok = true;
   const int nq_loads = (a.rows_pad + 255) / 256;  // 256-row TMA boxes of Q
 
-  if (warp == 4) {
+  if (warp == kTcIssueWarp) {
     if (lane == 0 && n > 0) {
       auto load_k = [&](int i) {
         const int item = i0 + i, u = item / nkt, kt = item - u * nkt;
@@ -341,16 +371,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     __syncwarp();
   } else {
-    // epilogue: thread = key = tensor-memory lane
-    const int row = warp * 32 + lane;
-    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    // epilogue: thread = key (tensor-memory lane); the 32-column chunks of the
+    // [A | B] accumulator columns go round-robin to warps w, w + 4, w + 8, w + 12
+    const int quarter = warp & 3, grp = warp >> 2;
+    const int row = quarter * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    float* part = reinterpret_cast<float*>(smem + L::kPartOff);
+    const int nch = a.rows_pad / 32;
     int cur_u = -1, par = 0, changes = 0;
     for (int i = 0; i < n; ++i) {
       const int item = i0 + i, u = item / nkt, kt = item - u * nkt;
       if (u != cur_u) {  // this unit's row log-sum-exps (padding rows contribute 0)
         par ^= 1;
         float* ls = lse_s + par * kTcMaxRows;
-        for (int r = row; r < a.rows_pad; r += 128)
+        for (int r = threadIdx.x; r < a.rows_pad; r += kTcEpi)
           ls[r] = r < a.n_obs ? a.lse2[(size_t)u * a.n_obs + r] : INFINITY;
         mbar_arrive(lse_ready);  // release: the rows this thread staged
         if (!mbar_wait_bounded(lse_ready, changes & 1)) {
@@ -361,7 +395,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         cur_u = u;
       }
       const float* ls = lse_s + par * kTcMaxRows;
-      float sum = 0.f;
+      float s4[4] = {0.f, 0.f, 0.f, 0.f};
       for (int hh = 0; hh < 2; ++hh) {
         const int ncols = hh == 0 ? a.n_a : a.n_b;
         if (ncols == 0) continue;
@@ -370,30 +404,50 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           break;
         }
         tc_fence_after();
-        const float* lh = ls + hh * a.n_a;
+        const int c0 = hh == 0 ? 0 : a.n_a / 32, c1 = hh == 0 ? a.n_a / 32 : nch;
+        // first chunk c >= c0 with c % groups == grp
+        const int cfirst = c0 + ((grp - c0 % kTcGroups) + kTcGroups) % kTcGroups;
 #pragma unroll 1
-        for (int c = 0; c < ncols / 32; ++c) {
+        for (int c = cfirst; c < c1; c += kTcGroups) {
           uint32_t r[32];
-          tmem_ld32(tmem + lane_base + hh * 256 + c * 32, r);
+          tmem_ld32(tmem + lane_base + hh * 256 + (c - c0) * 32, r);
           tmem_ld_wait();
-          float cs = 0.f;
+          const float4* l4 = reinterpret_cast<const float4*>(ls + c * 32);
 #pragma unroll
-          for (int t = 0; t < 32; ++t)
-            cs += exp2f(fmaf(__uint_as_float(r[t]), a.scale2, -lh[c * 32 + t]));
-          sum += cs;
+          for (int t = 0; t < 8; ++t) {
+            const float4 lv = l4[t];
+            s4[0] += exp2f(fmaf(__uint_as_float(r[4 * t + 0]), a.scale2, -lv.x));
+            s4[1] += exp2f(fmaf(__uint_as_float(r[4 * t + 1]), a.scale2, -lv.y));
+            s4[2] += exp2f(fmaf(__uint_as_float(r[4 * t + 2]), a.scale2, -lv.z));
+            s4[3] += exp2f(fmaf(__uint_as_float(r[4 * t + 3]), a.scale2, -lv.w));
+          }
         }
         tc_fence_before();
         mbar_arrive(&acc_empty[hh]);
       }
       if (!ok) break;
-      const int key = kt * kTcKeys2 + row;
-      if (key < a.n_ctx) a.scores[(size_t)u * a.n_ctx + key] = sum;
+      const float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+      float* pb = part + (i & 1) * kTcGroups * 128;
+      if (grp != 0) {
+        pb[grp * 128 + row] = sum;
+        mbar_arrive(part_ready);  // release
+      } else {
+        if (!mbar_wait_bounded(part_ready, i & 1)) {
+          ok = false;
+          break;
+        }
+        float tot = sum;
+#pragma unroll
+        for (int q = 1; q < kTcGroups; ++q) tot += pb[q * 128 + row];
+        const int key = kt * kTcKeys2 + row;
+        if (key < a.n_ctx) a.scores[(size_t)u * a.n_ctx + key] = tot;
+      }
     }
   }
   if (!ok) raise_status(a.dev_status, EBD_DEV_TIMEOUT);
   tc_fence_before();
   __syncthreads();
-  if (warp == 4) {
+  if (warp == kTcIssueWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
