@@ -200,8 +200,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         tmem_ld_wait();
         float x[32];
         const int nv = kvalid - c * 32;
+        if (nv >= 32) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) x[i] = (nv >= 32 || i < nv) ? __uint_as_float(r[i]) : -INFINITY;
+          for (int i = 0; i < 32; ++i) x[i] = __uint_as_float(r[i]);
+        } else {  // the unit's last keys: the rest of the chunk is another unit's
+#pragma unroll
+          for (int i = 0; i < 32; ++i) x[i] = i < nv ? __uint_as_float(r[i]) : -INFINITY;
+        }
         float m4[4] = {x[0], x[1], x[2], x[3]};
 #pragma unroll
         for (int i = 4; i < 32; ++i) m4[i & 3] = fmaxf(m4[i & 3], x[i]);
@@ -210,11 +215,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           ssum *= exp2f((m - cm) * sc);
           m = cm;
         }
-        const float mc = m * sc;
-        float s4[4] = {0.f, 0.f, 0.f, 0.f};
+        // 2^(x sc - m sc), two lanes of f32x2 arithmetic per instruction
+        const float2 sc2 = make_float2(sc, sc), nmc = make_float2(-m * sc, -m * sc);
+        float2 s2a = make_float2(0.f, 0.f), s2b = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) s4[i & 3] += exp2f(fmaf(x[i], sc, -mc));
-        ssum += (s4[0] + s4[1]) + (s4[2] + s4[3]);
+        for (int i = 0; i < 32; i += 4) {
+          const float2 ea = __ffma2_rn(make_float2(x[i], x[i + 1]), sc2, nmc);
+          const float2 eb = __ffma2_rn(make_float2(x[i + 2], x[i + 3]), sc2, nmc);
+          s2a = __fadd2_rn(s2a, make_float2(exp2f(ea.x), exp2f(ea.y)));
+          s2b = __fadd2_rn(s2b, make_float2(exp2f(eb.x), exp2f(eb.y)));
+        }
+        ssum += (s2a.x + s2a.y) + (s2b.x + s2b.y);
       }
       tc_fence_before();
       mbar_arrive(&acc_empty[b]);
@@ -385,7 +396,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         par ^= 1;
         float* ls = lse_s + par * kTcMaxRows;
         for (int r = threadIdx.x; r < a.rows_pad; r += kTcEpi)
-          ls[r] = r < a.n_obs ? a.lse2[(size_t)u * a.n_obs + r] : INFINITY;
+          ls[r] = r < a.n_obs ? -a.lse2[(size_t)u * a.n_obs + r] : -INFINITY;
         mbar_arrive(lse_ready);  // release: the rows this thread staged
         if (!mbar_wait_bounded(lse_ready, changes & 1)) {
           ok = false;
@@ -394,8 +405,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         ++changes;
         cur_u = u;
       }
-      const float* ls = lse_s + par * kTcMaxRows;
-      float s4[4] = {0.f, 0.f, 0.f, 0.f};
+      const float* ls = lse_s + par * kTcMaxRows;  // minus the row log-sum-exps
+      const float2 sc2 = make_float2(a.scale2, a.scale2);
+      float2 s2a = make_float2(0.f, 0.f), s2b = make_float2(0.f, 0.f);
       for (int hh = 0; hh < 2; ++hh) {
         const int ncols = hh == 0 ? a.n_a : a.n_b;
         if (ncols == 0) continue;
@@ -416,17 +428,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
           for (int t = 0; t < 8; ++t) {
             const float4 lv = l4[t];
-            s4[0] += exp2f(fmaf(__uint_as_float(r[4 * t + 0]), a.scale2, -lv.x));
-            s4[1] += exp2f(fmaf(__uint_as_float(r[4 * t + 1]), a.scale2, -lv.y));
-            s4[2] += exp2f(fmaf(__uint_as_float(r[4 * t + 2]), a.scale2, -lv.z));
-            s4[3] += exp2f(fmaf(__uint_as_float(r[4 * t + 3]), a.scale2, -lv.w));
+            const float2 ea = __ffma2_rn(make_float2(__uint_as_float(r[4 * t]),
+                                                     __uint_as_float(r[4 * t + 1])),
+                                         sc2, make_float2(lv.x, lv.y));
+            const float2 eb = __ffma2_rn(make_float2(__uint_as_float(r[4 * t + 2]),
+                                                     __uint_as_float(r[4 * t + 3])),
+                                         sc2, make_float2(lv.z, lv.w));
+            s2a = __fadd2_rn(s2a, make_float2(exp2f(ea.x), exp2f(ea.y)));
+            s2b = __fadd2_rn(s2b, make_float2(exp2f(eb.x), exp2f(eb.y)));
           }
         }
         tc_fence_before();
         mbar_arrive(&acc_empty[hh]);
       }
       if (!ok) break;
-      const float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+      const float sum = (s2a.x + s2a.y) + (s2b.x + s2b.y);
       float* pb = part + (i & 1) * kTcGroups * 128;
       if (grp != 0) {
         pb[grp * 128 + row] = sum;
