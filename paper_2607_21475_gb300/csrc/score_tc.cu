@@ -89,6 +89,13 @@ struct TcArgs {
   int32_t* dev_status;
 };
 
+// max(a, b, c) in one instruction (three-input form of max.f32).
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
 __device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
   return (unsigned char*)(((uintptr_t)p + 1023) & ~(uintptr_t)1023);
 }
@@ -209,8 +216,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         float m4[4] = {x[0], x[1], x[2], x[3]};
 #pragma unroll
-        for (int i = 4; i < 32; ++i) m4[i & 3] = fmaxf(m4[i & 3], x[i]);
-        const float cm = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+        for (int i = 4; i < 32; i += 8) {
+          m4[0] = fmax3(m4[0], x[i], x[i + 1]);
+          m4[1] = fmax3(m4[1], x[i + 2], x[i + 3]);
+          m4[2] = fmax3(m4[2], x[i + 4], x[i + 5]);
+          m4[3] = fmax3(m4[3], x[i + 6], x[i + 7]);
+        }
+        const float cm = fmaxf(fmax3(m4[0], m4[1], m4[2]), m4[3]);
         if (cm > m) {
           ssum *= exp2f((m - cm) * sc);
           m = cm;
