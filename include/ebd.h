@@ -234,6 +234,28 @@ ebd_status ebd_certified_decode_static(ebd_dtype dtype, int32_t batch, int32_t n
                                        float* lse, float* var_hat, float* b_t, float* radius,
                                        int32_t* dev_status, void* stream);
 
+/*
+ * Deployed certificate and red-flag rule (the experimental setup of Section 5
+ * and its appendix; the rule cert >= tau = 1 of Section 5).  At each of the
+ * first six decode steps the radii r_t of Eq. (4) (delta = 0.1) of every
+ * `head_stride`-th query head (4 in the paper) of every layer are averaged per
+ * sequence; the certificate is the maximum of those step averages.  Call once
+ * per probed step, after that step's certified decodes of all layers.
+ *   radius      device [L, B, Hq] float32: the step's r_t, layer-major (pass
+ *               radius + l * B * Hq as the radius output of layer l's decode)
+ *   head_stride query heads h with h % head_stride == 0 enter the average
+ *   tau         red-flag threshold (1 in the paper)
+ *   first_step  nonzero: cert = this step's average (no earlier value is read)
+ *   step_mean   device [B] float32 out, nullable: this step's average
+ *   cert        device [B] float32 in/out: maximum over the probed steps so far
+ *   red_flag    device [B] int32 out, nullable: 1 when cert >= tau
+ * The average of each row is summed in a fixed order (deterministic).
+ */
+ebd_status ebd_certificate_update(const float* radius, int32_t n_layers, int32_t batch,
+                                  int32_t n_q_heads, int32_t head_stride, float tau,
+                                  int32_t first_step, float* step_mean, float* cert,
+                                  int32_t* red_flag, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -411,3 +411,23 @@ def hajek_decode(q, K_c, V_c, logw_c, delta: float = 0.1, eps0: float = 1e-9) ->
     return DecodeResult(y, np.array(lses), var, b_exact, b_bound,
                         certificate_radius(var, b_exact, yn, delta, eps0),
                         certificate_radius(var, b_bound, yn, delta, eps0), np.array(scs))
+
+
+# ---------------------------------------------------------------------------
+# Deployed certificate (Section 5 experimental setup and its appendix): the
+# radius of Eq. (4) at delta = 0.1 on every fourth query head of every layer
+# during the first six decode steps, averaged, then maximized over the steps;
+# the label-free red-flag rule is cert >= tau = 1.
+# ---------------------------------------------------------------------------
+def deployed_certificate(radii, head_stride=4):
+    """radii: [T, L, B, Hq] radii of T probed steps.  Returns (cert [B],
+    step_means [T, B]): the average over layers and heads h % head_stride == 0
+    at each step, and its maximum over the steps."""
+    r = np.asarray(radii, dtype=np.float64)
+    step_means = r[:, :, :, ::head_stride].mean(axis=(1, 3))
+    return step_means.max(axis=0), step_means
+
+
+def red_flag(cert, tau=1.0):
+    """The label-free rule: raise a sequence whose certificate reaches tau."""
+    return np.asarray(cert) >= tau

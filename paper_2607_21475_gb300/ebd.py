@@ -25,7 +25,7 @@ __all__ = [
     "ebd_status_string", "ebd_abi_version", "ebd_philox_uniforms", "ebd_score_workspace_bytes",
     "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
     "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
-    "ebd_certified_decode_static", "design_for",
+    "ebd_certified_decode_static", "ebd_certificate_update", "design_for",
     "CompactCache",
     "alloc_compact", "ABI_FUNCTIONS",
 ]
@@ -40,7 +40,7 @@ ABI_FUNCTIONS = (
     "ebd_status_string", "ebd_abi_version", "ebd_philox_uniforms", "ebd_score_workspace_bytes",
     "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
     "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
-    "ebd_certified_decode_static",
+    "ebd_certified_decode_static", "ebd_certificate_update",
 )
 
 
@@ -105,6 +105,8 @@ def lib():
                 ctypes.c_int, i32, i32, i32, i32, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                 i32, f32, f32, ctypes.c_int, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                 c_void_p, c_void_p]),
+            "ebd_certificate_update": (ctypes.c_int, [c_void_p, i32, i32, i32, i32, f32, i32,
+                                                      c_void_p, c_void_p, c_void_p, c_void_p]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -341,3 +343,18 @@ def ebd_certified_decode_static(Q: torch.Tensor, K_c: torch.Tensor, V_c: torch.T
         _ptr(radius, f, (B, Hq), "radius"), _ptr(dev_status, torch.int32, (1,), "dev_status"),
         _stream(stream)))
     return y, lse, var_hat, b_t, radius
+
+
+def ebd_certificate_update(radius: torch.Tensor, cert: torch.Tensor, first_step: bool,
+                           head_stride: int = 4, tau: float = 1.0, step_mean=None, red_flag=None,
+                           stream=None):
+    """One probed decode step of the deployed certificate: radius [L, B, Hq]
+    (this step's r_t of every layer) -> cert [B] = max over probed steps of the
+    mean over layers and every `head_stride`-th head; red_flag [B] = cert >= tau."""
+    L, B, Hq = radius.shape
+    f = torch.float32
+    _check("ebd_certificate_update", lib().ebd_certificate_update(
+        _ptr(radius, f, (L, B, Hq), "radius"), L, B, Hq, int(head_stride), float(tau),
+        1 if first_step else 0, _ptr(step_mean, f, (B,), "step_mean"), _ptr(cert, f, (B,), "cert"),
+        _ptr(red_flag, torch.int32, (B,), "red_flag"), _stream(stream)))
+    return cert

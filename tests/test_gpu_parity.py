@@ -350,3 +350,25 @@ def test_score_matches_oracle(E, B, H, R, N, d, dtype):
             ref = O.accumulated_attention_scores(q[b, h].double().numpy(), K[b, h].double().numpy())
             np.testing.assert_allclose(got[b, h], ref, rtol=1e-4, atol=1e-7 * R)
             assert abs(got[b, h].sum() - R) < 1e-3 * R
+
+
+# ------------------------------------------------------ deployed certificate
+@pytest.mark.parametrize("L,B,Hq,stride", [(28, 5, 28, 4), (3, 1, 7, 4), (2, 70, 32, 1)])
+def test_certificate_update_matches_oracle(E, L, B, Hq, stride):
+    g = torch.Generator().manual_seed(L * 1000 + B)
+    steps = torch.rand((6, L, B, Hq), generator=g) * 2.0
+    cert = torch.full((B,), 123.0, device=DEV)  # overwritten at the first step
+    mean = torch.empty((B,), device=DEV)
+    flag = torch.empty((B,), dtype=torch.int32, device=DEV)
+    means = []
+    for t in range(6):
+        E.ebd_certificate_update(steps[t].to(DEV), cert, first_step=(t == 0), head_stride=stride,
+                                 tau=1.0, step_mean=mean, red_flag=flag)
+        means.append(mean.cpu().double().numpy().copy())
+    torch.cuda.synchronize()
+    ref, ref_means = O.deployed_certificate(steps.double().numpy(), head_stride=stride)
+    np.testing.assert_allclose(np.stack(means), ref_means, rtol=2e-6, atol=0)
+    got = cert.cpu().double().numpy()
+    np.testing.assert_allclose(got, ref, rtol=2e-6, atol=0)
+    sure = np.abs(ref - 1.0) > 1e-5
+    assert np.array_equal(flag.cpu().numpy()[sure].astype(bool), O.red_flag(ref)[sure])

@@ -14,6 +14,7 @@ import scipy.stats
 import torch
 
 from oracle.ebd_oracle import (
+    deployed_certificate, red_flag,
     accumulated_attention_scores,
     certainty_set,
     certificate_radius,
@@ -448,3 +449,48 @@ def test_theorem1_topk_only_design_is_blind_to_evicted_values():
     slope1 = (errs[3] - errs[2]) / 10.0
     slope2 = (errs[2] - errs[1]) / 5.0
     assert abs(slope1 - slope2) < 0.05 * slope1
+
+
+# ---------------------------------------------------------------- deployed certificate
+# The deployed certificate (Section 5 setup): average the radius over every
+# fourth head of every layer at each of the first six decode steps, then take
+# the maximum over the steps.  The pins separate that order from its
+# alternatives (max over units, mean over steps, all heads).
+def test_certificate_constant_radii_give_the_constant():
+    r = np.full((6, 28, 3, 28), 0.37)
+    cert, means = deployed_certificate(r)
+    assert np.allclose(cert, 0.37) and np.allclose(means, 0.37)
+
+
+def test_certificate_reads_only_every_fourth_head():
+    r = np.zeros((6, 4, 2, 28))
+    r[:, :, :, 1::4] = 5.0  # heads 1, 5, 9, ... are not probed
+    r[:, :, :, 2::4] = 7.0
+    r[:, :, :, 3::4] = 9.0
+    cert, _ = deployed_certificate(r)
+    assert np.all(cert == 0.0)
+    r[2, 1, 0, 8] = 2.8  # one probed head of one layer at step 3, row 0
+    cert, means = deployed_certificate(r)
+    # 4 layers x 7 probed heads = 28 terms in the step average
+    assert cert[0] == pytest.approx(2.8 / 28) and cert[1] == 0.0
+    assert means[2, 0] == pytest.approx(0.1) and np.all(np.delete(means[:, 0], 2) == 0)
+
+
+def test_certificate_is_mean_over_units_then_max_over_steps():
+    r = np.zeros((6, 2, 1, 4))
+    r[0, 0, 0, 0] = 1.0   # step 1: units (layer, head 0) average to 0.5
+    r[1, :, 0, 0] = 0.2   # step 2: average 0.2
+    cert, means = deployed_certificate(r)
+    assert cert[0] == pytest.approx(0.5)           # not 1.0 (max over units)
+    assert means[:, 0].mean() != pytest.approx(cert[0])  # not the mean over steps
+    assert means[0, 0] == pytest.approx(0.5) and means[1, 0] == pytest.approx(0.2)
+
+
+def test_certificate_invariant_to_layer_order_and_red_flag_threshold():
+    rng = np.random.default_rng(3)
+    r = rng.gamma(2.0, 0.4, size=(6, 28, 4, 28))
+    cert, _ = deployed_certificate(r)
+    cert_perm, _ = deployed_certificate(r[:, rng.permutation(28)])
+    assert np.allclose(cert, cert_perm)
+    assert np.array_equal(red_flag(cert), cert >= 1.0)
+    assert red_flag(np.array([1.0]))[0] and not red_flag(np.array([0.999999]))[0]
