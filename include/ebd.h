@@ -235,6 +235,48 @@ ebd_status ebd_certified_decode_static(ebd_dtype dtype, int32_t batch, int32_t n
                                        int32_t* dev_status, void* stream);
 
 /*
+ * Decode-time growth of a compact cache: one new token per unit joins the
+ * cache with pi = 1 (log(1/pi) = 0), as every token generated after an
+ * eviction is kept until the next one.  For each unit with n_kept < capacity,
+ * row n_kept of K_c/V_c receives k_new/v_new, logw_c gets 0 and idx_c the
+ * token position; n_kept grows by one.  A full unit keeps its rows, counts the
+ * token in n_kept anyway and raises EBD_DEV_CAPACITY (as eviction overflow).
+ *   k_new, v_new  device [B,Hkv,d] (dtype), 16-byte aligned
+ *   positions     device [B] int32: position of the new token of each row
+ *   K_c, V_c, logw_c, idx_c, n_kept, capacity: the compact cache (updated)
+ *   dev_status    device int32, required
+ */
+ebd_status ebd_append(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads, int32_t head_dim,
+                      const void* k_new, const void* v_new, const int32_t* positions, void* K_c,
+                      void* V_c, float* logw_c, int32_t* idx_c, int32_t* n_kept,
+                      int32_t capacity, int32_t* dev_status, void* stream);
+
+/*
+ * Re-eviction of a resident compact cache: the tail draws redrawn every T_r
+ * decode steps (the block schedule of the anytime argument, Section 4 and its
+ * appendix).  Each unit's resident rows (the first min(n_kept_in, cap_in)
+ * rows, in cache order) are the context of a new eviction with `design`:
+ * certainty set (the first n_sink and last n_recent resident rows, the
+ * k_head highest scores), Eq. (2) probabilities on the tail, Poisson draws
+ * keyed by (design->seed; resident position / 4, kvh, design->layer, b) -- pass
+ * a fresh seed per round -- and compaction.  A token kept by both rounds has
+ * inclusion probability pi_1 pi_2 (the two Poisson designs compose), so the
+ * output log(1/pi) is logw_in + log(1/pi_2), and idx_out holds the original
+ * token positions (idx_in of the kept rows).
+ *   design->n_ctx must equal cap_in (the row stride of scores and the inputs)
+ *   scores        device [B,Hkv,cap_in] float32: importance of the resident rows
+ *   K_in, V_in, logw_in, idx_in, n_kept_in, cap_in: the resident cache (read)
+ *   K_out, V_out, logw_out, idx_out, n_kept_out, cap_out: the new cache;
+ *                 distinct from the inputs (EBD_ERR_INVALID otherwise)
+ *   dev_status    device int32, required (EBD_DEV_CAPACITY, EBD_DEV_NONFINITE)
+ */
+ebd_status ebd_reevict(const ebd_design* design, ebd_dtype dtype, const float* scores,
+                       const void* K_in, const void* V_in, const float* logw_in,
+                       const int32_t* idx_in, const int32_t* n_kept_in, int32_t cap_in,
+                       void* K_out, void* V_out, float* logw_out, int32_t* idx_out,
+                       int32_t* n_kept_out, int32_t cap_out, int32_t* dev_status, void* stream);
+
+/*
  * Deployed certificate and red-flag rule (the experimental setup of Section 5
  * and its appendix; the rule cert >= tau = 1 of Section 5).  At each of the
  * first six decode steps the radii r_t of Eq. (4) (delta = 0.1) of every

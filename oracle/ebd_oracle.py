@@ -431,3 +431,39 @@ def deployed_certificate(radii, head_stride=4):
 def red_flag(cert, tau=1.0):
     """The label-free rule: raise a sequence whose certificate reaches tau."""
     return np.asarray(cert) >= tau
+
+
+# ---------------------------------------------------------------------------
+# Decode-time growth and re-eviction of a compact cache.  A token generated
+# after an eviction enters with pi = 1.  Redrawing the tail every T_r steps
+# (the block schedule of the anytime argument, Section 4 and its appendix)
+# evicts the resident cache again; a token kept by both rounds has inclusion
+# probability pi_1 pi_2 (two independent Poisson designs), so log(1/pi) adds.
+# ---------------------------------------------------------------------------
+def append_token(K_c, V_c, logw_c, idx_c, k_new, v_new, position):
+    """Resident cache of one unit plus one new token with log(1/pi) = 0."""
+    return (np.concatenate([K_c, np.asarray(k_new)[None]], 0),
+            np.concatenate([V_c, np.asarray(v_new)[None]], 0),
+            np.concatenate([logw_c, [0.0]]), np.concatenate([idx_c, [position]]).astype(np.int64))
+
+
+@dataclass
+class ReevictResult:
+    inner: EvictResult      # the second-round eviction over the resident rows
+    idx: np.ndarray         # original token positions of the kept rows
+    logw: np.ndarray        # log(1/pi_1) + log(1/pi_2) of the kept rows
+    K_c: np.ndarray
+    V_c: np.ndarray
+    n_kept: int
+
+
+def reevict_unit(K_c, V_c, logw_c, idx_c, scores, *, n_sink, n_recent, k_head, budget_tokens,
+                 eps, seed, layer, b, kvh, capacity, bisect_iters=200) -> ReevictResult:
+    """Evict the resident rows of one unit again (they are the new context, in
+    cache order) and compose the two designs."""
+    r = evict_unit(K_c, V_c, scores, n_sink=n_sink, n_recent=n_recent, k_head=k_head,
+                   budget_tokens=budget_tokens, eps=eps, seed=seed, layer=layer, b=b, kvh=kvh,
+                   capacity=capacity, bisect_iters=bisect_iters)
+    logw_c = np.asarray(logw_c, dtype=np.float64)
+    idx_c = np.asarray(idx_c)
+    return ReevictResult(r, idx_c[r.idx], logw_c[r.idx] + r.logw, r.K_c, r.V_c, r.n_kept)

@@ -703,7 +703,6 @@ void fast_decode_plan(DecodePlan& p, long long units, int group, int head_dim) {
                align_up((size_t)(units + W) * group * rec_floats(head_dim) * sizeof(float), 256);
 }
 
-static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
 bool fast_decode_usable(const DecodeArgs& a, const ReduceArgs& r, int units) {
   return aligned16(a.Kc) && aligned16(a.Vc) && aligned16(a.logw) && aligned16(a.Q) &&

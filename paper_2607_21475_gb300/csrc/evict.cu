@@ -31,8 +31,9 @@ constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kMaxCtx = 1 << 20;
 
 struct SelectArgs {
-  const float* scores;  // [units, N]
-  int n_ctx;
+  const float* scores;  // [units, n_ctx]
+  int n_ctx;            // row stride of scores (and pi_out, mask_out)
+  const int32_t* n_len; // nullable [units]: context length of each unit (<= n_ctx)
   int n_kv_heads;
   int layer;
   uint64_t seed;
@@ -147,10 +148,11 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
   const int unit = blockIdx.x;
   const int b = unit / a.n_kv_heads;
   const int kvh = unit - b * a.n_kv_heads;
-  const int N = a.n_ctx;
+  const int Nrow = a.n_ctx;
+  const int N = a.n_len ? min(max(__ldg(a.n_len + unit), 0), Nrow) : Nrow;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int words = (N + 31) >> 5;
-  const float* s = a.scores + (size_t)unit * N;
+  const float* s = a.scores + (size_t)unit * Nrow;
 
   const int ns = min(a.n_sink, N);
   const int rs = max(N - a.n_recent, 0);  // first protected trailing position
@@ -329,8 +331,8 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
         if (!isfinite(v)) { bad = true; v = 0.f; }
         pi = tail_pi(v, mode, c, eps);
       }
-      if (a.pi_out) a.pi_out[(size_t)unit * N + i] = pi;
-      if (a.mask_out) a.mask_out[(size_t)unit * N + i] = cert ? 1 : 0;
+      if (a.pi_out) a.pi_out[(size_t)unit * Nrow + i] = pi;
+      if (a.mask_out) a.mask_out[(size_t)unit * Nrow + i] = cert ? 1 : 0;
       if (compact) {
         const float u = word_to_uniform(draw_word(a.seed, a.layer, b, kvh, i));
         keep = cert || (u < pi);
@@ -497,9 +499,10 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
   const int unit = blockIdx.x;
   const int b = unit / a.n_kv_heads;
   const int kvh = unit - b * a.n_kv_heads;
-  const int N = a.n_ctx;
+  const int Nrow = a.n_ctx;
+  const int N = a.n_len ? min(max(__ldg(a.n_len + unit), 0), Nrow) : Nrow;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const float* sp = a.scores + (size_t)unit * N;
+  const float* sp = a.scores + (size_t)unit * Nrow;
   const int ns = min(a.n_sink, N);
   const int rs = max(N - a.n_recent, 0);
   const int n_prot = ns + (N - rs) - max(0, ns - rs);
@@ -779,8 +782,8 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
       if (!((valid >> (4 * g + r)) & 1u)) continue;
       const bool ct = (cert >> (4 * g + r)) & 1u;
       const float pi = ct ? 1.f : tail_pi(vv[r], mode, c, eps);
-      if (a.pi_out) a.pi_out[(size_t)unit * N + i] = pi;
-      if (a.mask_out) a.mask_out[(size_t)unit * N + i] = ct ? 1 : 0;
+      if (a.pi_out) a.pi_out[(size_t)unit * Nrow + i] = pi;
+      if (a.mask_out) a.mask_out[(size_t)unit * Nrow + i] = ct ? 1 : 0;
       if (compact && (ct || word_to_uniform(wr[r]) < pi)) keep |= 1u << (4 * g + r);
     }
   }
@@ -880,7 +883,7 @@ int sm_count() {
   return cached[dev];
 }
 
-static ebd_status check_design(const ebd_design* d) {
+ebd_status check_design(const ebd_design* d) {
   if (!d) return EBD_ERR_INVALID;
   if (d->batch < 1 || d->n_kv_heads < 1 || d->n_ctx < 1 || d->n_ctx > kMaxCtx) return EBD_ERR_INVALID;
   if ((long long)d->batch * d->n_kv_heads > 0x7fffffffLL) return EBD_ERR_INVALID;
@@ -890,12 +893,13 @@ static ebd_status check_design(const ebd_design* d) {
   return EBD_OK;
 }
 
-static ebd_status launch_select(const ebd_design* d, const float* scores, float* pi,
-                                uint8_t* mask, int32_t* idx_c, float* logw_c, int32_t* n_kept,
-                                int cap, int32_t* dev_status, cudaStream_t stream) {
+ebd_status launch_select(const ebd_design* d, const float* scores, const int32_t* n_len,
+                         float* pi, uint8_t* mask, int32_t* idx_c, float* logw_c, int32_t* n_kept,
+                         int cap, int32_t* dev_status, cudaStream_t stream) {
   SelectArgs a;
   a.scores = scores;
   a.n_ctx = d->n_ctx;
+  a.n_len = n_len;
   a.n_kv_heads = d->n_kv_heads;
   a.layer = d->layer;
   a.seed = d->seed;
@@ -916,29 +920,28 @@ static ebd_status launch_select(const ebd_design* d, const float* scores, float*
   const int units = d->batch * d->n_kv_heads;
   const int groups = (d->n_ctx + kGroupTokens - 1) / kGroupTokens;
   if (groups <= kRegMaxGroups) {
+    // the limit is set on every launch: with the kernel's static shared memory
+    // even 48 KB of dynamic memory is above the default
     const size_t smem = (size_t)groups * kRegThreads * sizeof(float4) + kRegWarps * 256 * 4;
-    if (smem > 48 * 1024 &&
-        cudaFuncSetAttribute(evict_select_smem_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(evict_select_smem_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem) != cudaSuccess)
       return EBD_ERR_CUDA;
     evict_select_smem_kernel<<<units, kRegThreads, smem, stream>>>(a, groups);
     return launch_status();
   }
   const size_t smem = (size_t)((d->n_ctx + 31) / 32) * 4;
-  if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(evict_select_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return EBD_ERR_CUDA;
-  }
+  if (cudaFuncSetAttribute(evict_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem) != cudaSuccess)
+    return EBD_ERR_CUDA;
   evict_select_kernel<<<units, kSelThreads, smem, stream>>>(a);
   return launch_status();
 }
 
-static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
-static ebd_status launch_gather(const ebd_design* d, ebd_dtype dtype, const void* K,
-                                const void* V, const int32_t* idx_c, const int32_t* n_kept,
-                                int cap, void* K_c, void* V_c, cudaStream_t s) {
+ebd_status launch_gather(const ebd_design* d, ebd_dtype dtype, const void* K, const void* V,
+                         const int32_t* idx_c, const int32_t* n_kept, int cap, void* K_c,
+                         void* V_c, cudaStream_t s) {
   const int eb = dtype == EBD_F32 ? 4 : 2;
   const int cpr = d->head_dim * eb / 16;
   const int units = d->batch * d->n_kv_heads;
@@ -991,7 +994,7 @@ extern "C" ebd_status ebd_compute_pi(const ebd_design* design, const float* scor
   ebd_status st = check_design(design);
   if (st != EBD_OK) return st;
   if (!scores || !pi) return EBD_ERR_INVALID;
-  return launch_select(design, scores, pi, certain_mask, nullptr, nullptr, nullptr, 0,
+  return launch_select(design, scores, nullptr, pi, certain_mask, nullptr, nullptr, nullptr, 0,
                        dev_status, (cudaStream_t)stream);
 }
 
@@ -1031,7 +1034,8 @@ extern "C" ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const
     if (st != EBD_OK) return st;
     sc = ws_scores;
   }
-  st = launch_select(design, sc, nullptr, nullptr, idx_c, logw_c, n_kept, capacity, dev_status, s);
+  st = launch_select(design, sc, nullptr, nullptr, nullptr, idx_c, logw_c, n_kept, capacity,
+                     dev_status, s);
   if (st != EBD_OK) return st;
   return launch_gather(design, dtype, K, V, idx_c, n_kept, capacity, K_c, V_c, s);
 }
@@ -1042,7 +1046,7 @@ extern "C" ebd_status ebd_select(const ebd_design* design, const float* scores, 
   ebd_status st = check_design(design);
   if (st != EBD_OK) return st;
   if (!scores || !idx_c || !logw_c || !n_kept || !dev_status || capacity < 1) return EBD_ERR_INVALID;
-  return launch_select(design, scores, nullptr, nullptr, idx_c, logw_c, n_kept, capacity,
+  return launch_select(design, scores, nullptr, nullptr, nullptr, idx_c, logw_c, n_kept, capacity,
                        dev_status, (cudaStream_t)stream);
 }
 

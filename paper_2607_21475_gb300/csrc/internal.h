@@ -19,6 +19,24 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // Number of SMs of the current device (cached per device).
 int sm_count();
 
+// Design validation shared by the eviction entry points (evict.cu).
+ebd_status check_design(const ebd_design* d);
+
+// E1-E4a for every unit (evict.cu): certainty set, pi, draws, index
+// compaction.  n_len (nullable, device [units]) gives each unit's context
+// length when it is below the row stride d->n_ctx of `scores`.
+ebd_status launch_select(const ebd_design* d, const float* scores, const int32_t* n_len,
+                         float* pi, uint8_t* mask, int32_t* idx_c, float* logw_c, int32_t* n_kept,
+                         int cap, int32_t* dev_status, cudaStream_t stream);
+
+// E4b for every unit (evict.cu): rows K[idx_c[p]], V[idx_c[p]] (row stride
+// d->n_ctx) to K_c[p], V_c[p] for p < min(n_kept, cap).
+ebd_status launch_gather(const ebd_design* d, ebd_dtype dtype, const void* K, const void* V,
+                         const int32_t* idx_c, const int32_t* n_kept, int cap, void* K_c,
+                         void* V_c, cudaStream_t s);
+
+bool aligned16(const void* p);
+
 // E0: accumulated attention scores into `scores` using `workspace` for the
 // per-row log-sum-exp.  Arguments validated by the caller; dev_status nullable.
 ebd_status launch_score(ebd_dtype dtype, int batch, int n_kv_heads, int head_dim, int n_ctx,

@@ -25,7 +25,8 @@ __all__ = [
     "ebd_status_string", "ebd_abi_version", "ebd_philox_uniforms", "ebd_score_workspace_bytes",
     "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
     "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
-    "ebd_certified_decode_static", "ebd_certificate_update", "design_for",
+    "ebd_certified_decode_static", "ebd_certificate_update", "ebd_append", "ebd_reevict",
+    "design_for",
     "CompactCache",
     "alloc_compact", "ABI_FUNCTIONS",
 ]
@@ -40,7 +41,7 @@ ABI_FUNCTIONS = (
     "ebd_status_string", "ebd_abi_version", "ebd_philox_uniforms", "ebd_score_workspace_bytes",
     "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
     "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
-    "ebd_certified_decode_static", "ebd_certificate_update",
+    "ebd_certified_decode_static", "ebd_certificate_update", "ebd_append", "ebd_reevict",
 )
 
 
@@ -107,6 +108,12 @@ def lib():
                 c_void_p, c_void_p]),
             "ebd_certificate_update": (ctypes.c_int, [c_void_p, i32, i32, i32, i32, f32, i32,
                                                       c_void_p, c_void_p, c_void_p, c_void_p]),
+            "ebd_append": (ctypes.c_int, [ctypes.c_int, i32, i32, i32, c_void_p, c_void_p,
+                                          c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                          c_void_p, i32, c_void_p, c_void_p]),
+            "ebd_reevict": (ctypes.c_int, [P, ctypes.c_int, c_void_p, c_void_p, c_void_p, c_void_p,
+                                           c_void_p, c_void_p, i32, c_void_p, c_void_p, c_void_p,
+                                           c_void_p, c_void_p, i32, c_void_p, c_void_p]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -358,3 +365,43 @@ def ebd_certificate_update(radius: torch.Tensor, cert: torch.Tensor, first_step:
         1 if first_step else 0, _ptr(step_mean, f, (B,), "step_mean"), _ptr(cert, f, (B,), "cert"),
         _ptr(red_flag, torch.int32, (B,), "red_flag"), _stream(stream)))
     return cert
+
+
+def ebd_append(cc: "CompactCache", k_new: torch.Tensor, v_new: torch.Tensor,
+               positions: torch.Tensor, stream=None) -> "CompactCache":
+    """Append one token per unit (pi = 1) to the compact cache `cc` in place.
+    k_new, v_new: [B, Hkv, d]; positions: [B] int32 token positions."""
+    B, H, cap, d = cc.K_c.shape
+    dt = _dtype_code(cc.K_c)
+    _check("ebd_append", lib().ebd_append(
+        dt, B, H, d, _ptr(k_new, cc.K_c.dtype, (B, H, d), "k_new"),
+        _ptr(v_new, cc.K_c.dtype, (B, H, d), "v_new"), _ptr(positions, torch.int32, (B,), "positions"),
+        _ptr(cc.K_c, name="K_c"), _ptr(cc.V_c, cc.K_c.dtype, (B, H, cap, d), "V_c"),
+        _ptr(cc.logw_c, torch.float32, (B, H, cap), "logw_c"),
+        _ptr(cc.idx_c, torch.int32, (B, H, cap), "idx_c"),
+        _ptr(cc.n_kept, torch.int32, (B, H), "n_kept"), cap,
+        _ptr(cc.dev_status, torch.int32, (1,), "dev_status"), _stream(stream)))
+    return cc
+
+
+def ebd_reevict(design: EbdDesign, scores: torch.Tensor, cc_in: "CompactCache",
+                out: "CompactCache", stream=None) -> "CompactCache":
+    """Evict the resident cache `cc_in` again into `out` (distinct buffers):
+    scores [B, Hkv, cap_in] for the resident rows; design.n_ctx == cap_in."""
+    B, H, cap_in, d = cc_in.K_c.shape
+    cap_out = out.K_c.shape[2]
+    dt = _dtype_code(cc_in.K_c)
+    f = torch.float32
+    _check("ebd_reevict", lib().ebd_reevict(
+        ctypes.byref(design), dt, _ptr(scores, f, (B, H, cap_in), "scores"),
+        _ptr(cc_in.K_c, name="K_in"), _ptr(cc_in.V_c, cc_in.K_c.dtype, (B, H, cap_in, d), "V_in"),
+        _ptr(cc_in.logw_c, f, (B, H, cap_in), "logw_in"),
+        _ptr(cc_in.idx_c, torch.int32, (B, H, cap_in), "idx_in"),
+        _ptr(cc_in.n_kept, torch.int32, (B, H), "n_kept_in"), cap_in,
+        _ptr(out.K_c, cc_in.K_c.dtype, (B, H, cap_out, d), "K_out"),
+        _ptr(out.V_c, cc_in.K_c.dtype, (B, H, cap_out, d), "V_out"),
+        _ptr(out.logw_c, f, (B, H, cap_out), "logw_out"),
+        _ptr(out.idx_c, torch.int32, (B, H, cap_out), "idx_out"),
+        _ptr(out.n_kept, torch.int32, (B, H), "n_kept_out"), cap_out,
+        _ptr(out.dev_status, torch.int32, (1,), "dev_status"), _stream(stream)))
+    return out

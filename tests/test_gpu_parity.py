@@ -8,7 +8,7 @@ import pytest
 import torch
 
 from oracle import ebd_oracle as O
-from tests.parity import compare_decode_heads, compare_evict_unit, oracle_unit
+from tests.parity import TIE_BAND, compare_decode_heads, compare_evict_unit, oracle_unit
 
 pytestmark = pytest.mark.gpu
 
@@ -372,3 +372,86 @@ def test_certificate_update_matches_oracle(E, L, B, Hq, stride):
     np.testing.assert_allclose(got, ref, rtol=2e-6, atol=0)
     sure = np.abs(ref - 1.0) > 1e-5
     assert np.array_equal(flag.cpu().numpy()[sure].astype(bool), O.red_flag(ref)[sure])
+
+
+# ------------------------------------------------------- append and re-eviction
+def bits_t(t):
+    """Bit patterns of a device tensor (bf16 compared as int16)."""
+    return t.view(torch.int16) if t.dtype == torch.bfloat16 else t
+
+def test_append_then_reevict_then_decode_matches_oracle(E):
+    """A compact cache grows by 40 decode tokens (pi = 1), is evicted again with
+    fresh draws (log(1/pi) composes), and the certified decode runs on the
+    result; each step against the oracle on the same inputs."""
+    from paper_2607_21475_gb300.workloads import WORKLOADS, make_layer_inputs
+    w = WORKLOADS["qwen7b_16k_b25"].with_(batch=2, n_ctx=3000)
+    layer = 2
+    inp = make_layer_inputs(w, layer, DEV)
+    B, H, G, d, N = w.batch, w.n_kv_heads, w.group, w.head_dim, w.n_ctx
+    n_app = 40
+    cap = w.capacity + n_app
+    des = _design(E, B, H, G, d, N, layer, w.philox_seed, w.k_head, w.budget_tokens)
+    cc = E.alloc_compact(B, H, cap, d, w.torch_dtype, DEV)
+    E.ebd_evict(des, inp["K"], inp["V"], inp["scores"], None, cc)
+    torch.cuda.synchronize()
+    n0 = cc.n_kept.clone()
+    g = torch.Generator().manual_seed(17)
+    k_new = torch.randn((n_app, B, H, d), generator=g).to(w.torch_dtype)
+    v_new = torch.randn((n_app, B, H, d), generator=g).to(w.torch_dtype)
+    for t in range(n_app):
+        pos = torch.full((B,), N + t, dtype=torch.int32, device=DEV)
+        E.ebd_append(cc, k_new[t].to(DEV), v_new[t].to(DEV), pos)
+    torch.cuda.synchronize()
+    assert cc.dev_status.item() == 0
+    assert torch.equal(cc.n_kept, n0 + n_app)
+    for b in range(B):
+        for h in range(H):
+            n = int(n0[b, h])
+            assert torch.equal(bits_t(cc.K_c[b, h, n:n + n_app]), bits_t(k_new[:, b, h].to(DEV)))
+            assert torch.equal(bits_t(cc.V_c[b, h, n:n + n_app]), bits_t(v_new[:, b, h].to(DEV)))
+            assert torch.all(cc.logw_c[b, h, n:n + n_app] == 0)
+            assert torch.equal(cc.idx_c[b, h, n:n + n_app].cpu(), torch.arange(N, N + n_app, dtype=torch.int32))
+    # re-evict with new scores and a new seed
+    scores2 = torch.exp(torch.randn((B, H, cap), generator=g) * 1.5).to(DEV)
+    budget2 = w.budget_tokens // 2
+    cap2 = w.with_(budget=budget2 / N).capacity
+    des2 = _design(E, B, H, G, d, cap, layer, w.philox_seed + 1, budget2 // 5, budget2)
+    out = E.alloc_compact(B, H, cap2, d, w.torch_dtype, DEV)
+    E.ebd_reevict(des2, scores2, cc, out)
+    torch.cuda.synchronize()
+    assert out.dev_status.item() == 0
+    y = torch.empty((B, H * G, d), dtype=torch.float32, device=DEV)
+    lse, var, bt, r = (torch.empty((B, H * G), dtype=torch.float32, device=DEV) for _ in range(4))
+    E.ebd_certified_decode(inp["Q"], out.K_c, out.V_c, out.logw_c, out.n_kept, y, lse, var, bt, r)
+    torch.cuda.synchronize()
+    ties = 0
+    for b in range(B):
+        for h in range(H):
+            n = int(cc.n_kept[b, h])
+            Kr = cc.K_c[b, h, :n].double().cpu().numpy()
+            Vr = cc.V_c[b, h, :n].double().cpu().numpy()
+            lw = cc.logw_c[b, h, :n].double().cpu().numpy()
+            ix = cc.idx_c[b, h, :n].cpu().numpy()
+            ref = O.reevict_unit(Kr, Vr, lw, ix, scores2[b, h, :n].cpu().numpy(), n_sink=w.n_sink,
+                                 n_recent=w.n_recent, k_head=des2.k_head, budget_tokens=budget2,
+                                 eps=w.eps, seed=w.philox_seed + 1, layer=layer, b=b, kvh=h,
+                                 capacity=cap2)
+            inner = ref.inner
+            near = (~inner.certain) & (np.abs(inner.u - inner.pi) < TIE_BAND)
+            ties += int(near.sum())
+            m = min(int(out.n_kept[b, h]), cap2)
+            got_pos = set(np.searchsorted(ix, out.idx_c[b, h, :m].cpu().numpy()).tolist())
+            diff = got_pos ^ set(inner.idx.tolist())
+            assert all(near[i] for i in diff), f"unit {(b, h)}: kept sets differ at {sorted(diff)[:8]}"
+            if diff:
+                continue
+            assert np.array_equal(out.idx_c[b, h, :m].cpu().numpy(), ref.idx)
+            np.testing.assert_allclose(out.logw_c[b, h, :m].double().cpu().numpy(), ref.logw,
+                                       rtol=2e-5, atol=4e-6)
+            assert torch.equal(bits_t(out.K_c[b, h, :m]), bits_t(cc.K_c[b, h, inner.idx]))
+            dec = O.hajek_decode(inp["Q"][b, h * G:(h + 1) * G].double().cpu().numpy(), ref.K_c,
+                                 ref.V_c, ref.logw)
+            sl = slice(h * G, (h + 1) * G)
+            compare_decode_heads(dec, *(t[b, sl].double().cpu().numpy() for t in (y, lse, var, bt, r)),
+                                 False)
+    print("near ties", ties)

@@ -14,7 +14,7 @@ import scipy.stats
 import torch
 
 from oracle.ebd_oracle import (
-    deployed_certificate, red_flag,
+    deployed_certificate, red_flag, append_token, reevict_unit,
     accumulated_attention_scores,
     certainty_set,
     certificate_radius,
@@ -494,3 +494,78 @@ def test_certificate_invariant_to_layer_order_and_red_flag_threshold():
     assert np.allclose(cert, cert_perm)
     assert np.array_equal(red_flag(cert), cert >= 1.0)
     assert red_flag(np.array([1.0]))[0] and not red_flag(np.array([0.999999]))[0]
+
+
+
+# ---------------------------------------------------------------- append and re-eviction
+# A token generated after an eviction enters with pi = 1; re-evicting the
+# resident cache composes two independent Poisson designs (pi = pi_1 pi_2, so
+# log(1/pi) adds).  Pins: a budget that covers the resident cache reproduces
+# it, appended recent tokens are certain, and the composed weights keep the
+# Horvitz-Thompson total unbiased over both rounds' draws.
+def _resident(n=200, d=8, seed=1, budget=60, cap=128):
+    rng = np.random.default_rng(seed)
+    K = rng.standard_normal((n, d))
+    V = rng.standard_normal((n, d))
+    s = rng.lognormal(0.0, 1.5, n)
+    r = evict_unit(K, V, s, n_sink=4, n_recent=8, k_head=6, budget_tokens=budget, eps=1e-6,
+                   seed=seed, layer=0, b=0, kvh=0, capacity=cap)
+    return r, rng
+
+
+def test_reevict_with_a_covering_budget_reproduces_the_cache():
+    r, rng = _resident()
+    n = r.n_kept
+    s2 = rng.lognormal(0.0, 1.0, n)
+    rr = reevict_unit(r.K_c, r.V_c, r.logw, r.idx, s2, n_sink=4, n_recent=8, k_head=6,
+                      budget_tokens=n + 5, eps=1e-6, seed=9, layer=0, b=0, kvh=0, capacity=256)
+    assert rr.n_kept == n
+    assert np.array_equal(rr.idx, r.idx) and np.allclose(rr.logw, r.logw)
+    assert np.array_equal(rr.K_c, r.K_c) and np.array_equal(rr.V_c, r.V_c)
+
+
+def test_appended_tokens_enter_certain_and_survive_reeviction():
+    r, rng = _resident()
+    K_c, V_c, lw, idx = r.K_c, r.V_c, r.logw, r.idx
+    for t in range(5):
+        K_c, V_c, lw, idx = append_token(K_c, V_c, lw, idx, rng.standard_normal(8),
+                                         rng.standard_normal(8), 200 + t)
+    assert np.all(lw[-5:] == 0.0) and list(idx[-5:]) == [200, 201, 202, 203, 204]
+    s2 = rng.lognormal(0.0, 1.0, len(idx))
+    rr = reevict_unit(K_c, V_c, lw, idx, s2, n_sink=4, n_recent=8, k_head=6, budget_tokens=40,
+                      eps=1e-6, seed=3, layer=0, b=0, kvh=0, capacity=256)
+    # the recency window of the resident order holds the appended tokens: certain, kept, pi = 1
+    assert set(range(200, 205)) <= set(rr.idx.tolist())
+    kept_new = np.isin(rr.idx, np.arange(200, 205))
+    assert np.all(rr.logw[kept_new] == 0.0)
+    # a token kept twice carries both rounds' log(1/pi)
+    pos = {int(t): k for k, t in enumerate(idx)}
+    for t, l in zip(rr.idx, rr.logw):
+        j = pos[int(t)]
+        assert l == pytest.approx(lw[j] + (-np.log(rr.inner.pi[j])), rel=1e-12, abs=1e-12)
+
+
+def test_composed_weights_keep_the_total_unbiased_over_two_rounds():
+    # Horvitz-Thompson total of x over both rounds' draws: E[sum_kept x e^{logw}] = sum x
+    rng = np.random.default_rng(5)
+    n, d = 30, 2
+    K = rng.standard_normal((n, d))
+    V = rng.standard_normal((n, d))
+    s1 = rng.lognormal(0.0, 1.0, n)
+    s2_full = rng.lognormal(0.0, 1.0, n)
+    x = rng.uniform(0.5, 2.0, n)
+    est, one_round = [], []
+    for seed in range(3000):
+        r = evict_unit(K, V, s1, n_sink=2, n_recent=2, k_head=2, budget_tokens=16, eps=1e-6,
+                       seed=seed, layer=0, b=0, kvh=0, capacity=n)
+        rr = reevict_unit(r.K_c, r.V_c, r.logw, r.idx, s2_full[r.idx], n_sink=2, n_recent=2,
+                          k_head=1, budget_tokens=9, eps=1e-6, seed=10_000 + seed, layer=1, b=0,
+                          kvh=0, capacity=n)
+        est.append(np.sum(x[rr.idx] * np.exp(rr.logw)))
+        one_round.append(np.sum(x[rr.idx] * np.exp(rr.inner.logw)))
+    est = np.asarray(est)
+    se = est.std(ddof=1) / np.sqrt(len(est))
+    assert abs(est.mean() - x.sum()) < 4 * se
+    # the second round's weights alone (the first round forgotten) are biased low
+    one_round = np.asarray(one_round)
+    assert one_round.mean() < x.sum() - 4 * one_round.std(ddof=1) / np.sqrt(len(one_round))
