@@ -68,6 +68,18 @@ typedef enum { EBD_RANGE_BOUND = 0, EBD_RANGE_EXACT = 1 } ebd_range_mode;
 #define EBD_DEV_TIMEOUT 0x4   /* an in-kernel pipeline wait hit its bound and the
                                  kernel returned early; outputs are unspecified      */
 
+/* Tail design.  POISSON: independent Bernoulli(pi_i) draws (Section 3.3).
+ * SYSTEMATIC: fixed-size systematic sampling at the same pi_i (Hajek 1964;
+ * the exact-budget variant of Section 5): the tail in token order, cumulative
+ * sums C_i of pi in units of 2^-40 (each pi_i rounded to the nearest unit),
+ * one uniform u = (x >> 8) 2^-24 per unit with x = word 0 of Philox4x32-10 at
+ * counter (2^32 - 1, kvh, layer, b); token i is kept when an integer lies in
+ * (C_{i-1} - u, C_i - u].  Its inclusion probability is pi_i and the tail
+ * sample has floor or ceil of sum pi tokens; joint inclusion probabilities do
+ * not factor, so the certificate's variance form is then an approximation.
+ * Supported for N <= 32768. */
+typedef enum { EBD_SAMPLING_POISSON = 0, EBD_SAMPLING_SYSTEMATIC = 1 } ebd_sampling;
+
 /* Design of one layer's eviction (Section 3.3 and Appendix B of the paper). */
 typedef struct {
   int32_t batch;         /* B                                                    */
@@ -83,6 +95,7 @@ typedef struct {
   int32_t budget_tokens; /* B_t: expected retained tokens per unit (A + tail)    */
   int32_t bisect_iters;  /* bisection steps for the scale c of Eq. (2), 1..200   */
   float eps;             /* probability floor, 1e-6 in the paper                 */
+  int32_t sampling;      /* ebd_sampling of the tail (POISSON = 0)               */
 } ebd_design;
 
 /* Human-readable name of a status code (static string, never NULL). */

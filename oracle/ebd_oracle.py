@@ -467,3 +467,51 @@ def reevict_unit(K_c, V_c, logw_c, idx_c, scores, *, n_sink, n_recent, k_head, b
     logw_c = np.asarray(logw_c, dtype=np.float64)
     idx_c = np.asarray(idx_c)
     return ReevictResult(r, idx_c[r.idx], logw_c[r.idx] + r.logw, r.K_c, r.V_c, r.n_kept)
+
+
+# ---------------------------------------------------------------------------
+# Fixed-size systematic sampling at the same inclusion probabilities (Hajek
+# 1964; the exact-budget variant the paper measures in Section 5): the tail in
+# token order, cumulative sums C_i of pi, one uniform u per unit; token i is
+# kept when an integer lies in (C_{i-1} - u, C_i - u].  Each pi_i is first
+# rounded to the nearest multiple of 2^-40 and the sums are exact integers, so
+# every implementation takes the same decision.  The uniform is word 0 of
+# Philox4x32-10 at counter (2^32 - 1, kvh, layer, b), u = (x >> 8) 2^-24.
+# ---------------------------------------------------------------------------
+SYSTEMATIC_SCALE = 1 << 40
+
+
+def systematic_uniform(seed: int, layer: int, b: int, kvh: int) -> int:
+    """The unit's uniform, as an integer multiple of 2^-24."""
+    key = (seed & 0xFFFFFFFF, (seed >> 32) & 0xFFFFFFFF)
+    w = philox4x32_10((0xFFFFFFFF, kvh & 0xFFFFFFFF, layer & 0xFFFFFFFF, b & 0xFFFFFFFF), key)
+    return int(w[0]) >> 8
+
+
+def systematic_keep(pi, certain, u24: int):
+    """Kept mask of the systematic design; pi is rounded to float32 first (the
+    precision the probabilities are stored in), then to units of 2^-40."""
+    pi32 = np.asarray(pi, dtype=np.float32).astype(np.float64)
+    units = np.rint(pi32 * SYSTEMATIC_SCALE).astype(np.int64)
+    u = u24 << 16
+    keep = np.asarray(certain, dtype=bool).copy()
+    C = 0
+    for i in np.flatnonzero(~np.asarray(certain, dtype=bool)):
+        Cp = C
+        C += int(units[i])
+        if (C - u) // SYSTEMATIC_SCALE != (Cp - u) // SYSTEMATIC_SCALE:
+            keep[i] = True
+    return keep
+
+
+def evict_unit_systematic(K, V, scores, *, n_sink, n_recent, k_head, budget_tokens, eps, seed,
+                          layer, b, kvh, capacity, bisect_iters=200):
+    """evict_unit with the systematic tail design."""
+    scores = np.asarray(scores)
+    certain, topk = certainty_set(scores, n_sink, n_recent, k_head)
+    pi, c, m = inclusion_probabilities(scores, certain, budget_tokens, eps, bisect_iters)
+    u24 = systematic_uniform(seed, layer, b, kvh)
+    keep = systematic_keep(pi, certain, u24)
+    K_c, V_c, logw, idx, n_kept = compact(K, V, keep, pi, capacity)
+    return EvictResult(certain, topk, pi, c, m, np.full(len(scores), u24 * 2.0 ** -24),
+                       np.zeros(len(scores), dtype=np.uint32), keep, idx, logw, K_c, V_c, n_kept)

@@ -51,6 +51,7 @@ struct SelectArgs {
   int cap;
   int32_t* dev_status;  // nullable
   int vec4;             // scores rows start 16-byte aligned (float4 loads)
+  int systematic;       // tail design: 0 Poisson, 1 systematic at the same pi
 };
 
 struct BlockScratch {
@@ -378,6 +379,7 @@ constexpr int kRegMaxGroups = 8;
 constexpr int kGroupTokens = 4 * kRegThreads;
 
 struct RegScratch {
+  long long ll[kRegWarps];  // systematic design: per-warp prefix totals
   unsigned hist[256];
   int tot[kRegMaxGroups][kRegWarps];
   int off[kRegMaxGroups][kRegWarps];
@@ -767,13 +769,66 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
   // ---- E3 + E4a: draws and ordered compaction of (index, log 1/pi) --------
   const bool compact = a.n_kept != nullptr;
   uint32_t keep = 0u;
+  if (compact && a.systematic) {
+    // Fixed-size systematic sampling at the same pi (Hajek 1964): the tail in
+    // token order, cumulative sums C_i of pi in fixed point (2^-40 units, exact
+    // integer sums), one uniform u per unit; token i is kept when an integer
+    // lies in (C_{i-1} - u, C_i - u].  Inclusion probability pi_i, and the tail
+    // sample size is floor or ceil of sum pi.
+    const uint4 wu = draw_block(a.seed, a.layer, b, kvh, -1);  // counter word 0 = 2^32 - 1
+    const long long ufx = (long long)(wu.x >> 8) << 16;
+    const long long kOne = 1LL << 40;
+    long long carry = 0;
+#pragma unroll 1
+    for (int g = 0; g < JG; ++g) {
+      const float4 v4 = s4[g * kRegThreads + tid];
+      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+      long long pf[4];
+      long long tsum = 0;
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        pf[r] = is_tail(g, r) ? __float2ll_rn(tail_pi(vv[r], mode, c, eps) * 1099511627776.f) : 0;
+        tsum += pf[r];
+      }
+      // block-wide exclusive prefix of tsum in thread order, and the total
+      long long incl = tsum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const long long n = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += n;
+      }
+      __syncthreads();  // earlier readers of sh.ll are done
+      if (lane == 31) sh.ll[warp] = incl;
+      __syncthreads();
+      long long before = 0, total = 0;
+#pragma unroll 8
+      for (int w2 = 0; w2 < kRegWarps; ++w2) {
+        const long long x = sh.ll[w2];
+        before += w2 < warp ? x : 0;
+        total += x;
+      }
+      long long C = carry + before + incl - tsum;
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        if (!((valid >> (4 * g + r)) & 1u)) continue;
+        if ((cert >> (4 * g + r)) & 1u) {
+          keep |= 1u << (4 * g + r);
+          continue;
+        }
+        const long long Cp = C;
+        C += pf[r];
+        if (((C + kOne - ufx) >> 40) != ((Cp + kOne - ufx) >> 40)) keep |= 1u << (4 * g + r);
+      }
+      carry += total;
+    }
+  }
 #pragma unroll 1
   for (int g = 0; g < JG; ++g) {
     const float4 v4 = s4[g * kRegThreads + tid];
     const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
     const bool any_tail = ((tail >> (4 * g)) & 0xFu) != 0u;
     uint4 w = make_uint4(0u, 0u, 0u, 0u);
-    if (compact && __any_sync(0xffffffffu, any_tail))
+    if (compact && !a.systematic && __any_sync(0xffffffffu, any_tail))
       w = draw_block(a.seed, a.layer, b, kvh, g * kRegThreads + tid);
     const uint32_t wr[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
@@ -784,7 +839,8 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
       const float pi = ct ? 1.f : tail_pi(vv[r], mode, c, eps);
       if (a.pi_out) a.pi_out[(size_t)unit * Nrow + i] = pi;
       if (a.mask_out) a.mask_out[(size_t)unit * Nrow + i] = ct ? 1 : 0;
-      if (compact && (ct || word_to_uniform(wr[r]) < pi)) keep |= 1u << (4 * g + r);
+      if (compact && !a.systematic && (ct || word_to_uniform(wr[r]) < pi))
+        keep |= 1u << (4 * g + r);
     }
   }
   if (compact) {
@@ -889,6 +945,8 @@ ebd_status check_design(const ebd_design* d) {
   if ((long long)d->batch * d->n_kv_heads > 0x7fffffffLL) return EBD_ERR_INVALID;
   if (d->n_sink < 0 || d->n_recent < 0 || d->k_head < 0 || d->budget_tokens < 0) return EBD_ERR_INVALID;
   if (d->bisect_iters < 1 || d->bisect_iters > 200) return EBD_ERR_INVALID;
+  if (d->sampling != EBD_SAMPLING_POISSON && d->sampling != EBD_SAMPLING_SYSTEMATIC)
+    return EBD_ERR_INVALID;
   if (!(d->eps > 0.f && d->eps <= 1.f)) return EBD_ERR_INVALID;
   return EBD_OK;
 }
@@ -917,8 +975,10 @@ ebd_status launch_select(const ebd_design* d, const float* scores, const int32_t
   a.cap = cap;
   a.dev_status = dev_status;
   a.vec4 = (((uintptr_t)scores & 15u) == 0 && (d->n_ctx & 3) == 0) ? 1 : 0;
+  a.systematic = d->sampling == EBD_SAMPLING_SYSTEMATIC ? 1 : 0;
   const int units = d->batch * d->n_kv_heads;
   const int groups = (d->n_ctx + kGroupTokens - 1) / kGroupTokens;
+  if (a.systematic && groups > kRegMaxGroups && idx_c) return EBD_ERR_UNSUPPORTED;
   if (groups <= kRegMaxGroups) {
     // the limit is set on every launch: with the kernel's static shared memory
     // even 48 KB of dynamic memory is above the default
@@ -974,7 +1034,7 @@ extern "C" const char* ebd_status_string(ebd_status s) {
   return "EBD_ERR_UNKNOWN";
 }
 
-extern "C" int32_t ebd_abi_version(void) { return 1; }
+extern "C" int32_t ebd_abi_version(void) { return 2; }
 
 extern "C" ebd_status ebd_philox_uniforms(uint64_t seed, int32_t layer, int32_t batch,
                                           int32_t n_kv_heads, int32_t n_ctx, uint32_t* x0,

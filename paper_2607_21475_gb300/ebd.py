@@ -21,7 +21,8 @@ from .build import LIB
 
 __all__ = [
     "EbdError", "EbdDesign", "EBD_F32", "EBD_BF16", "EBD_RANGE_BOUND", "EBD_RANGE_EXACT",
-    "EBD_DEV_CAPACITY", "EBD_DEV_NONFINITE", "EBD_DEV_TIMEOUT", "lib", "lib_path",
+    "EBD_DEV_CAPACITY", "EBD_DEV_NONFINITE", "EBD_DEV_TIMEOUT", "EBD_SAMPLING_POISSON",
+    "EBD_SAMPLING_SYSTEMATIC", "lib", "lib_path",
     "ebd_status_string", "ebd_abi_version", "ebd_philox_uniforms", "ebd_score_workspace_bytes",
     "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
     "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
@@ -35,6 +36,7 @@ EBD_OK = 0
 EBD_F32, EBD_BF16 = 0, 1
 EBD_RANGE_BOUND, EBD_RANGE_EXACT = 0, 1
 EBD_DEV_CAPACITY, EBD_DEV_NONFINITE, EBD_DEV_TIMEOUT = 0x1, 0x2, 0x4
+EBD_SAMPLING_POISSON, EBD_SAMPLING_SYSTEMATIC = 0, 1
 
 # Every symbol include/ebd.h declares.
 ABI_FUNCTIONS = (
@@ -58,7 +60,7 @@ class EbdDesign(ctypes.Structure):
         ("head_dim", ctypes.c_int32), ("n_ctx", ctypes.c_int32), ("layer", ctypes.c_int32),
         ("seed", ctypes.c_uint64), ("n_sink", ctypes.c_int32), ("n_recent", ctypes.c_int32),
         ("k_head", ctypes.c_int32), ("budget_tokens", ctypes.c_int32),
-        ("bisect_iters", ctypes.c_int32), ("eps", ctypes.c_float),
+        ("bisect_iters", ctypes.c_int32), ("eps", ctypes.c_float), ("sampling", ctypes.c_int32),
     ]
 
 
@@ -203,9 +205,10 @@ def ebd_score(q_obs: torch.Tensor, K: torch.Tensor, scores: torch.Tensor, worksp
 
 
 def design_for(*, batch, n_kv_heads, group, head_dim, n_ctx, layer=0, seed=0, n_sink=4,
-               n_recent=32, k_head, budget_tokens, bisect_iters=40, eps=1e-6) -> EbdDesign:
+               n_recent=32, k_head, budget_tokens, bisect_iters=40, eps=1e-6,
+               sampling=0) -> EbdDesign:
     return EbdDesign(batch, n_kv_heads, group, head_dim, n_ctx, layer, seed, n_sink, n_recent,
-                     k_head, budget_tokens, bisect_iters, eps)
+                     k_head, budget_tokens, bisect_iters, eps, sampling)
 
 
 def ebd_compute_pi(design: EbdDesign, scores: torch.Tensor, pi: torch.Tensor,

@@ -69,7 +69,7 @@ def test_status_strings_and_version(E):
     L = E.lib()
     for code in range(6):
         assert L.ebd_status_string(code).startswith(b"EBD_")
-    assert E.ebd_abi_version() == 1
+    assert E.ebd_abi_version() == 2
 
 
 def test_bad_arguments_are_rejected_synchronously(E):

@@ -455,3 +455,59 @@ def test_append_then_reevict_then_decode_matches_oracle(E):
             compare_decode_heads(dec, *(t[b, sl].double().cpu().numpy() for t in (y, lse, var, bt, r)),
                                  False)
     print("near ties", ties)
+
+
+# ------------------------------------------------------- systematic design
+@pytest.mark.parametrize("B,H,N,budget,dist", [(2, 3, 1000, 100, "lognormal"),
+                                               (1, 4, 20000, 2000, "pareto"),
+                                               (2, 2, 32768, 3277, "lognormal")])
+def test_systematic_select_matches_oracle(E, B, H, N, budget, dist):
+    g = torch.Generator().manual_seed(N + budget)
+    if dist == "lognormal":
+        s = torch.exp(torch.randn((B, H, N), generator=g, dtype=torch.float64) * 1.5).float()
+    else:
+        s = (1.0 / torch.rand((B, H, N), generator=g, dtype=torch.float64) ** (1 / 1.2)).float()
+    k_head = budget // 5
+    cap = budget + 64
+    des = _design(E, B, H, 1, 64, N, 3, 0xABCDEF, k_head, budget)
+    des.sampling = E.EBD_SAMPLING_SYSTEMATIC
+    cc = E.alloc_compact(B, H, cap, 64, torch.bfloat16, DEV)
+    idx, logw, n_kept, st = cc.idx_c, cc.logw_c, cc.n_kept, cc.dev_status
+    sd = s.to(DEV)
+    E.ebd_select(des, sd, cc)
+    pi_gpu = torch.empty_like(sd)
+    E.ebd_compute_pi(des, sd, pi_gpu)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    ties = 0
+    for b in range(B):
+        for h in range(H):
+            sc = s[b, h].double().numpy()
+            ref = O.evict_unit_systematic(np.zeros((N, 1)), np.zeros((N, 1)), s[b, h].numpy(),
+                                          n_sink=4, n_recent=32, k_head=k_head, budget_tokens=budget,
+                                          eps=1e-6, seed=0xABCDEF, layer=3, b=b, kvh=h, capacity=cap)
+            n = int(n_kept[b, h])
+            got = idx[b, h, :min(n, cap)].cpu().numpy()
+            # the tail sample size is floor/ceil of the device's own sum of pi
+            tail = ~ref.certain
+            S = pi_gpu[b, h].double().cpu().numpy()[tail].sum()
+            n_tail = n - int(ref.certain.sum())
+            assert math.floor(S) - 1 <= n_tail <= math.ceil(S) + 1
+            # the kept set: identical except where a cumulative sum sits within
+            # the float32 rounding of pi (accumulated along the tail) of an integer
+            C = np.cumsum(np.where(tail, ref.pi, 0.0))
+            u = ref.u[0]
+            band = 1e-6 * (1.0 + C)
+            d_hi = np.abs((C - u) - np.round(C - u))
+            Cp = C - np.where(tail, ref.pi, 0.0)
+            d_lo = np.abs((Cp - u) - np.round(Cp - u))
+            near = tail & ((d_hi < band) | (d_lo < band))
+            diff = set(got.tolist()) ^ set(ref.idx.tolist())
+            bad = [i for i in diff if not near[i]]
+            assert not bad, f"unit {(b, h)}: kept sets differ at {bad[:8]}"
+            ties += int(near.sum())
+            assert set(np.flatnonzero(ref.certain).tolist()) <= set(got.tolist())
+            lw_ref = -np.log(ref.pi[got])
+            np.testing.assert_allclose(logw[b, h, :len(got)].double().cpu().numpy(), lw_ref,
+                                       rtol=2e-5, atol=2e-6)
+    print("systematic near crossings", ties)

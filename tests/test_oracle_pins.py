@@ -14,7 +14,8 @@ import scipy.stats
 import torch
 
 from oracle.ebd_oracle import (
-    deployed_certificate, red_flag, append_token, reevict_unit,
+    deployed_certificate, red_flag, append_token, reevict_unit, systematic_keep,
+    systematic_uniform, evict_unit_systematic,
     accumulated_attention_scores,
     certainty_set,
     certificate_radius,
@@ -569,3 +570,65 @@ def test_composed_weights_keep_the_total_unbiased_over_two_rounds():
     # the second round's weights alone (the first round forgotten) are biased low
     one_round = np.asarray(one_round)
     assert one_round.mean() < x.sum() - 4 * one_round.std(ddof=1) / np.sqrt(len(one_round))
+
+
+
+# ---------------------------------------------------------------- systematic design
+# Systematic sampling at the same pi (Hajek 1964): each token is kept with
+# probability exactly pi_i over the uniform, the tail sample size is floor or
+# ceil of sum pi for every uniform, and the certainty set is always kept.
+# Enumerating the uniform over an even grid makes these exact checks.
+def _sys_case(n=23, seed=4):
+    rng = np.random.default_rng(seed)
+    pi = np.minimum(1.0, rng.uniform(0.02, 0.9, n))
+    pi[5] = 1.0
+    certain = np.zeros(n, dtype=bool)
+    certain[[0, 7, 22]] = True
+    pi[certain] = 1.0
+    return pi, certain
+
+
+def test_systematic_inclusion_probabilities_are_pi():
+    pi, certain = _sys_case()
+    grid = 1 << 12
+    hits = np.zeros(len(pi))
+    for k in range(grid):
+        hits += systematic_keep(pi, certain, k << 12)
+    freq = hits / grid
+    assert np.all(freq[certain] == 1.0)
+    pi32 = pi.astype(np.float32).astype(np.float64)
+    np.testing.assert_allclose(freq[~certain], pi32[~certain], atol=1.0 / grid + 1e-9)
+
+
+def test_systematic_sample_size_is_floor_or_ceil_of_sum():
+    pi, certain = _sys_case()
+    total = pi.astype(np.float32).astype(np.float64)[~certain].sum()
+    for k in range(0, 1 << 24, 99991):
+        keep = systematic_keep(pi, certain, k)
+        n_tail = int(keep[~certain].sum())
+        assert math.floor(total) <= n_tail <= math.ceil(total)
+        assert np.all(keep[certain])
+
+
+def test_systematic_horvitz_thompson_total_is_exact_in_expectation():
+    pi, certain = _sys_case(n=31, seed=9)
+    x = np.random.default_rng(2).uniform(0.1, 3.0, len(pi))
+    pi32 = pi.astype(np.float32).astype(np.float64)
+    grid = 1 << 12
+    est = np.mean([np.sum((x / pi32)[systematic_keep(pi, certain, k << 12)])
+                   for k in range(grid)])
+    assert est == pytest.approx(x.sum(), rel=2e-3)
+
+
+def test_systematic_eviction_keeps_the_budget():
+    rng = np.random.default_rng(12)
+    n = 400
+    s = rng.lognormal(0.0, 1.5, n)
+    K = rng.standard_normal((n, 4))
+    for seed in range(6):
+        r = evict_unit_systematic(K, K, s, n_sink=4, n_recent=8, k_head=10, budget_tokens=60,
+                                  eps=1e-6, seed=seed, layer=2, b=1, kvh=3, capacity=128)
+        n_cert = int(r.certain.sum())
+        assert r.m == 60 - n_cert
+        assert abs(r.n_kept - 60) <= 1  # the Poisson design only matches it in expectation
+    assert 0 <= systematic_uniform(7, 2, 1, 3) < (1 << 24)
