@@ -290,6 +290,54 @@ ebd_status ebd_reevict(const ebd_design* design, ebd_dtype dtype, const float* s
                        int32_t* n_kept_out, int32_t cap_out, int32_t* dev_status, void* stream);
 
 /*
+ * Observation queries for E0 (Appendix, experimental details: accumulated
+ * attention from strided prefill queries, a SnapKV-style window of the last 64
+ * prefill positions, or question-position queries).  Copies the prefill query
+ * rows at `positions` into the observation layout ebd_score reads:
+ *   q_obs[b, kvh, g * P + p, :] = Q[b, kvh * G + g, positions[p], :]
+ *   Q         device [B, Hkv*G, n_rows_q, d] (dtype), 16-byte aligned
+ *   positions device [P] int32, each in [0, n_rows_q) (not checked on device)
+ *   q_obs     device [B, Hkv, G*P, d] (dtype) out
+ */
+ebd_status ebd_gather_queries(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads, int32_t group,
+                              int32_t head_dim, int32_t n_rows_q, const void* Q,
+                              const int32_t* positions, int32_t n_pos, void* q_obs,
+                              void* stream);
+
+/*
+ * Per-token variance contributions: the terms of Theorem 2's estimator,
+ *   contrib[b, h, i] = (1 - pi_i) p_i^2 ||v_i - y_hat_h||^2,  p_i = w_i / N_hat,
+ * so that sum_i contrib[b, h, i] = V_hat of head h.  Certain rows (pi = 1) and
+ * rows at or past min(n_kept, cap) get 0.  A second pass over the compact
+ * cache after ebd_certified_decode, whose y and lse it reads (Section 5's
+ * fine-grained probe records these per retained token).
+ *   Q, K_c, V_c, logw_c, n_kept, capacity: as for ebd_certified_decode
+ *   y, lse     device [B, Hkv*G, d] / [B, Hkv*G] float32 from the decode
+ *   contrib    device [B, Hkv*G, capacity] float32 out
+ * Supports d in {64, 128} and G <= 8.
+ */
+ebd_status ebd_variance_contributions(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads,
+                                      int32_t group, int32_t head_dim, const void* Q,
+                                      const void* K_c, const void* V_c, const float* logw_c,
+                                      const int32_t* n_kept, int32_t capacity, const float* y,
+                                      const float* lse, float* contrib, void* stream);
+
+/*
+ * Block scores for contribution-guided retrieval (Section 5, finer grains):
+ * for every block k of `block` original positions, the sum over the unit's G
+ * query heads of the contributions of its retained rows with idx_c in
+ * [k * block, (k + 1) * block) -- the blocks whose evicted tokens sit among
+ * high-contribution retained neighbours rank first.  Deterministic order.
+ *   contrib  device [B, Hkv*G, capacity] from ebd_variance_contributions
+ *   idx_c, n_kept, capacity: the compact cache (idx_c increasing per unit)
+ *   out      device [B, Hkv, n_blocks] float32
+ */
+ebd_status ebd_block_scores(int32_t batch, int32_t n_kv_heads, int32_t group,
+                            const float* contrib, const int32_t* idx_c, const int32_t* n_kept,
+                            int32_t capacity, int32_t block, int32_t n_blocks, float* out,
+                            void* stream);
+
+/*
  * Deployed certificate and red-flag rule (the experimental setup of Section 5
  * and its appendix; the rule cert >= tau = 1 of Section 5).  At each of the
  * first six decode steps the radii r_t of Eq. (4) (delta = 0.1) of every

@@ -515,3 +515,51 @@ def evict_unit_systematic(K, V, scores, *, n_sink, n_recent, k_head, budget_toke
     K_c, V_c, logw, idx, n_kept = compact(K, V, keep, pi, capacity)
     return EvictResult(certain, topk, pi, c, m, np.full(len(scores), u24 * 2.0 ** -24),
                        np.zeros(len(scores), dtype=np.uint32), keep, idx, logw, K_c, V_c, n_kept)
+
+
+# ---------------------------------------------------------------------------
+# Observation queries (Appendix, experimental details) and per-token variance
+# contributions (Theorem 2's terms; Section 5's fine-grained probe).
+# ---------------------------------------------------------------------------
+def gather_queries(Q, positions, n_kv_heads):
+    """Q [B, Hq, Nq, d] -> q_obs [B, Hkv, G*P, d], row g*P + p = Q[b, kvh*G + g, positions[p]]."""
+    Q = np.asarray(Q)
+    B, Hq, _, d = Q.shape
+    G = Hq // n_kv_heads
+    pos = np.asarray(positions)
+    sel = Q[:, :, pos, :]                      # [B, Hq, P, d]
+    return sel.reshape(B, n_kv_heads, G * len(pos), d)
+
+
+def variance_contributions(q, K_c, V_c, logw_c):
+    """[G, n] terms (1 - pi_i) p_i^2 ||v_i - y_hat||^2 of V_hat (Theorem 2) for
+    the query heads q [G, d] over one unit's retained rows."""
+    q = np.atleast_2d(np.asarray(q, dtype=np.float64))
+    K_c = np.asarray(K_c, dtype=np.float64)
+    V_c = np.asarray(V_c, dtype=np.float64)
+    logw = np.asarray(logw_c, dtype=np.float64)
+    n = K_c.shape[0]
+    if n == 0:
+        return np.zeros((q.shape[0], 0))
+    d = K_c.shape[1]
+    x = q @ K_c.T / math.sqrt(d) + logw[None, :]
+    p = np.exp(x - scipy_logsumexp(x))
+    y = p @ V_c
+    omp = -np.expm1(-logw)
+    dist = ((V_c[None, :, :] - y[:, None, :]) ** 2).sum(-1)
+    return omp[None, :] * p ** 2 * dist
+
+
+def scipy_logsumexp(x):
+    m = x.max(axis=1, keepdims=True)
+    return m + np.log(np.exp(x - m).sum(axis=1, keepdims=True))
+
+
+def block_scores(contrib, idx_c, block, n_blocks):
+    """Sum over heads and retained rows of the contributions, per block of
+    `block` original positions: contrib [G, n], idx_c [n] -> [n_blocks]."""
+    out = np.zeros(n_blocks)
+    tot = np.asarray(contrib).sum(axis=0)
+    for i, t in enumerate(np.asarray(idx_c)):
+        out[int(t) // block] += tot[i]
+    return out

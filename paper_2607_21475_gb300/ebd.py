@@ -27,7 +27,7 @@ __all__ = [
     "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
     "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
     "ebd_certified_decode_static", "ebd_certificate_update", "ebd_append", "ebd_reevict",
-    "design_for",
+    "ebd_gather_queries", "ebd_variance_contributions", "ebd_block_scores", "design_for",
     "CompactCache",
     "alloc_compact", "ABI_FUNCTIONS",
 ]
@@ -44,6 +44,7 @@ ABI_FUNCTIONS = (
     "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
     "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
     "ebd_certified_decode_static", "ebd_certificate_update", "ebd_append", "ebd_reevict",
+    "ebd_gather_queries", "ebd_variance_contributions", "ebd_block_scores",
 )
 
 
@@ -116,6 +117,14 @@ def lib():
             "ebd_reevict": (ctypes.c_int, [P, ctypes.c_int, c_void_p, c_void_p, c_void_p, c_void_p,
                                            c_void_p, c_void_p, i32, c_void_p, c_void_p, c_void_p,
                                            c_void_p, c_void_p, i32, c_void_p, c_void_p]),
+            "ebd_gather_queries": (ctypes.c_int, [ctypes.c_int, i32, i32, i32, i32, i32, c_void_p,
+                                                  c_void_p, i32, c_void_p, c_void_p]),
+            "ebd_variance_contributions": (ctypes.c_int, [ctypes.c_int, i32, i32, i32, i32,
+                                                          c_void_p, c_void_p, c_void_p, c_void_p,
+                                                          c_void_p, i32, c_void_p, c_void_p,
+                                                          c_void_p, c_void_p]),
+            "ebd_block_scores": (ctypes.c_int, [i32, i32, i32, c_void_p, c_void_p, c_void_p, i32,
+                                                i32, i32, c_void_p, c_void_p]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -407,4 +416,56 @@ def ebd_reevict(design: EbdDesign, scores: torch.Tensor, cc_in: "CompactCache",
         _ptr(out.idx_c, torch.int32, (B, H, cap_out), "idx_out"),
         _ptr(out.n_kept, torch.int32, (B, H), "n_kept_out"), cap_out,
         _ptr(out.dev_status, torch.int32, (1,), "dev_status"), _stream(stream)))
+    return out
+
+
+def ebd_gather_queries(Q: torch.Tensor, positions: torch.Tensor, n_kv_heads: int,
+                       q_obs=None, stream=None) -> torch.Tensor:
+    """Observation rows for ebd_score from prefill queries Q [B, Hq, Nq, d] at
+    positions [P] (int32, device): q_obs [B, Hkv, G*P, d], row g*P + p."""
+    B, Hq, Nq, d = Q.shape
+    if Hq % n_kv_heads:
+        raise ValueError("query heads must be a multiple of KV heads")
+    G = Hq // n_kv_heads
+    P = positions.shape[0]
+    if q_obs is None:
+        q_obs = torch.empty((B, n_kv_heads, G * P, d), dtype=Q.dtype, device=Q.device)
+    _check("ebd_gather_queries", lib().ebd_gather_queries(
+        _dtype_code(Q), B, n_kv_heads, G, d, Nq, _ptr(Q, name="Q"),
+        _ptr(positions, torch.int32, (P,), "positions"), P,
+        _ptr(q_obs, Q.dtype, (B, n_kv_heads, G * P, d), "q_obs"), _stream(stream)))
+    return q_obs
+
+
+def ebd_variance_contributions(Q: torch.Tensor, K_c: torch.Tensor, V_c: torch.Tensor,
+                               logw_c: torch.Tensor, n_kept: torch.Tensor, y: torch.Tensor,
+                               lse: torch.Tensor, contrib=None, stream=None) -> torch.Tensor:
+    """Theorem 2's per-token terms [B, Hq, cap] (they sum to V_hat per head)."""
+    B, H, cap, d = K_c.shape
+    Hq = Q.shape[1]
+    G = Hq // H
+    f = torch.float32
+    if contrib is None:
+        contrib = torch.empty((B, Hq, cap), dtype=f, device=K_c.device)
+    _check("ebd_variance_contributions", lib().ebd_variance_contributions(
+        _dtype_code(K_c), B, H, G, d, _ptr(Q, K_c.dtype, (B, Hq, d), "Q"), _ptr(K_c, name="K_c"),
+        _ptr(V_c, K_c.dtype, (B, H, cap, d), "V_c"), _ptr(logw_c, f, (B, H, cap), "logw_c"),
+        _ptr(n_kept, torch.int32, (B, H), "n_kept"), cap, _ptr(y, f, (B, Hq, d), "y"),
+        _ptr(lse, f, (B, Hq), "lse"), _ptr(contrib, f, (B, Hq, cap), "contrib"), _stream(stream)))
+    return contrib
+
+
+def ebd_block_scores(contrib: torch.Tensor, idx_c: torch.Tensor, n_kept: torch.Tensor,
+                     block: int, n_blocks: int, out=None, stream=None) -> torch.Tensor:
+    """Sum of retained contributions per block of `block` original positions."""
+    B, H, cap = idx_c.shape
+    Hq = contrib.shape[1]
+    G = Hq // H
+    if out is None:
+        out = torch.empty((B, H, n_blocks), dtype=torch.float32, device=idx_c.device)
+    _check("ebd_block_scores", lib().ebd_block_scores(
+        B, H, G, _ptr(contrib, torch.float32, (B, Hq, cap), "contrib"),
+        _ptr(idx_c, torch.int32, (B, H, cap), "idx_c"), _ptr(n_kept, torch.int32, (B, H), "n_kept"),
+        cap, int(block), int(n_blocks), _ptr(out, torch.float32, (B, H, n_blocks), "out"),
+        _stream(stream)))
     return out

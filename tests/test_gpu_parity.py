@@ -511,3 +511,55 @@ def test_systematic_select_matches_oracle(E, B, H, N, budget, dist):
             np.testing.assert_allclose(logw[b, h, :len(got)].double().cpu().numpy(), lw_ref,
                                        rtol=2e-5, atol=2e-6)
     print("systematic near crossings", ties)
+
+
+# --------------------------------------------- observation queries and contributions
+def test_snapkv_window_scores_match_oracle(E):
+    """E0 from the SnapKV-style window (queries of the last 64 prefill positions)."""
+    B, H, G, N, d = 2, 2, 4, 1500, 128
+    g = torch.Generator().manual_seed(31)
+    Qp = torch.randn((B, H * G, N, d), generator=g).to(torch.bfloat16)
+    K = (torch.randn((B, H, N, d), generator=g) * 1.3).to(torch.bfloat16)
+    pos = torch.arange(N - 64, N, dtype=torch.int32)
+    q_obs = E.ebd_gather_queries(Qp.to(DEV), pos.to(DEV), H)
+    ref_q = O.gather_queries(Qp.view(torch.int16).numpy(), pos.numpy(), H)
+    assert np.array_equal(q_obs.cpu().view(torch.int16).numpy(), ref_q)
+    s = torch.empty((B, H, N), dtype=torch.float32, device=DEV)
+    E.ebd_score(q_obs, K.to(DEV), s)
+    torch.cuda.synchronize()
+    qd = O.gather_queries(Qp.double().numpy(), pos.numpy(), H)
+    for b in range(B):
+        for h in range(H):
+            ref = O.accumulated_attention_scores(qd[b, h], K[b, h].double().numpy())
+            np.testing.assert_allclose(f64(s)[b, h], ref, rtol=1e-4, atol=1e-7 * G * 64)
+
+
+@pytest.mark.parametrize("B,H,G,d,cap,dtype", [(2, 4, 7, 128, 1600, torch.bfloat16),
+                                               (1, 2, 4, 64, 300, torch.float32)])
+def test_variance_contributions_and_block_scores_match_oracle(E, B, H, G, d, cap, dtype):
+    Kc, Vc, logw, n = _synthetic_cache(B, H, cap, d, dtype, "random", seed=77)
+    idx = torch.sort(torch.randperm(cap * 4, generator=torch.Generator().manual_seed(5))[:cap])[0]
+    idx_c = idx.int().view(1, 1, cap).expand(B, H, cap).contiguous()
+    Q = torch.randn((B, H * G, d), generator=torch.Generator().manual_seed(8)).to(dtype)
+    args = [t.to(DEV) for t in (Q, Kc, Vc, logw, n)]
+    y = torch.empty((B, H * G, d), dtype=torch.float32, device=DEV)
+    lse, var, bt, r = (torch.empty((B, H * G), dtype=torch.float32, device=DEV) for _ in range(4))
+    E.ebd_certified_decode(*args, y, lse, var, bt, r)
+    contrib = E.ebd_variance_contributions(*args, y, lse)
+    n_blocks = (cap * 4 + 63) // 64
+    bs = E.ebd_block_scores(contrib, idx_c.to(DEV), args[4], 64, n_blocks)
+    torch.cuda.synchronize()
+    cg, bg, vg = f64(contrib), f64(bs), f64(var)
+    for b in range(B):
+        for h in range(H):
+            k = int(n[b, h])
+            sl = slice(h * G, (h + 1) * G)
+            ref = O.variance_contributions(Q[b, sl].double().numpy(), Kc[b, h, :k].double().numpy(),
+                                           Vc[b, h, :k].double().numpy(), logw[b, h, :k].double().numpy())
+            scale = ref.max(axis=1, keepdims=True) + 1e-30
+            assert np.all(np.abs(cg[b, sl, :k] - ref) <= 2e-3 * scale + 1e-12)
+            assert np.all(cg[b, sl, k:] == 0.0)
+            # they add up to the decode's own V_hat
+            np.testing.assert_allclose(cg[b, sl, :k].sum(axis=1), vg[b, sl], rtol=2e-3, atol=1e-9)
+            ref_bs = O.block_scores(ref, idx[:k].numpy(), 64, n_blocks)
+            assert np.all(np.abs(bg[b, h] - ref_bs) <= 2e-3 * ref_bs.max() + 1e-12)

@@ -15,7 +15,8 @@ import torch
 
 from oracle.ebd_oracle import (
     deployed_certificate, red_flag, append_token, reevict_unit, systematic_keep,
-    systematic_uniform, evict_unit_systematic,
+    systematic_uniform, evict_unit_systematic, gather_queries, variance_contributions,
+    block_scores,
     accumulated_attention_scores,
     certainty_set,
     certificate_radius,
@@ -632,3 +633,41 @@ def test_systematic_eviction_keeps_the_budget():
         assert r.m == 60 - n_cert
         assert abs(r.n_kept - 60) <= 1  # the Poisson design only matches it in expectation
     assert 0 <= systematic_uniform(7, 2, 1, 3) < (1 << 24)
+
+
+
+# ---------------------------------------------------------------- contributions and queries
+# The per-token contributions are the terms of Theorem 2's V_hat: they sum to
+# the decode's V_hat (pinned above by enumeration and Monte Carlo), certain
+# rows add nothing, and the block scores partition their total.
+def test_contributions_sum_to_v_hat_and_certain_rows_add_nothing():
+    rng = np.random.default_rng(21)
+    n, d, G = 120, 16, 3
+    K = rng.standard_normal((n, d))
+    V = rng.standard_normal((n, d)) + 0.5
+    pi = rng.uniform(0.05, 1.0, n)
+    pi[:30] = 1.0
+    logw = -np.log(pi)
+    q = rng.standard_normal((G, d))
+    c = variance_contributions(q, K, V, logw)
+    dec = hajek_decode(q, K, V, logw)
+    np.testing.assert_allclose(c.sum(axis=1), dec.var, rtol=1e-10)
+    assert np.all(c[:, :30] == 0.0) and np.all(c >= 0.0)
+
+
+def test_block_scores_partition_the_contributions():
+    c = np.array([[1.0, 2.0, 3.0, 4.0, 5.0], [0.5, 0.0, 0.25, 0.0, 1.0]])
+    idx = np.array([3, 63, 64, 130, 200])
+    out = block_scores(c, idx, 64, 4)
+    assert list(out) == [3.5, 3.25, 4.0, 6.0]
+    assert out.sum() == c.sum()
+
+
+def test_gather_queries_layout():
+    Q = np.arange(2 * 4 * 10 * 2).reshape(2, 4, 10, 2)  # B=2, Hq=4, Nq=10, d=2
+    pos = [9, 3]
+    q = gather_queries(Q, pos, n_kv_heads=2)             # G = 2, P = 2
+    assert q.shape == (2, 2, 4, 2)
+    # unit (b=1, kvh=1): rows g*P + p = Q[1, 2 + g, pos[p]]
+    assert np.array_equal(q[1, 1, 0], Q[1, 2, 9]) and np.array_equal(q[1, 1, 1], Q[1, 2, 3])
+    assert np.array_equal(q[1, 1, 2], Q[1, 3, 9]) and np.array_equal(q[1, 1, 3], Q[1, 3, 3])
