@@ -535,14 +535,15 @@ def run_ours(args, world, rank, local):
         if "alg_bytes_per_launch" in v:
             v["gbs"] = v["alg_bytes_per_launch"] / (v["ms_per_launch"] * 1e-3) / 1e9
     dom = max(kern, key=lambda k: kern[k]["ms_per_launch"])
-    kname = {"select": "evict_select_kernel", "gather": "gather_rows_kernel",
-             "decode": "certified decode (split kernel + reduce)", "score": "score kernels"}[dom]
+    kname = {"select": "evict_select_smem_kernel", "gather": "gather_rows_kernel",
+             "decode": "decode_mma_kernel + decode_merge_kernel",
+             "score": "score_lse_tc_kernel + score_col_tc_kernel"}[dom]
     if dom == "score":
-        # dense bf16 contraction (mma.sync): measured cuBLAS bf16 burst peak
+        # dense bf16 contraction on tcgen05: measured cuBLAS bf16 burst peak
         tpk = float(peaks.get("bf16_tflops", 1900.0))
         ach = kern[dom]["alg_flops_per_launch"] / (kern[dom]["ms_per_launch"] * 1e-3) / 1e12
         roof = {"bound": "tensor", "achieved": ach, "peak": tpk, "unit": "TFLOP/s",
-                "frac": ach / tpk, "traffic": None, "kernel": kname,
+                "frac": ach / tpk, "traffic": traffic_for(dom, w.name), "kernel": kname,
                 "peak_source": f"{peak_kind} bf16 dense (MEASURED_PEAKS.json bf16_tflops)"}
     else:
         ach = kern[dom]["gbs"]
