@@ -29,13 +29,11 @@
 // lazily: accumulators are rescaled only when a row's maximum grows by more
 // than 2^8, so weights stay below 2^8 and u below 2^16.
 //
-// Each warp streams its own tiles: one lane issues the 2D TMA copies (128-byte
-// swizzle) of K and V and a 64-byte bulk copy of log(1/pi) for tile j + 2 into
-// its private 3-stage ring while tile j is consumed; every stage has one
-// transaction-counting mbarrier.  A stage is refilled only after the same warp
-// has read it (ordered by a proxy fence), so no empty barrier is needed.
-// Every wait is bounded (~2 s); on timeout the kernel raises EBD_DEV_TIMEOUT,
-// drains the copies it issued and returns.
+// Each warp streams its own tiles: all 32 lanes issue 16-byte cp.async copies
+// of K, V (into the 128-byte-swizzled layout ldmatrix reads) and log(1/pi) for
+// tile j + 2 into the warp's private 3-stage ring while tile j is consumed, one
+// commit group per tile; a stage is read after the lane's wait on its group and
+// a warp barrier, and refilled only after the warp has read it.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
@@ -61,19 +59,19 @@ constexpr int kLocalUnits = 4096;  // tile prefix kept in shared memory up to th
 
 template <int D>
 struct MmaLayout {
-  static constexpr int kHalves = D / 64;                 // 64-column TMA boxes per row
+  static constexpr int kHalves = D / 64;                 // 64-column (128-byte) boxes per row
   static constexpr int kBoxBytes = kMmaTile * 128;      // one box: 16 rows x 128 B
   static constexpr int kStageBytes = 2 * kHalves * kBoxBytes;
   static constexpr int kLogwOff = kMmaStages * kStageBytes;
-  static constexpr int kBarOff = kLogwOff + kMmaStages * kMmaTile * 4;
-  static constexpr int kScanOff = kBarOff + kMmaStages * 8;       // [kMmaConsumers] ints
+  static constexpr int kScanOff = kLogwOff + kMmaStages * kMmaTile * 4;  // [kMmaConsumers] ints
   static constexpr int kPlanOff = kScanOff + 64;                  // [kLocalUnits + 1] ints
   static constexpr int kBytes = kPlanOff + (kLocalUnits + 1) * 4 + 1024;  // + alignment slack
-  static constexpr uint32_t kTxBytes = 2 * kHalves * kBoxBytes + kMmaTile * 4;
 };
 
 struct FastArgs {
   const __nv_bfloat16* Q;    // [units * G, D]
+  const __nv_bfloat16* Kc;   // [units, cap, D]
+  const __nv_bfloat16* Vc;   // [units, cap, D]
   const float* logw;         // [units, cap]
   const int32_t* n_kept;     // [units]
   int32_t* tile_off;         // [units + 1]: written by CTA 0, or by the prefix kernel
@@ -209,21 +207,15 @@ __device__ void block_tile_prefix(const int32_t* __restrict__ n_kept, int units,
 
 template <int D>
 __global__ void __launch_bounds__(kMmaThreads, 1)
-    decode_mma_kernel(const __grid_constant__ CUtensorMap tmK,
-                      const __grid_constant__ CUtensorMap tmV, FastArgs a) {
+    decode_mma_kernel(FastArgs a) {
   using L = MmaLayout<D>;
   constexpr int REC = rec_floats(D);
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
       (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);  // swizzle atoms
   float* lw_s = reinterpret_cast<float*>(smem + L::kLogwOff);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + L::kBarOff);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < kMmaStages; ++s) mbar_init(&full[s], 1);
-    fence_barrier_init();
-  }
   const int units = a.units;
   const int32_t* toff = a.tile_off;
   if (!a.plan_done) {
@@ -248,25 +240,31 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
   const int G = a.group;
   const int g = lane >> 2, q = lane & 3;
   const float kscale = kLog2e * rsqrtf((float)D);
-  uint64_t* my_full = full + warp * kMmaStagesPerWarp;
 
-  // copies: lane 0 walks its own cursor through the warp's tiles
+  // copies: the warp walks its tiles with one cursor; every lane copies 16-byte
+  // chunks of K and V into the 128-byte-swizzled stage layout (chunk ch of row
+  // r of a 64-column half at r * 128 + ((ch ^ (r & 7)) << 4)) and lanes 0-3 the
+  // tile's log(1/pi); one commit group per tile (empty past the range)
   int pf_t = tb, pf_u = unit_of_tile(toff, units, tb);
   int pf_lo = toff[pf_u], pf_hi = toff[pf_u + 1];
   int issued = 0;
   auto issue_next = [&]() {
-    if (lane == 0 && pf_t < te) {
-      const int s = issued % kMmaStagesPerWarp;
-      const int stage = warp * kMmaStagesPerWarp + s;
-      const int row0 = pf_u * a.cap + (pf_t - pf_lo) * kMmaTile;
+    if (pf_t < te) {
+      constexpr int CPR = D / 8;                   // 16-byte chunks per row
+      constexpr int PER = kMmaTile * CPR / 32;     // chunks per lane per tile (K or V)
+      const int stage = warp * kMmaStagesPerWarp + issued % kMmaStagesPerWarp;
+      const size_t row0 = (size_t)pf_u * a.cap + (size_t)(pf_t - pf_lo) * kMmaTile;
       unsigned char* st = smem + (size_t)stage * L::kStageBytes;
-      mbar_arrive_expect_tx(&my_full[s], L::kTxBytes);
 #pragma unroll
-      for (int h = 0; h < L::kHalves; ++h) {
-        tma_load_2d(st + h * L::kBoxBytes, &tmK, h * 64, row0, &my_full[s]);
-        tma_load_2d(st + (L::kHalves + h) * L::kBoxBytes, &tmV, h * 64, row0, &my_full[s]);
+      for (int i = 0; i < PER; ++i) {
+        const int c = lane + 32 * i;
+        const int r = c / CPR, ch = c - r * CPR;
+        const int off = (ch >> 3) * L::kBoxBytes + r * 128 + (((ch & 7) ^ (r & 7)) << 4);
+        const size_t src = (row0 + r) * D + ch * 8;
+        cp_async16(st + off, a.Kc + src);
+        cp_async16(st + L::kHalves * L::kBoxBytes + off, a.Vc + src);
       }
-      bulk_load(lw_s + stage * kMmaTile, a.logw + row0, kMmaTile * 4, &my_full[s]);
+      if (lane < kMmaTile / 4) cp_async16(lw_s + stage * kMmaTile + 4 * lane, a.logw + row0 + 4 * lane);
       ++pf_t;
       if (pf_t < te && pf_t == pf_hi) {
         pf_u = next_unit(toff, pf_u);
@@ -274,6 +272,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
         pf_hi = toff[pf_u + 1];
       }
     }
+    cp_async_commit();
     ++issued;
   };
 
@@ -333,7 +332,6 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
   for (int p = 0; p < kMmaStagesPerWarp - 1; ++p) issue_next();
 
   begin_segment();
-  bool ok = true;
   int j = 0;
   for (int t = tb; t < te; ++t, ++j) {
     issue_next();  // tile j + 2 into the stage tile j - 1 left
@@ -343,12 +341,9 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
       begin_segment();
     }
     const int n_valid = min(kMmaTile, n_u - (t - seg_start) * kMmaTile);
-    const int sl = j % kMmaStagesPerWarp;
-    const int s = warp * kMmaStagesPerWarp + sl;
-    if (!mbar_wait_bounded(&my_full[sl], (uint32_t)((j / kMmaStagesPerWarp) & 1))) {
-      ok = false;
-      break;
-    }
+    const int s = warp * kMmaStagesPerWarp + j % kMmaStagesPerWarp;
+    cp_async_wait<kMmaStagesPerWarp - 1>();  // this lane's copies of tile j are done
+    __syncwarp();                             // and every lane's
     const uint32_t kbase = smem_u32(smem + (size_t)s * L::kStageBytes);
     const uint32_t vbase = kbase + L::kHalves * L::kBoxBytes;
 
@@ -456,8 +451,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
         mma_bf16_16816(acc[2 * jp + 1], r0, r1, r2, r3, v2, v3);
       }
     }
-    // reads of this stage are done before a later copy overwrites it
-    fence_proxy_async_smem();
+    // every lane's reads of this stage are done before it is refilled
     __syncwarp();
     float vn[4] = {vn01.x, vn01.y, vn23.x, vn23.y};
 #pragma unroll
@@ -469,15 +463,8 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
       cmax = fmaxf(cmax, suv[i] * sqrtf(vn[i]));
     }
   }
-  if (!ok) raise_status(a.dev_status, EBD_DEV_TIMEOUT);
-  else flush_segment();
-  // never leave with copies in flight into this CTA's shared memory
-  if (lane == 0) {
-    const int n_iss = min(issued, te - tb);
-#pragma unroll 1
-    for (int k = max(0, n_iss - kMmaStagesPerWarp); k < n_iss; ++k)
-      mbar_wait_bounded(&my_full[k % kMmaStagesPerWarp], (uint32_t)((k / kMmaStagesPerWarp) & 1));
-  }
+  flush_segment();
+  cp_async_wait<0>();
 }
 
 // Merge the partial records of one query head (Eq. 3, Theorem 2, Eq. 4).  One
@@ -659,33 +646,6 @@ __global__ void __launch_bounds__(MW * 32) decode_merge_kernel(MergeArgs a) {
 // ---------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------
-static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  });
-  return fn;
-}
-
-// [rows, D] bf16 viewed as 2D; box = 64 columns x 16 rows, 128-byte swizzle.
-static bool encode_rows_map(CUtensorMap* map, const void* base, long long rows, int D) {
-  auto enc = tensor_map_encoder();
-  if (!enc) return false;
-  const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
-  const cuuint64_t strides[1] = {(cuuint64_t)D * 2};
-  const cuuint32_t box[2] = {64, (cuuint32_t)kMmaTile};
-  const cuuint32_t estr[2] = {1, 1};
-  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
-             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 bool fast_decode_supported(ebd_dtype dtype, int group, int head_dim, int capacity) {
   return dtype == EBD_BF16 && (head_dim == 64 || head_dim == 128) && group >= 1 && group <= 8 &&
          capacity % kMmaTile == 0;
@@ -706,17 +666,12 @@ void fast_decode_plan(DecodePlan& p, long long units, int group, int head_dim) {
 
 bool fast_decode_usable(const DecodeArgs& a, const ReduceArgs& r, int units) {
   return aligned16(a.Kc) && aligned16(a.Vc) && aligned16(a.logw) && aligned16(a.Q) &&
-         aligned16(r.y) && (long long)units * a.cap < 0x7fffffffLL &&
-         tensor_map_encoder() != nullptr;
+         aligned16(r.y) && (long long)units * a.cap < 0x7fffffffLL;
 }
 
 template <int D>
 static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, const ReduceArgs& r,
                                 int units, void* ws, cudaStream_t s) {
-  CUtensorMap tmK, tmV;
-  const long long rows = (long long)units * a.cap;
-  if (!encode_rows_map(&tmK, a.Kc, rows, D) || !encode_rows_map(&tmV, a.Vc, rows, D))
-    return EBD_ERR_CUDA;
   int32_t* tile_off = reinterpret_cast<int32_t*>(ws);
   float* recs = reinterpret_cast<float*>(reinterpret_cast<char*>(ws) + fast_plan_bytes(units));
   const bool plan_done = units > kLocalUnits;
@@ -727,6 +682,8 @@ static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, con
   }
   FastArgs f;
   f.Q = reinterpret_cast<const __nv_bfloat16*>(a.Q);
+  f.Kc = reinterpret_cast<const __nv_bfloat16*>(a.Kc);
+  f.Vc = reinterpret_cast<const __nv_bfloat16*>(a.Vc);
   f.logw = a.logw;
   f.n_kept = a.n_kept;
   f.tile_off = tile_off;
@@ -740,7 +697,7 @@ static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, con
   if (cudaFuncSetAttribute(decode_mma_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            smem) != cudaSuccess)
     return EBD_ERR_CUDA;
-  decode_mma_kernel<D><<<plan.ctas, kMmaThreads, smem, s>>>(tmK, tmV, f);
+  decode_mma_kernel<D><<<plan.ctas, kMmaThreads, smem, s>>>(f);
   ebd_status st = launch_status();
   if (st != EBD_OK) return st;
 
