@@ -91,13 +91,20 @@ def barrier(world):
         dist.barrier()
 
 
-def max_over_ranks(x: float, world: int) -> float:
+def max_over_ranks(x: float, world: int, device: str = "cuda") -> float:
+    """The slowest rank's time: every rank's value, all-reduced with MAX."""
     if world == 1:
         return x
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    t = torch.tensor([x], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def whole_job_rate(units_per_rank: float, world: int, max_seconds: float) -> float:
+    """Weak scaling: every rank processes the same replica of the workload, so
+    the job processes world * units in the slowest rank's time."""
+    return world * units_per_rank / max_seconds
 
 
 def measured_peaks():
@@ -518,9 +525,9 @@ def run_ours(args, world, rank, local):
 
     L = w.n_layers
     dbytes = decode_bytes(w, n_kept)
-    value = world * dbytes / (ph_ms["decode"] * 1e-3) / 1e9
+    value = whole_job_rate(dbytes, world, ph_ms["decode"] * 1e-3) / 1e9
     evict_ms = sum(ph_ms[p] for p in path.phases if p != "decode")
-    evict_mtok = world * w.batch * w.n_ctx * L / (evict_ms * 1e-3) / 1e6
+    evict_mtok = whole_job_rate(w.batch * w.n_ctx * L, world, evict_ms * 1e-3) / 1e6
     kern = {
         "select": {"ms_per_launch": ph_ms["select"] / L,
                    "alg_bytes_per_launch": select_bytes(w, n_kept) / L},
@@ -555,7 +562,7 @@ def run_ours(args, world, rank, local):
     if not args.no_e2e:
         e2e_ms, h2d, d2h = e2e_run(path, args.steps)
         e2e_ms = max_over_ranks(e2e_ms, world)
-        e2e = {"value": world * dbytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
+        e2e = {"value": whole_job_rate(dbytes, world, e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
 
     cpu = None
