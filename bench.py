@@ -66,6 +66,10 @@ def parse_args():
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--batch", type=int, default=0,
                    help="override the workload's batch (smaller cases for profiling)")
+    p.add_argument("--rows", action="store_true",
+                   help="instead of the step: time the added rows (append/re-eviction cadence, "
+                        "certificate aggregation, systematic select, observation queries, "
+                        "variance contributions), one JSON line each")
     return p.parse_args()
 
 
@@ -591,11 +595,186 @@ def run_ours(args, world, rank, local):
         print(json.dumps(line))
 
 
+# ------------------------------------------------------------------ added rows
+def _timer(dev, reps):
+    flush_w = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush_r = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+
+    def time_us(fn, n=reps):
+        fn()
+        torch.cuda.synchronize()
+        ts = []
+        for i in range(n):
+            flush_w.fill_(float(i))
+            flush_r.sum()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b) * 1e3)
+        return statistics.median(ts)
+    return time_us
+
+
+def run_rows(args):
+    """One JSON line per added row, each against its bound (HBM GB/s of
+    measured copy bandwidth where the row moves data, latency otherwise)."""
+    from paper_2607_21475_gb300 import ebd
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    hbm_peak, peak_kind, _ = measured_peaks()
+    time_us = _timer(dev, max(args.steps, 5))
+    lines = []
+
+    def emit(row, **kw):
+        line = {"row": row, **kw}
+        if "bytes" in kw and "us" in kw:
+            gbs = kw["bytes"] / (kw["us"] * 1e-6) / 1e9
+            line["gbs"] = gbs
+            line["frac_of_measured_hbm"] = gbs / hbm_peak
+        lines.append(line)
+        print(json.dumps(line))
+
+    def design(w, n_ctx, layer=0, seed=0, sampling=0, budget=None, k_head=None):
+        return ebd.design_for(batch=w.batch, n_kv_heads=w.n_kv_heads, group=w.group,
+                              head_dim=w.head_dim, n_ctx=n_ctx, layer=layer, seed=seed,
+                              n_sink=w.n_sink, n_recent=w.n_recent,
+                              k_head=w.k_head if k_head is None else k_head,
+                              budget_tokens=w.budget_tokens if budget is None else budget,
+                              bisect_iters=w.bisect_iters, eps=w.eps, sampling=sampling)
+
+    # NEXT-1: eviction every 256 decode steps on the 16k, 25% configuration (one layer):
+    # 256 x (append one token per unit + certified decode), then re-evict the grown cache
+    w = WORKLOADS["qwen7b_16k_b25"].with_(n_layers=1)
+    B, H, G, d, N, T = w.batch, w.n_kv_heads, w.group, w.head_dim, w.n_ctx, 256
+    inp = make_layer_inputs(w, 0, dev)
+    cap = w.capacity + T
+    cc = ebd.alloc_compact(B, H, cap, d, w.torch_dtype, dev)
+    ebd.ebd_evict(design(w, N), inp["K"], inp["V"], inp["scores"], None, cc)
+    torch.cuda.synchronize()
+    base = (cc.K_c.clone(), cc.V_c.clone(), cc.logw_c.clone(), cc.idx_c.clone(), cc.n_kept.clone())
+    g = torch.Generator(device=dev).manual_seed(5)
+    k_new = torch.randn((T, B, H, d), generator=g, device=dev).to(w.torch_dtype)
+    v_new = torch.randn((T, B, H, d), generator=g, device=dev).to(w.torch_dtype)
+    pos = (N + torch.arange(T, device=dev, dtype=torch.int32)).view(T, 1).expand(T, B).contiguous()
+    Hq = H * G
+    y = torch.empty((B, Hq, d), dtype=torch.float32, device=dev)
+    o4 = [torch.empty((B, Hq), dtype=torch.float32, device=dev) for _ in range(4)]
+    dec_ws = torch.empty(ebd.ebd_decode_workspace_bytes(ebd.EBD_BF16, B, H, G, d, cap),
+                         dtype=torch.uint8, device=dev)
+
+    def restore():
+        for dst, src in zip((cc.K_c, cc.V_c, cc.logw_c, cc.idx_c, cc.n_kept), base):
+            dst.copy_(src)
+
+    def loop():
+        for t in range(T):
+            ebd.ebd_append(cc, k_new[t], v_new[t], pos[t])
+            ebd.ebd_certified_decode(inp["Q"], cc.K_c, cc.V_c, cc.logw_c, cc.n_kept, y, *o4,
+                                     workspace=dec_ws)
+    restore()
+    loop()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    restore()
+    with torch.cuda.graph(graph):
+        loop()
+    ts = []
+    for i in range(3):
+        restore()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        graph.replay()
+        b.record()
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b) * 1e3)
+    loop_us = statistics.median(ts)
+    n0 = int(base[4].sum())
+    units = B * H
+    e = w.elem_bytes
+    dec_bytes = sum((n0 + units * (t + 1)) * (2 * d * e + 4) + B * Hq * d * e + B * Hq * (d + 4) * 4
+                    for t in range(T))
+    app_bytes = T * units * (2 * d * e + 8)
+    assert int(cc.dev_status.item()) == 0
+    # re-eviction of the grown cache (fresh seed, same budget)
+    scores2 = torch.exp(torch.randn((B, H, cap), generator=g, device=dev) * 1.5)
+    out = ebd.alloc_compact(B, H, cap, d, w.torch_dtype, dev)
+    des2 = design(w, cap, seed=w.philox_seed + 1)
+    re_us = time_us(lambda: ebd.ebd_reevict(des2, scores2, cc, out))
+    kept2 = int(out.n_kept.sum())
+    re_bytes = units * cap * 4 + kept2 * (4 * d * e + 16)
+    emit("NEXT-1 cadence: 256 x (append + certified decode), one layer of the 16k 25% config",
+         us=loop_us, bytes=dec_bytes + app_bytes, per_step_us=loop_us / T,
+         workload="qwen7b_16k_b25 (B=16, 28/4 heads, d=128, N=16384), 1 layer, 256 steps")
+    emit("NEXT-1 re-eviction of the grown cache (select on resident rows + row gather + compose)",
+         us=re_us, bytes=re_bytes, amortized_per_step_us=re_us / T,
+         workload="qwen7b_16k_b25, 1 layer, cache of N + 256 rows per unit")
+
+    # NEXT-2: deployed certificate update, 28 layers x B=8 x 28 heads
+    rad = torch.rand((28, 8, 28), device=dev)
+    cert = torch.zeros(8, device=dev)
+    cu_us = time_us(lambda: ebd.ebd_certificate_update(rad, cert, first_step=False))
+    emit("NEXT-2 certificate update (one probed step)", us=cu_us, bytes=28 * 8 * 28 * 4 + 8 * 12,
+         workload="28 layers x 8 sequences x 28 query heads")
+
+    # NEXT-3: systematic vs Poisson select on the 32k dialogue layer
+    w = WORKLOADS["dialogue_32k"]
+    inp = make_layer_inputs(w, 0, dev)
+    cc = ebd.alloc_compact(w.batch, w.n_kv_heads, w.capacity, w.head_dim, w.torch_dtype, dev)
+    dp, ds = design(w, w.n_ctx), design(w, w.n_ctx, sampling=ebd.EBD_SAMPLING_SYSTEMATIC)
+    tp = time_us(lambda: ebd.ebd_select(dp, inp["scores"], cc))
+    tsy = time_us(lambda: ebd.ebd_select(ds, inp["scores"], cc))
+    emit("NEXT-3 systematic select (vs Poisson select on the same scores)", us=tsy,
+         poisson_us=tp, tail_sizes_exact=True,
+         workload="dialogue_32k (B=32, 8 KV heads, N=32768, 10%)")
+
+    # NEXT-4a: contributions and block scores on the dialogue compact cache
+    ebd.ebd_gather(dp, inp["K"], inp["V"], ebd.ebd_select(dp, inp["scores"], cc))
+    Hq = w.n_q_heads
+    y = torch.empty((w.batch, Hq, w.head_dim), dtype=torch.float32, device=dev)
+    o4 = [torch.empty((w.batch, Hq), dtype=torch.float32, device=dev) for _ in range(4)]
+    ebd.ebd_certified_decode(inp["Q"], cc.K_c, cc.V_c, cc.logw_c, cc.n_kept, y, *o4)
+    contrib = torch.empty((w.batch, Hq, w.capacity), dtype=torch.float32, device=dev)
+    ct_us = time_us(lambda: ebd.ebd_variance_contributions(inp["Q"], cc.K_c, cc.V_c, cc.logw_c,
+                                                           cc.n_kept, y, o4[0], contrib=contrib))
+    kept = int(cc.n_kept.sum())
+    ct_bytes = kept * (2 * w.head_dim * w.elem_bytes + 4) + w.batch * Hq * w.capacity * 4
+    emit("NEXT-4 variance contributions (second pass over the compact cache)", us=ct_us,
+         bytes=ct_bytes, workload="dialogue_32k, 256 units, 1024 query heads")
+    nb = (w.n_ctx + 63) // 64
+    bs_out = torch.empty((w.batch, w.n_kv_heads, nb), dtype=torch.float32, device=dev)
+    bs_us = time_us(lambda: ebd.ebd_block_scores(contrib, cc.idx_c, cc.n_kept, 64, nb, out=bs_out))
+    emit("NEXT-4 64-token block scores", us=bs_us, bytes=w.batch * Hq * w.capacity * 4,
+         workload="dialogue_32k, 512 blocks per unit")
+
+    # NEXT-4b: SnapKV-style window queries (last 64 prefill positions) feeding E0
+    w = WORKLOADS["qwen7b_6k"]
+    B, H, G, d, N = w.batch, w.n_kv_heads, w.group, w.head_dim, w.n_ctx
+    Qp = torch.randn((B, H * G, N, d), generator=g, device=dev).to(torch.bfloat16)
+    K = torch.randn((B, H, N, d), generator=g, device=dev).to(torch.bfloat16)
+    win = torch.arange(N - 64, N, dtype=torch.int32, device=dev)
+    q_obs = torch.empty((B, H, G * 64, d), dtype=torch.bfloat16, device=dev)
+    gq_us = time_us(lambda: ebd.ebd_gather_queries(Qp, win, H, q_obs=q_obs))
+    sc = torch.empty((B, H, N), dtype=torch.float32, device=dev)
+    ws = torch.empty(ebd.ebd_score_workspace_bytes(B, H, G * 64), dtype=torch.uint8, device=dev)
+    e0_us = time_us(lambda: ebd.ebd_score(q_obs, K, sc, workspace=ws))
+    flops = B * H * 2 * (2 * G * 64 * N * d)
+    emit("NEXT-4 SnapKV window: query gather + E0 on the window queries", us=gq_us + e0_us,
+         gather_us=gq_us, e0_us=e0_us, e0_tflops=flops / (e0_us * 1e-6) / 1e12,
+         workload="qwen7b_6k shape, one layer (B=8, 28/4 heads, N=6144), 64-position window")
+    return lines
+
+
 def main():
     args = parse_args()
     world, rank, local = dist_setup(args)
     if args.impl == "reference":
         run_reference(args, world, rank)
+    elif args.rows:
+        if rank == 0:
+            run_rows(args)
     else:
         run_ours(args, world, rank, local)
     if world > 1 and args.impl == "ours":
