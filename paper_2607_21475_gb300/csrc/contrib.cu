@@ -13,11 +13,13 @@
 // Section 5 ranks evicted 64-token blocks by the contribution of their retained
 // neighbours; ebd_block_scores sums the contributions over blocks of original
 // token positions.  A second pass over the compact cache (y_hat and log N_hat
-// come from the certified decode), one warp per token of a split.
+// come from the certified decode): on tensor cores for bf16 caches whose
+// capacity is a multiple of 16, else one warp per token of a split.
 #include <cuda_runtime.h>
 
 #include "common.cuh"
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace ebd {
 
@@ -102,6 +104,164 @@ __global__ void __launch_bounds__(kCtbThreads)
     }
     if (lane < G) contrib[(hq0 + lane) * cap + t] = out;
   }
+}
+
+// Tensor-core contributions (bf16, d in {64, 128}, G <= 8).  A warp takes a
+// run of 16-token tiles of one unit, streamed by 16-byte cp.async into a
+// 3-stage ring in the 128-byte-swizzled layout.  With tokens as the MMA's M
+// and the query heads as its N (padded to 8), both products share one
+// fragment layout: S^T = K Q^T (Q fragments in registers) and V Y^T (y_hat as
+// bf16 hi + lo, about 16 bits), so each lane holds, for tokens g and g + 8
+// (g = lane / 4) and heads 2q, 2q + 1 (q = lane % 4): the logit, v . y_hat,
+// and ||v||^2 from the same V fragments.  The contribution is
+// (1 - pi) p^2 (||v||^2 - 2 v . y_hat + ||y_hat||^2), p = 2^(x log2e - lse log2e).
+constexpr int kCtmWarps = 8;
+constexpr int kCtmTilesPerWarp = 16;
+constexpr int kCtmStages = 3;
+
+template <int D>
+__global__ void __launch_bounds__(kCtmWarps * 32)
+    contrib_mma_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ Kc,
+                       const __nv_bfloat16* __restrict__ Vc, const float* __restrict__ logw,
+                       const int32_t* __restrict__ n_kept, const float* __restrict__ y,
+                       const float* __restrict__ lse, int group, int cap,
+                       float* __restrict__ contrib) {
+  constexpr int kBox = 16 * 128;                 // 16 rows x 128 B (64 columns)
+  constexpr int kHalves = D / 64;
+  constexpr int kTile = 2 * kHalves * kBox;      // K then V
+  constexpr int CPR = D / 8;                     // 16-byte chunks per row
+  constexpr int PER = 16 * CPR / 32;             // chunks per lane per tile (K or V)
+  extern __shared__ unsigned char ctm_raw[];
+  unsigned char* base = (unsigned char*)(((uintptr_t)ctm_raw + 1023) & ~(uintptr_t)1023);
+  auto sm = reinterpret_cast<unsigned char(*)[kCtmStages][kTile]>(base);
+  auto slw = reinterpret_cast<float(*)[kCtmStages][16]>(base + kCtmWarps * kCtmStages * kTile);
+  const int unit = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, q = lane & 3;
+  const int G = group;
+  const int n = min(max(n_kept[unit], 0), cap);
+  const int ntiles = (cap + 15) / 16;
+  const int t_begin = (blockIdx.x * kCtmWarps + warp) * kCtmTilesPerWarp;
+  if (t_begin >= ntiles) return;
+  const int t_end = min(ntiles, t_begin + kCtmTilesPerWarp);
+  const size_t hq0 = (size_t)unit * G;
+
+  // B fragments (k = d index, n = head): Q and y_hat (hi, lo) of head g
+  uint32_t qb[D / 16][2], yh[D / 16][2], yl[D / 16][2];
+  {
+    const bool hv = g < G;
+    const __nv_bfloat16* qrow = Q + (hq0 + (hv ? g : 0)) * D;
+    const float* yrow = y + (hq0 + (hv ? g : 0)) * D;
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+      const uint32_t* q32 = reinterpret_cast<const uint32_t*>(qrow + 16 * kk);
+      qb[kk][0] = hv ? q32[q] : 0u;
+      qb[kk][1] = hv ? q32[4 + q] : 0u;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const float y0 = hv ? yrow[16 * kk + 8 * h + 2 * q] : 0.f;
+        const float y1 = hv ? yrow[16 * kk + 8 * h + 2 * q + 1] : 0.f;
+        const uint32_t hi = pack_bf16(y0, y1);
+        yh[kk][h] = hi;
+        yl[kk][h] = pack_bf16(y0 - bf16_lo(hi), y1 - bf16_hi(hi));
+      }
+    }
+  }
+  // per-head constants for the heads this lane's C fragments hold (2q, 2q + 1)
+  float l2[2], yy[2] = {0.f, 0.f};
+#pragma unroll
+  for (int c = 0; c < 2; ++c) {
+    const int h = 2 * q + c;
+    l2[c] = h < G ? lse[hq0 + h] * kLog2e : 0.f;
+  }
+  for (int h = 0; h < G; ++h) {  // ||y_hat_h||^2 by a warp reduction
+    float s2 = 0.f;
+#pragma unroll
+    for (int e = lane; e < D; e += 32) s2 = fmaf(y[(hq0 + h) * D + e], y[(hq0 + h) * D + e], s2);
+    s2 = warp_sum(s2);
+    if (h == 2 * q) yy[0] = s2;
+    if (h == 2 * q + 1) yy[1] = s2;
+  }
+  const float kscale = kLog2e * rsqrtf((float)D);
+
+  auto issue = [&](int t, int slot) {
+    if (t < t_end) {
+      const size_t row0 = (size_t)unit * cap + (size_t)t * 16;
+      unsigned char* st = sm[warp][slot];
+#pragma unroll
+      for (int i = 0; i < PER; ++i) {
+        const int c = lane + 32 * i;
+        const int r = c / CPR, ch = c - r * CPR;
+        const int off = (ch >> 3) * kBox + r * 128 + (((ch & 7) ^ (r & 7)) << 4);
+        const size_t src = (row0 + r) * D + ch * 8;
+        cp_async16(st + off, Kc + src);  // cap % 16 == 0: every row of the tile exists
+        cp_async16(st + kHalves * kBox + off, Vc + src);
+      }
+      if (lane < 4) cp_async16(&slw[warp][slot][4 * lane], logw + row0 + 4 * lane);
+    }
+    cp_async_commit();
+  };
+
+#pragma unroll
+  for (int p = 0; p < kCtmStages - 1; ++p) issue(t_begin + p, p);
+  for (int t = t_begin; t < t_end; ++t) {
+    const int slot = (t - t_begin) % kCtmStages;
+    issue(t + kCtmStages - 1, (t - t_begin + kCtmStages - 1) % kCtmStages);
+    cp_async_wait<kCtmStages - 1>();
+    __syncwarp();
+    const int tok0 = t * 16;
+    const int nv = min(16, n - tok0);  // retained rows of this tile (<= 0: none)
+    if (nv > 0) {
+      const uint32_t kbase = smem_u32(sm[warp][slot]);
+      const uint32_t vbase = kbase + kHalves * kBox;
+      float st[4] = {0.f, 0.f, 0.f, 0.f}, vy[4] = {0.f, 0.f, 0.f, 0.f};
+      float vn0 = 0.f, vn1 = 0.f;  // ||v||^2 partials of tokens g and g + 8
+      const int tok = (lane & 7) + ((lane >> 3) & 1) * 8;
+      const int csel = lane >> 4;
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const int chunk = 2 * kk + csel;
+        const uint32_t off = (chunk >> 3) * kBox + tok * 128 + (((chunk & 7) ^ (tok & 7)) << 4);
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4(kbase + off, a0, a1, a2, a3);
+        mma_bf16_16816(st, a0, a1, a2, a3, qb[kk][0], qb[kk][1]);
+        uint32_t v0, v1, v2, v3;
+        ldsm_x4(vbase + off, v0, v1, v2, v3);
+        mma_bf16_16816(vy, v0, v1, v2, v3, yh[kk][0], yh[kk][1]);
+        mma_bf16_16816(vy, v0, v1, v2, v3, yl[kk][0], yl[kk][1]);
+        // v0, v2: token g; v1, v3: token g + 8 (two bf16 each)
+        vn0 = fmaf(bf16_lo(v0), bf16_lo(v0), fmaf(bf16_hi(v0), bf16_hi(v0), vn0));
+        vn0 = fmaf(bf16_lo(v2), bf16_lo(v2), fmaf(bf16_hi(v2), bf16_hi(v2), vn0));
+        vn1 = fmaf(bf16_lo(v1), bf16_lo(v1), fmaf(bf16_hi(v1), bf16_hi(v1), vn1));
+        vn1 = fmaf(bf16_lo(v3), bf16_lo(v3), fmaf(bf16_hi(v3), bf16_hi(v3), vn1));
+      }
+      vn0 += __shfl_xor_sync(0xffffffffu, vn0, 1);
+      vn0 += __shfl_xor_sync(0xffffffffu, vn0, 2);
+      vn1 += __shfl_xor_sync(0xffffffffu, vn1, 1);
+      vn1 += __shfl_xor_sync(0xffffffffu, vn1, 2);
+      // C fragment: st[0], st[1] = (token g, heads 2q, 2q+1); st[2], st[3] = (token g + 8, ...)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int r = g + (e >> 1) * 8;   // token in the tile
+        const int h = 2 * q + (e & 1);    // query head
+        if (r >= nv || h >= G) continue;
+        const float lw = slw[warp][slot][r];
+        const float p = exp2f(fmaf(st[e], kscale, fmaf(lw, kLog2e, -l2[e & 1])));
+        const float vv = (e >> 1) ? vn1 : vn0;
+        const float dist = fmaxf(0.f, vv - 2.f * vy[e] + yy[e & 1]);
+        const float omp = lw > 0.f ? one_minus_exp_neg(lw) : 0.f;
+        contrib[(hq0 + h) * cap + tok0 + r] = omp * p * p * dist;
+      }
+    }
+    // rows of this tile at or past n_kept (within capacity) get 0
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int r = g + (e >> 1) * 8, h = 2 * q + (e & 1);
+      if (r >= max(nv, 0) && h < G && tok0 + r < cap) contrib[(hq0 + h) * cap + tok0 + r] = 0.f;
+    }
+    __syncwarp();  // every lane's reads of this stage are done before it is refilled
+  }
+  cp_async_wait<0>();
 }
 
 // out[b, kvh, k] = sum over the unit's G heads and retained rows whose
@@ -198,6 +358,21 @@ extern "C" ebd_status ebd_variance_contributions(ebd_dtype dtype, int32_t batch,
                                          contrib, s);
     return launch_contrib_t<float, 128>(u, group, capacity, Q, K_c, V_c, logw_c, n_kept, y, lse,
                                         contrib, s);
+  }
+  if (capacity % 16 == 0 && aligned16(Q) && aligned16(K_c) && aligned16(V_c) &&
+      aligned16(logw_c)) {
+    const int ntiles = capacity / 16;
+    const int per_cta = kCtmWarps * kCtmTilesPerWarp;
+    const dim3 grid((ntiles + per_cta - 1) / per_cta, u);
+    const int smem = kCtmWarps * kCtmStages * (2 * (head_dim / 64) * 16 * 128 + 16 * 4) + 1024;
+    auto kern = head_dim == 64 ? contrib_mma_kernel<64> : contrib_mma_kernel<128>;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+        cudaSuccess)
+      return EBD_ERR_CUDA;
+    kern<<<grid, kCtmWarps * 32, smem, s>>>((const __nv_bfloat16*)Q, (const __nv_bfloat16*)K_c,
+                                            (const __nv_bfloat16*)V_c, logw_c, n_kept, y, lse,
+                                            group, capacity, contrib);
+    return launch_status();
   }
   if (head_dim == 64)
     return launch_contrib_t<__nv_bfloat16, 64>(u, group, capacity, Q, K_c, V_c, logw_c, n_kept, y,
