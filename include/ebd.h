@@ -71,7 +71,7 @@ typedef enum { EBD_RANGE_BOUND = 0, EBD_RANGE_EXACT = 1 } ebd_range_mode;
 /* Tail design.  POISSON: independent Bernoulli(pi_i) draws (Section 3.3).
  * SYSTEMATIC: fixed-size systematic sampling at the same pi_i (Hajek 1964;
  * the exact-budget variant of Section 5): the tail in token order, cumulative
- * sums C_i of pi in units of 2^-40 (each pi_i rounded to the nearest unit),
+ * sums C_i of pi in units of 2^-32 (each pi_i rounded to the nearest unit),
  * one uniform u = (x >> 8) 2^-24 per unit with x = word 0 of Philox4x32-10 at
  * counter (2^32 - 1, kvh, layer, b); token i is kept when an integer lies in
  * (C_{i-1} - u, C_i - u].  Its inclusion probability is pi_i and the tail

@@ -474,11 +474,11 @@ def reevict_unit(K_c, V_c, logw_c, idx_c, scores, *, n_sink, n_recent, k_head, b
 # 1964; the exact-budget variant the paper measures in Section 5): the tail in
 # token order, cumulative sums C_i of pi, one uniform u per unit; token i is
 # kept when an integer lies in (C_{i-1} - u, C_i - u].  Each pi_i is first
-# rounded to the nearest multiple of 2^-40 and the sums are exact integers, so
+# rounded to the nearest multiple of 2^-32 and the sums are exact integers, so
 # every implementation takes the same decision.  The uniform is word 0 of
 # Philox4x32-10 at counter (2^32 - 1, kvh, layer, b), u = (x >> 8) 2^-24.
 # ---------------------------------------------------------------------------
-SYSTEMATIC_SCALE = 1 << 40
+SYSTEMATIC_SCALE = 1 << 32
 
 
 def systematic_uniform(seed: int, layer: int, b: int, kvh: int) -> int:
@@ -490,10 +490,10 @@ def systematic_uniform(seed: int, layer: int, b: int, kvh: int) -> int:
 
 def systematic_keep(pi, certain, u24: int):
     """Kept mask of the systematic design; pi is rounded to float32 first (the
-    precision the probabilities are stored in), then to units of 2^-40."""
+    precision the probabilities are stored in), then to units of 2^-32."""
     pi32 = np.asarray(pi, dtype=np.float32).astype(np.float64)
     units = np.rint(pi32 * SYSTEMATIC_SCALE).astype(np.int64)
-    u = u24 << 16
+    u = u24 << 8
     keep = np.asarray(certain, dtype=bool).copy()
     C = 0
     for i in np.flatnonzero(~np.asarray(certain, dtype=bool)):

@@ -133,6 +133,7 @@ __device__ __forceinline__ int block_rank(bool flag, int& total, BlockScratch& s
 
 enum PiMode : int { kPiFloor = 0, kPiAll = 1, kPiLinear = 2 };
 
+
 __device__ __forceinline__ float tail_pi(float s, int mode, float c, float eps) {
   if (mode == kPiFloor) return eps;
   if (mode == kPiAll) return s > 0.f ? 1.f : eps;
@@ -771,55 +772,84 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
   uint32_t keep = 0u;
   if (compact && a.systematic) {
     // Fixed-size systematic sampling at the same pi (Hajek 1964): the tail in
-    // token order, cumulative sums C_i of pi in fixed point (2^-40 units, exact
-    // integer sums), one uniform u per unit; token i is kept when an integer
-    // lies in (C_{i-1} - u, C_i - u].  Inclusion probability pi_i, and the tail
-    // sample size is floor or ceil of sum pi.
+    // token order, cumulative sums C_i of pi in units of 2^-32 (each pi rounded
+    // to the nearest unit), one uniform u per unit; token i is kept when an
+    // integer lies in (C_{i-1} - u, C_i - u].  Only the fractional part of
+    // C - u matters, so the walk adds pi_i (mod 2^32) to it and keeps the token
+    // on a carry out (pi_i = 1: always).  Inclusion probability pi_i, tail size
+    // floor or ceil of sum pi.  Warp w walks tokens [1024 w, 1024 w + 1024) in
+    // rows of 32 (lane = consecutive token: conflict-free reads) with a warp
+    // scan per row, after one block scan of the warps' totals.  Tail and keep
+    // flags move to and from the load layout through two bit arrays in the
+    // (now free) histogram scratch.
     const uint4 wu = draw_block(a.seed, a.layer, b, kvh, -1);  // counter word 0 = 2^32 - 1
-    const long long ufx = (long long)(wu.x >> 8) << 16;
-    const long long kOne = 1LL << 40;
-    long long carry = 0;
+    const uint32_t u32 = (wu.x >> 8) << 8;                     // u in units of 2^-32
+    uint32_t* tailbits = whist;                                  // [kRegMaxGroups * 4096 / 32]
+    uint32_t* keepbits = whist + kRegMaxGroups * kGroupTokens / 32;
+    const int ntok = JG * kGroupTokens;
+    const int nwords = ntok / 32;                                // == JG * 128 <= 1024
+    if (tid < nwords) tailbits[tid] = 0u;
+    __syncthreads();
 #pragma unroll 1
     for (int g = 0; g < JG; ++g) {
-      const float4 v4 = s4[g * kRegThreads + tid];
-      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
-      long long pf[4];
-      long long tsum = 0;
-#pragma unroll
-      for (int r = 0; r < 4; ++r) {
-        pf[r] = is_tail(g, r) ? __float2ll_rn(tail_pi(vv[r], mode, c, eps) * 1099511627776.f) : 0;
-        tsum += pf[r];
+      const uint32_t t4 = (tail >> (4 * g)) & 0xFu;
+      const int i0 = tok(g, 0);
+      if (t4) atomicOr(&tailbits[i0 >> 5], t4 << (i0 & 31));
+    }
+    __syncthreads();
+    const float* sflat = reinterpret_cast<const float*>(s4);
+    auto score_at = [&](int i) {  // token i of the load layout
+      return sflat[((i >> 12) * kRegThreads + ((i & 4095) >> 2)) * 4 + (i & 3)];
+    };
+    // pi in units of 2^-32 (mod 2^32: pi = 1 adds 0 to the fraction)
+    auto units32 = [&](float sv, bool& full) {
+      const float p = tail_pi(sv, mode, c, eps);
+      full = p >= 1.f;
+      return full ? 0u : __float2uint_rn(p * 4294967296.f);
+    };
+    const int wbase = 1024 * warp;
+    uint32_t part = 0u;
+    if (wbase < ntok) {
+#pragma unroll 4
+      for (int j = 0; j < 32; ++j) {
+        const int i = wbase + 32 * j + lane;
+        bool full;
+        if ((tailbits[i >> 5] >> lane) & 1u) part += units32(score_at(i), full);
       }
-      // block-wide exclusive prefix of tsum in thread order, and the total
-      long long incl = tsum;
+    }
 #pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const long long n = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += n;
-      }
-      __syncthreads();  // earlier readers of sh.ll are done
-      if (lane == 31) sh.ll[warp] = incl;
-      __syncthreads();
-      long long before = 0, total = 0;
+    for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+    if (lane == 0) sh.ll[warp] = (long long)part;
+    __syncthreads();
+    uint32_t frac = 0u - u32;  // fractional part of C - u before this warp's tokens
 #pragma unroll 8
-      for (int w2 = 0; w2 < kRegWarps; ++w2) {
-        const long long x = sh.ll[w2];
-        before += w2 < warp ? x : 0;
-        total += x;
-      }
-      long long C = carry + before + incl - tsum;
+    for (int w2 = 0; w2 < kRegWarps; ++w2) frac += w2 < warp ? (uint32_t)sh.ll[w2] : 0u;
+    if (wbase < ntok) {
+#pragma unroll 1
+      for (int j = 0; j < 32; ++j) {
+        const int i = wbase + 32 * j + lane;
+        const bool is_t = (tailbits[i >> 5] >> lane) & 1u;
+        bool full = false;
+        const uint32_t v = is_t ? units32(score_at(i), full) : 0u;
+        uint32_t incl = v;
 #pragma unroll
-      for (int r = 0; r < 4; ++r) {
-        if (!((valid >> (4 * g + r)) & 1u)) continue;
-        if ((cert >> (4 * g + r)) & 1u) {
-          keep |= 1u << (4 * g + r);
-          continue;
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t nb = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += nb;
         }
-        const long long Cp = C;
-        C += pf[r];
-        if (((C + kOne - ufx) >> 40) != ((Cp + kOne - ufx) >> 40)) keep |= 1u << (4 * g + r);
+        const uint32_t after = frac + incl, before = after - v;
+        const bool sel = is_t && (full || after < before);  // a carry: an integer crossed
+        const uint32_t m = __ballot_sync(0xffffffffu, sel);
+        if (lane == 0) keepbits[i >> 5] = m;
+        frac += __shfl_sync(0xffffffffu, incl, 31);
       }
-      carry += total;
+    }
+    __syncthreads();
+#pragma unroll 1
+    for (int g = 0; g < JG; ++g) {
+      const int i0 = tok(g, 0);
+      const uint32_t k4 = (keepbits[i0 >> 5] >> (i0 & 31)) & 0xFu;
+      keep |= (k4 | ((cert & valid) >> (4 * g) & 0xFu)) << (4 * g);
     }
   }
 #pragma unroll 1
