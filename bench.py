@@ -1,14 +1,17 @@
 #!/usr/bin/env python
 """Benchmark of the eviction-by-design hot path on one or more GB300s.
 
-One step = one pass of the whole path over one batch: (scoring, for the
-attention-scored workload) -> select (certainty set, pi, Poisson draw, index
-compaction) -> gather (kept K/V rows) -> certified decode, for every layer of
-the workload.  Each phase runs every layer back to back (a CUDA graph when
-there is more than one layer) between two CUDA events on the launching
-stream; L2 is flushed before every phase, outside the events (a 256 MB buffer
-is written, then another 256 MB buffer read, so that dirty lines are written
-back before the phase starts).
+One step = one pass of the whole path over one batch: the eviction of every
+layer through `ebd_evict` ((scoring, for the attention-scored workload) ->
+select (certainty set, pi, Poisson draw, index compaction) -> gather (kept
+K/V rows); the layers are independent and spread over four streams, and
+within a layer the library pipelines unit chunks over its own side streams),
+then the certified decode of every layer in order.  Each phase is a CUDA
+graph timed between two CUDA events on the launching stream; L2 is flushed
+before every phase, outside the events (a 256 MB buffer is written, then
+another 256 MB buffer read, so that dirty lines are written back before the
+phase starts).  The kernels of the eviction are also timed alone, one phase
+each (score, select, gather), for the per-kernel rates and the roofline.
 
 Prints ONE JSON line (rank 0).  `value` is the certified decode-step HBM
 throughput in GB/s: algorithmic bytes (compact K/V rows, one log(1/pi) per
@@ -310,14 +313,45 @@ class Path:
         dt = ebd.EBD_BF16 if w.dtype == "bf16" else ebd.EBD_F32
         self.dec_ws = torch.empty(max(1, ebd.ebd_decode_workspace_bytes(dt, B, H, G, d, w.capacity)),
                                   dtype=torch.uint8, device=dev)
-        self.phases = (["score"] if self.scored else []) + ["select", "gather", "decode"]
-        self.launches = {"score": 2, "select": 1, "gather": 1, "decode": 2}
+        self.kernel_phases = (["score"] if self.scored else []) + ["select", "gather"]
+        self.step_phases = ["evict", "decode"]
+        self.phases = self.kernel_phases + self.step_phases
+        # ebd_evict runs one select and one gather per chunk of SM-count units
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
+        chunks = -(-(B * H) // sms)
+        self.launches = {"score": 2, "select": 1, "gather": 1, "decode": 2,
+                         "evict": (2 if self.scored else 0) + 2 * chunks}
+        # independent layers are evicted concurrently on a few streams
+        n_ev = min(L, 4) if L > 1 else 0
+        self.ev_streams = [torch.cuda.Stream(device=dev) for _ in range(n_ev)]
+        self.ev_ws = []
+        if self.scored:
+            self.ev_ws = [torch.empty(ebd.ebd_evict_workspace_bytes(self.designs[0], w.n_obs * G),
+                                      dtype=torch.uint8, device=dev) for _ in range(max(1, n_ev))]
         self.use_graph = use_graph
         self.graphs = {}
+
+    def _evict(self):
+        ebd, w = self.ebd, self.w
+        cur = torch.cuda.current_stream()
+        streams = self.ev_streams or [cur]
+        for s in self.ev_streams:
+            s.wait_stream(cur)
+        for l in range(w.n_layers):
+            k = l % len(streams)
+            inp = self.inputs[l]
+            ebd.ebd_evict(self.designs[l], inp["K"], inp["V"],
+                          None if self.scored else inp["scores"],
+                          inp["q_obs"] if self.scored else None, self.cc[l],
+                          workspace=self.ev_ws[k] if self.scored else None, stream=streams[k])
+        for s in self.ev_streams:
+            cur.wait_stream(s)
 
     # one phase over every layer
     def _run(self, phase):
         ebd, w = self.ebd, self.w
+        if phase == "evict":
+            return self._evict()
         for l in range(w.n_layers):
             inp, cc, o = self.inputs[l], self.cc[l], self.out[l]
             if phase == "score":
@@ -525,13 +559,15 @@ def run_ours(args, world, rank, local):
     clk = clocks.stop()
     ph_ms = {ph: statistics.mean(a.elapsed_time(b) for a, b in ev[ph]) for ph in path.phases}
     ph_ms = {ph: max_over_ranks(v, world) for ph, v in ph_ms.items()}
-    ms_step = sum(ph_ms.values())
+    ms_step = sum(ph_ms[p] for p in path.step_phases)
 
     L = w.n_layers
     dbytes = decode_bytes(w, n_kept)
     value = whole_job_rate(dbytes, world, ph_ms["decode"] * 1e-3) / 1e9
-    evict_ms = sum(ph_ms[p] for p in path.phases if p != "decode")
-    evict_mtok = whole_job_rate(w.batch * w.n_ctx * L, world, evict_ms * 1e-3) / 1e6
+    evict_mtok = whole_job_rate(w.batch * w.n_ctx * L, world, ph_ms["evict"] * 1e-3) / 1e6
+    # the eviction kernels run back to back, each phase alone (no overlap)
+    serial_ms = sum(ph_ms[p] for p in path.kernel_phases)
+    evict_serial_mtok = whole_job_rate(w.batch * w.n_ctx * L, world, serial_ms * 1e-3) / 1e6
     kern = {
         "select": {"ms_per_launch": ph_ms["select"] / L,
                    "alg_bytes_per_launch": select_bytes(w, n_kept) / L},
@@ -586,7 +622,7 @@ def run_ours(args, world, rank, local):
         "config": config_of(w),
         "decode_pct_of_8tbs": 100.0 * value / world / NORTH_STAR_HBM_GBS,
         "decode_pct_of_measured_hbm": 100.0 * value / world / hbm_peak,
-        "evict_mtok_s": evict_mtok,
+        "evict_mtok_s": evict_mtok, "evict_kernels_back_to_back_mtok_s": evict_serial_mtok,
         "phases_ms": ph_ms, "kernels": kern,
         "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
         "clocks": clk,

@@ -158,6 +158,13 @@ ebd_status ebd_compute_pi(const ebd_design* design, const float* scores, float* 
  *   dev_status device int32, required
  * Rows [n_kept, cap) of the outputs are left untouched.  Needs workspace of
  * ebd_evict_workspace_bytes(...) bytes (0 when scores are given).
+ * Stream order: all work is ordered after earlier work on `stream` and
+ * before later work on it.  With more units (B * Hkv) than SMs the call cuts
+ * the units into chunks of one SM count and runs each chunk's select and
+ * gather on its own stream (side streams of the library, one set per host
+ * thread and device, created on the first such call made outside stream
+ * capture), forked from and joined back into `stream` with events; this works
+ * under stream capture and gives the same outputs as the single-stream order.
  */
 size_t ebd_evict_workspace_bytes(const ebd_design* design, int32_t n_obs);
 ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const void* K, const void* V,
@@ -167,8 +174,8 @@ ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const void* K, c
 
 /*
  * The two halves of ebd_evict, for callers that keep their own cache layout
- * (and for per-kernel timing).  ebd_evict(scores given) == ebd_select then
- * ebd_gather on the same stream.
+ * (and for per-kernel timing).  ebd_evict(scores given) gives the outputs
+ * of ebd_select then ebd_gather on the same stream.
  *
  * ebd_select: certainty set, Eq. (2) probabilities, Poisson draw and the
  * stable compaction of indices (Section 3.3, Appendix B) -- everything but

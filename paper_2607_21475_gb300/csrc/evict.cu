@@ -52,6 +52,7 @@ struct SelectArgs {
   int32_t* dev_status;  // nullable
   int vec4;             // scores rows start 16-byte aligned (float4 loads)
   int systematic;       // tail design: 0 Poisson, 1 systematic at the same pi
+  int unit0;            // first unit of this launch (CTA x handles unit unit0 + x)
 };
 
 struct BlockScratch {
@@ -147,7 +148,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
   __shared__ unsigned sh_prefix, sh_remaining;
   __shared__ int sh_bad;
 
-  const int unit = blockIdx.x;
+  const int unit = a.unit0 + blockIdx.x;
   const int b = unit / a.n_kv_heads;
   const int kvh = unit - b * a.n_kv_heads;
   const int Nrow = a.n_ctx;
@@ -499,7 +500,7 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
   // followed by the per-warp top-digit histograms [kRegWarps][256]
   unsigned* whist = reinterpret_cast<unsigned*>(s4 + JG * kRegThreads);
   __shared__ RegScratch sh;
-  const int unit = blockIdx.x;
+  const int unit = a.unit0 + blockIdx.x;
   const int b = unit / a.n_kv_heads;
   const int kvh = unit - b * a.n_kv_heads;
   const int Nrow = a.n_ctx;
@@ -907,8 +908,8 @@ constexpr int kGatherUnroll = 4;
 __global__ void __launch_bounds__(kGatherThreads) gather_rows_kernel(
     const uint4* __restrict__ K, const uint4* __restrict__ V, uint4* __restrict__ Kc,
     uint4* __restrict__ Vc, const int32_t* __restrict__ idx_c, const int32_t* __restrict__ n_kept,
-    int n_ctx, int cap, int cpr) {
-  const int unit = blockIdx.y;
+    int n_ctx, int cap, int cpr, int unit0) {
+  const int unit = unit0 + blockIdx.y;
   const int n = min(n_kept[unit], cap);
   const long long items = (long long)n * cpr;
   const long long stride = (long long)gridDim.x * kGatherThreads;
@@ -981,9 +982,10 @@ ebd_status check_design(const ebd_design* d) {
   return EBD_OK;
 }
 
-ebd_status launch_select(const ebd_design* d, const float* scores, const int32_t* n_len,
-                         float* pi, uint8_t* mask, int32_t* idx_c, float* logw_c, int32_t* n_kept,
-                         int cap, int32_t* dev_status, cudaStream_t stream) {
+ebd_status launch_select_range(const ebd_design* d, const float* scores, const int32_t* n_len,
+                               float* pi, uint8_t* mask, int32_t* idx_c, float* logw_c,
+                               int32_t* n_kept, int cap, int32_t* dev_status, int unit0,
+                               int n_units, cudaStream_t stream) {
   SelectArgs a;
   a.scores = scores;
   a.n_ctx = d->n_ctx;
@@ -1006,7 +1008,9 @@ ebd_status launch_select(const ebd_design* d, const float* scores, const int32_t
   a.dev_status = dev_status;
   a.vec4 = (((uintptr_t)scores & 15u) == 0 && (d->n_ctx & 3) == 0) ? 1 : 0;
   a.systematic = d->sampling == EBD_SAMPLING_SYSTEMATIC ? 1 : 0;
-  const int units = d->batch * d->n_kv_heads;
+  a.unit0 = unit0;
+  const int units = n_units;
+  if (units < 1) return EBD_OK;
   const int groups = (d->n_ctx + kGroupTokens - 1) / kGroupTokens;
   if (a.systematic && groups > kRegMaxGroups && idx_c) return EBD_ERR_UNSUPPORTED;
   if (groups <= kRegMaxGroups) {
@@ -1027,14 +1031,23 @@ ebd_status launch_select(const ebd_design* d, const float* scores, const int32_t
   return launch_status();
 }
 
+ebd_status launch_select(const ebd_design* d, const float* scores, const int32_t* n_len,
+                         float* pi, uint8_t* mask, int32_t* idx_c, float* logw_c, int32_t* n_kept,
+                         int cap, int32_t* dev_status, cudaStream_t stream) {
+  return launch_select_range(d, scores, n_len, pi, mask, idx_c, logw_c, n_kept, cap, dev_status,
+                             0, d->batch * d->n_kv_heads, stream);
+}
+
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
-ebd_status launch_gather(const ebd_design* d, ebd_dtype dtype, const void* K, const void* V,
-                         const int32_t* idx_c, const int32_t* n_kept, int cap, void* K_c,
-                         void* V_c, cudaStream_t s) {
+ebd_status launch_gather_range(const ebd_design* d, ebd_dtype dtype, const void* K,
+                               const void* V, const int32_t* idx_c, const int32_t* n_kept,
+                               int cap, void* K_c, void* V_c, int unit0, int n_units,
+                               cudaStream_t s) {
   const int eb = dtype == EBD_F32 ? 4 : 2;
   const int cpr = d->head_dim * eb / 16;
-  const int units = d->batch * d->n_kv_heads;
+  const int units = n_units;
+  if (units < 1) return EBD_OK;
   if (units > 65535) return EBD_ERR_UNSUPPORTED;
   const long long items = (long long)cap * cpr;
   long long bx = (items + (long long)kGatherThreads * kGatherUnroll - 1) /
@@ -1044,8 +1057,15 @@ ebd_status launch_gather(const ebd_design* d, ebd_dtype dtype, const void* K, co
   dim3 grid((unsigned)bx, (unsigned)units);
   gather_rows_kernel<<<grid, kGatherThreads, 0, s>>>((const uint4*)K, (const uint4*)V,
                                                      (uint4*)K_c, (uint4*)V_c, idx_c, n_kept,
-                                                     d->n_ctx, cap, cpr);
+                                                     d->n_ctx, cap, cpr, unit0);
   return launch_status();
+}
+
+ebd_status launch_gather(const ebd_design* d, ebd_dtype dtype, const void* K, const void* V,
+                         const int32_t* idx_c, const int32_t* n_kept, int cap, void* K_c,
+                         void* V_c, cudaStream_t s) {
+  return launch_gather_range(d, dtype, K, V, idx_c, n_kept, cap, K_c, V_c, 0,
+                             d->batch * d->n_kv_heads, s);
 }
 
 }  // namespace ebd
@@ -1095,6 +1115,124 @@ extern "C" size_t ebd_evict_workspace_bytes(const ebd_design* design, int32_t n_
          align_up(units * (size_t)n_obs * sizeof(float), 256);
 }
 
+namespace ebd {
+
+// ---- pipelined eviction -------------------------------------------------------
+// A select CTA holds a whole SM (1024 threads, the unit's scores in shared
+// memory) for tens of microseconds at a low HBM rate, while the row gather is
+// HBM-bound and light on the SM.  With more units than SMs the units are cut
+// into chunks of one select wave (one unit per SM) and each chunk's
+// select -> gather pair runs on its own stream: chunk 0 on the caller's
+// stream, the others on side streams forked from it and joined back into it
+// by events.  The gather of the first wave then streams while the second wave
+// selects, instead of both waves selecting before any row moves.  Chunks
+// cover disjoint units, so the outputs do not depend on the schedule.
+constexpr int kEvictSideStreams = 3;
+
+struct EvictStreams {
+  bool tried = false, ok = false;
+  cudaStream_t side[kEvictSideStreams] = {};
+  cudaEvent_t fork = nullptr;
+  cudaEvent_t join[kEvictSideStreams] = {};
+  ~EvictStreams() {
+    if (!ok) return;
+    for (int i = 0; i < kEvictSideStreams; ++i) {
+      cudaStreamDestroy(side[i]);
+      cudaEventDestroy(join[i]);
+    }
+    cudaEventDestroy(fork);
+  }
+};
+
+// Side streams and events of this host thread on the current device, created
+// on first use outside stream capture (nullptr when unavailable: the caller
+// then runs the chunks in order on its own stream).
+EvictStreams* evict_streams(cudaStream_t s) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  static thread_local EvictStreams tl[64];
+  EvictStreams& e = tl[dev];
+  if (!e.tried) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(s, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) {
+      cudaGetLastError();
+      return nullptr;  // create nothing while a graph is being captured
+    }
+    e.tried = true;
+    int made = 0;
+    bool ok = cudaEventCreateWithFlags(&e.fork, cudaEventDisableTiming) == cudaSuccess;
+    for (; ok && made < kEvictSideStreams; ++made) {
+      if (cudaStreamCreateWithFlags(&e.side[made], cudaStreamNonBlocking) != cudaSuccess) {
+        ok = false;
+        break;
+      }
+      if (cudaEventCreateWithFlags(&e.join[made], cudaEventDisableTiming) != cudaSuccess) {
+        cudaStreamDestroy(e.side[made]);
+        ok = false;
+        break;
+      }
+    }
+    if (!ok) {
+      cudaGetLastError();
+      for (int i = 0; i < made; ++i) {
+        cudaStreamDestroy(e.side[i]);
+        cudaEventDestroy(e.join[i]);
+      }
+      if (e.fork) cudaEventDestroy(e.fork);
+    }
+    e.ok = ok;
+  }
+  return e.ok ? &e : nullptr;
+}
+
+// E1-E4 for every unit: chunks of sm_count() units, pipelined over streams.
+ebd_status select_and_gather(const ebd_design* d, ebd_dtype dtype, const float* scores,
+                             const void* K, const void* V, void* K_c, void* V_c, float* logw_c,
+                             int32_t* idx_c, int32_t* n_kept, int cap, int32_t* dev_status,
+                             cudaStream_t s) {
+  const int units = d->batch * d->n_kv_heads;
+  const int chunk = sm_count();
+  EvictStreams* es = units > chunk ? evict_streams(s) : nullptr;
+  if (!es) {
+    ebd_status st = launch_select(d, scores, nullptr, nullptr, nullptr, idx_c, logw_c, n_kept,
+                                  cap, dev_status, s);
+    if (st != EBD_OK) return st;
+    return launch_gather(d, dtype, K, V, idx_c, n_kept, cap, K_c, V_c, s);
+  }
+  const int n_chunks = (units + chunk - 1) / chunk;
+  const int n_side = n_chunks - 1 < kEvictSideStreams ? n_chunks - 1 : kEvictSideStreams;
+  if (cudaEventRecord(es->fork, s) != cudaSuccess) return EBD_ERR_CUDA;
+  int forked = 0;
+  ebd_status st = EBD_OK;
+  for (; forked < n_side; ++forked)
+    if (cudaStreamWaitEvent(es->side[forked], es->fork, 0) != cudaSuccess) {
+      st = EBD_ERR_CUDA;
+      break;
+    }
+  for (int c = 0; st == EBD_OK && c < n_chunks; ++c) {
+    const int lane = c % (n_side + 1);
+    cudaStream_t cs = lane == 0 ? s : es->side[lane - 1];
+    const int u0 = c * chunk;
+    const int n = units - u0 < chunk ? units - u0 : chunk;
+    st = launch_select_range(d, scores, nullptr, nullptr, nullptr, idx_c, logw_c, n_kept, cap,
+                             dev_status, u0, n, cs);
+    if (st == EBD_OK)
+      st = launch_gather_range(d, dtype, K, V, idx_c, n_kept, cap, K_c, V_c, u0, n, cs);
+  }
+  // every forked stream is joined back, also after an error (a capture needs it)
+  for (int i = 0; i < forked; ++i) {
+    if (cudaEventRecord(es->join[i], es->side[i]) != cudaSuccess ||
+        cudaStreamWaitEvent(s, es->join[i], 0) != cudaSuccess)
+      st = EBD_ERR_CUDA;
+  }
+  return st;
+}
+
+}  // namespace ebd
+
 extern "C" ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const void* K,
                                 const void* V, const float* scores, const void* q_obs,
                                 int32_t n_obs, void* K_c, void* V_c, float* logw_c,
@@ -1124,10 +1262,8 @@ extern "C" ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const
     if (st != EBD_OK) return st;
     sc = ws_scores;
   }
-  st = launch_select(design, sc, nullptr, nullptr, nullptr, idx_c, logw_c, n_kept, capacity,
-                     dev_status, s);
-  if (st != EBD_OK) return st;
-  return launch_gather(design, dtype, K, V, idx_c, n_kept, capacity, K_c, V_c, s);
+  return select_and_gather(design, dtype, sc, K, V, K_c, V_c, logw_c, idx_c, n_kept, capacity,
+                           dev_status, s);
 }
 
 extern "C" ebd_status ebd_select(const ebd_design* design, const float* scores, int32_t* idx_c,

@@ -35,6 +35,16 @@ ebd_status launch_gather(const ebd_design* d, ebd_dtype dtype, const void* K, co
                          const int32_t* idx_c, const int32_t* n_kept, int cap, void* K_c,
                          void* V_c, cudaStream_t s);
 
+// The same for the units [unit0, unit0 + n_units) only.
+ebd_status launch_select_range(const ebd_design* d, const float* scores, const int32_t* n_len,
+                               float* pi, uint8_t* mask, int32_t* idx_c, float* logw_c,
+                               int32_t* n_kept, int cap, int32_t* dev_status, int unit0,
+                               int n_units, cudaStream_t stream);
+ebd_status launch_gather_range(const ebd_design* d, ebd_dtype dtype, const void* K,
+                               const void* V, const int32_t* idx_c, const int32_t* n_kept,
+                               int cap, void* K_c, void* V_c, int unit0, int n_units,
+                               cudaStream_t s);
+
 bool aligned16(const void* p);
 
 // E0: accumulated attention scores into `scores` using `workspace` for the

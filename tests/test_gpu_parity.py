@@ -173,6 +173,61 @@ def test_evict_matches_oracle(E, B, H, N, d, dtype, k_head, budget, cap):
     print(f"near ties: {ties}")
 
 
+@pytest.mark.parametrize("B,H,N,d,dtype,cap", [
+    (41, 8, 1000, 64, torch.bfloat16, 256),   # 328 units: three chunks of one SM count
+    (100, 8, 300, 128, torch.float32, 128),   # 800 units: more chunks than side streams
+])
+def test_evict_pipelined_chunks_match_single_stream_and_oracle(E, B, H, N, d, dtype, cap):
+    """With more units than SMs ebd_evict pipelines unit chunks over side
+    streams; the outputs equal select then gather on one stream, eagerly and
+    replayed from a captured graph, and sampled units (chunk edges) match the
+    oracle."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    assert B * H > sms
+    k_head, budget = N // 50, N // 10
+    g = torch.Generator().manual_seed(21)
+    K = torch.randn((B, H, N, d), generator=g).to(dtype)
+    V = torch.randn((B, H, N, d), generator=g).to(dtype)
+    s = torch.exp(1.5 * torch.randn((B, H, N), generator=g))
+    Kg, Vg, sg = K.to(DEV), V.to(DEV), s.to(DEV)
+    des = _design(E, B, H, 1, d, N, 2, 77, k_head, budget)
+    ref = E.alloc_compact(B, H, cap, d, dtype, DEV)
+    E.ebd_select(des, sg, ref)
+    E.ebd_gather(des, Kg, Vg, ref)
+    piped = E.alloc_compact(B, H, cap, d, dtype, DEV)
+    E.ebd_evict(des, Kg, Vg, sg, None, piped)
+    graphed = E.alloc_compact(B, H, cap, d, dtype, DEV)
+    torch.cuda.synchronize()
+    gr = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gr):
+        E.ebd_evict(des, Kg, Vg, sg, None, graphed)
+    gr.replay()
+    torch.cuda.synchronize()
+    for cc in (piped, graphed):
+        assert cc.dev_status.item() == 0
+        assert torch.equal(cc.n_kept, ref.n_kept)
+        for b in range(B):
+            for h in range(H):
+                n = min(int(ref.n_kept[b, h]), cap)
+                assert torch.equal(cc.idx_c[b, h, :n], ref.idx_c[b, h, :n])
+                assert torch.equal(cc.logw_c[b, h, :n], ref.logw_c[b, h, :n])
+                assert torch.equal(cc.K_c[b, h, :n], ref.K_c[b, h, :n])
+                assert torch.equal(cc.V_c[b, h, :n], ref.V_c[b, h, :n])
+    Kb, Vb = bits(K), bits(V)
+    Kd, Vd, sn = K.double().numpy(), V.double().numpy(), s.numpy()
+    for u in sorted({0, sms - 1, sms, min(2 * sms, B * H - 1), B * H - 1}):
+        b, h = divmod(u, H)
+        r = O.evict_unit(Kd[b, h], Vd[b, h], sn[b, h], n_sink=4, n_recent=32, k_head=k_head,
+                         budget_tokens=budget, eps=1e-6, seed=77, layer=2, b=b, kvh=h,
+                         capacity=cap)
+        n = int(piped.n_kept[b, h])
+        kg = min(n, cap)
+        compare_evict_unit(r, n, piped.idx_c[b, h, :kg].cpu().numpy(),
+                           piped.logw_c[b, h, :kg].cpu().double().numpy(),
+                           bits(piped.K_c[b, h, :kg]), bits(piped.V_c[b, h, :kg]),
+                           Kb[b, h], Vb[b, h], cap)
+
+
 def test_evict_capacity_overflow_is_flagged_and_bounded(E):
     B, H, N, d = 1, 2, 2000, 64
     cap = 64  # far below the ~400 kept tokens
