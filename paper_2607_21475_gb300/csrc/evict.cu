@@ -392,7 +392,7 @@ struct RegScratch {
   int res_i[2];
   float c, lo, hi;  // solve state, updated by thread 0 only
   int mode, stop;
-  unsigned prefix, remaining;
+  unsigned prefix, remaining, eqcount;
   int total;
 };
 
@@ -615,6 +615,7 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
             if (cum + c[q] >= remaining) {
               sh.prefix = (unsigned)(255 - 8 * lane - q);  // the chosen digit
               sh.remaining = remaining - cum;
+              sh.eqcount = c[q];  // live tokens with this digit
               break;
             }
             cum += c[q];
@@ -637,18 +638,23 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
       }
     }
     // `live` now holds exactly the tokens whose key equals the k-th largest;
-    // the `remaining` lowest-index ones complete the top slice
+    // the `remaining` lowest-index ones complete the top slice (all of them,
+    // without an ordered scan, when there are no more than that)
     const uint32_t eq = live;
-    ordered_scan(eq, JG, sh);
+    if (sh.eqcount <= remaining) {
+      cert |= eq;
+    } else {
+      ordered_scan(eq, JG, sh);
 #pragma unroll 1
-    for (int g = 0; g < JG; ++g) {
-      int run = sh.off[g][warp] + lane_prefix(eq, g);
+      for (int g = 0; g < JG; ++g) {
+        int run = sh.off[g][warp] + lane_prefix(eq, g);
 #pragma unroll
-      for (int r = 0; r < 4; ++r) {
-        const uint32_t bit = 1u << (4 * g + r);
-        if (eq & bit) {
-          if (run < (int)remaining) cert |= bit;
-          ++run;
+        for (int r = 0; r < 4; ++r) {
+          const uint32_t bit = 1u << (4 * g + r);
+          if (eq & bit) {
+            if (run < (int)remaining) cert |= bit;
+            ++run;
+          }
         }
       }
     }
@@ -902,7 +908,7 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
 }
 
 // E4b: copy kept K and V rows (16-byte chunks, `cpr` chunks per row).
-constexpr int kGatherThreads = 256;
+constexpr int kGatherThreads = 128;  // small CTAs also fit beside a select CTA
 constexpr int kGatherUnroll = 4;
 
 __global__ void __launch_bounds__(kGatherThreads) gather_rows_kernel(
