@@ -158,6 +158,12 @@ ebd_status ebd_compute_pi(const ebd_design* design, const float* scores, float* 
  *   dev_status device int32, required
  * Rows [n_kept, cap) of the outputs are left untouched.  Needs workspace of
  * ebd_evict_workspace_bytes(...) bytes (0 when scores are given).
+ * Host-resident cache: with the scores given, K, V and the scores may be
+ * page-locked host memory (cudaHostAlloc / cudaHostRegister, addressable by
+ * the device): the select then reads every score and the gather only the kept
+ * rows over the host link, instead of the whole cache being copied first.
+ * Scoring (scores NULL) needs K and q_obs in device memory
+ * (EBD_ERR_UNSUPPORTED otherwise).  Pageable host memory: EBD_ERR_INVALID.
  * Stream order: all work is ordered after earlier work on `stream` and
  * before later work on it.  With more units (B * Hkv) than SMs the call cuts
  * the units into chunks of one SM count and runs each chunk's select and
@@ -189,6 +195,8 @@ ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const void* K, c
  * ebd_gather: copies rows K[idx_c[p]], V[idx_c[p]] to K_c[p], V_c[p] for
  * p < min(n_kept, cap) of every unit (16-byte loads; d * elem must be a
  * multiple of 16 bytes and the four tensors 16-byte aligned).
+ * The scores of ebd_select and K, V of ebd_gather may be page-locked host
+ * memory, as for ebd_evict.
  */
 ebd_status ebd_select(const ebd_design* design, const float* scores, int32_t* idx_c,
                       float* logw_c, int32_t* n_kept, int32_t capacity, int32_t* dev_status,

@@ -1110,7 +1110,9 @@ extern "C" ebd_status ebd_compute_pi(const ebd_design* design, const float* scor
   ebd_status st = check_design(design);
   if (st != EBD_OK) return st;
   if (!scores || !pi) return EBD_ERR_INVALID;
-  return launch_select(design, scores, nullptr, pi, certain_mask, nullptr, nullptr, nullptr, 0,
+  const float* sc = (const float*)device_address(scores);
+  if (!sc) return EBD_ERR_INVALID;
+  return launch_select(design, sc, nullptr, pi, certain_mask, nullptr, nullptr, nullptr, 0,
                        dev_status, (cudaStream_t)stream);
 }
 
@@ -1122,6 +1124,36 @@ extern "C" size_t ebd_evict_workspace_bytes(const ebd_design* design, int32_t n_
 }
 
 namespace ebd {
+
+// Address under which the kernels read a buffer the caller passed: device or
+// managed memory as it is; page-locked host memory through its device mapping
+// (the kernels then read it over the host link, only the parts they use);
+// nullptr for memory the device cannot address (pageable host memory).
+const void* device_address(const void* p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  switch (at.type) {
+    case cudaMemoryTypeDevice:
+    case cudaMemoryTypeManaged:
+      return p;
+    case cudaMemoryTypeHost:
+      return at.devicePointer;
+    default:
+      return nullptr;
+  }
+}
+
+bool is_device_memory(const void* p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
 
 // ---- pipelined eviction -------------------------------------------------------
 // A select CTA holds a whole SM (1024 threads, the unit's scores in shared
@@ -1256,8 +1288,17 @@ extern "C" ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const
   if (!aligned16(K) || !aligned16(V) || !aligned16(K_c) || !aligned16(V_c)) return EBD_ERR_INVALID;
   cudaStream_t s = (cudaStream_t)stream;
   const float* sc = scores;
-  if (!sc) {
+  if (sc) {  // K, V and the scores may be page-locked host memory
+    K = device_address(K);
+    V = device_address(V);
+    sc = (const float*)device_address(sc);
+    if (!K || !V || !sc || !aligned16(K) || !aligned16(V)) return EBD_ERR_INVALID;
+  } else {
+    // scoring reads every key: K and the observation queries in device memory
     if (!q_obs || n_obs < 1) return EBD_ERR_INVALID;
+    if (!is_device_memory(K) || !is_device_memory(q_obs)) return EBD_ERR_UNSUPPORTED;
+    V = device_address(V);
+    if (!V) return EBD_ERR_INVALID;
     const size_t need = ebd_evict_workspace_bytes(design, n_obs);
     if (!workspace || ws_bytes < need) return EBD_ERR_CAPACITY;
     const size_t units = (size_t)design->batch * design->n_kv_heads;
@@ -1278,7 +1319,9 @@ extern "C" ebd_status ebd_select(const ebd_design* design, const float* scores, 
   ebd_status st = check_design(design);
   if (st != EBD_OK) return st;
   if (!scores || !idx_c || !logw_c || !n_kept || !dev_status || capacity < 1) return EBD_ERR_INVALID;
-  return launch_select(design, scores, nullptr, nullptr, nullptr, idx_c, logw_c, n_kept, capacity,
+  const float* sc = (const float*)device_address(scores);
+  if (!sc) return EBD_ERR_INVALID;
+  return launch_select(design, sc, nullptr, nullptr, nullptr, idx_c, logw_c, n_kept, capacity,
                        dev_status, (cudaStream_t)stream);
 }
 
@@ -1292,6 +1335,9 @@ extern "C" ebd_status ebd_gather(const ebd_design* design, ebd_dtype dtype, cons
   const int eb = dtype == EBD_F32 ? 4 : 2;
   if (design->head_dim < 1 || (design->head_dim * eb) % 16 != 0) return EBD_ERR_UNSUPPORTED;
   if (!aligned16(K) || !aligned16(V) || !aligned16(K_c) || !aligned16(V_c)) return EBD_ERR_INVALID;
+  K = device_address(K);  // page-locked host rows are read over the host link
+  V = device_address(V);
+  if (!K || !V || !aligned16(K) || !aligned16(V)) return EBD_ERR_INVALID;
   return launch_gather(design, dtype, K, V, idx_c, n_kept, capacity, K_c, V_c,
                        (cudaStream_t)stream);
 }

@@ -47,6 +47,12 @@ ebd_status launch_gather_range(const ebd_design* d, ebd_dtype dtype, const void*
 
 bool aligned16(const void* p);
 
+// Address under which kernels read a caller's buffer: device or managed memory
+// as is, page-locked host memory through its device mapping (read over the
+// host link); nullptr for memory the device cannot address (evict.cu).
+const void* device_address(const void* p);
+bool is_device_memory(const void* p);
+
 // E0: accumulated attention scores into `scores` using `workspace` for the
 // per-row log-sum-exp.  Arguments validated by the caller; dev_status nullable.
 ebd_status launch_score(ebd_dtype dtype, int batch, int n_kv_heads, int head_dim, int n_ctx,

@@ -285,8 +285,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   uint64_t* acc_full = bars + 5;   // [2] accumulator halves
   uint64_t* acc_empty = bars + 7;  // [2]
   uint64_t* lse_ready = bars + 9;   // the epilogue staged a unit's row log-sum-exps
-  uint64_t* part_ready = bars + 10;  // warps 4-15 left their partial key sums
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 11);
+  uint64_t* part_ready = bars + 10;  // [2] warps 4-15 left their partial key sums (item parity)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nkt = (a.n_ctx + kTcKeys2 - 1) / kTcKeys2;
@@ -302,7 +302,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_init(&acc_empty[s], kTcEpi);
     }
     mbar_init(lse_ready, kTcEpi);
-    mbar_init(part_ready, kTcEpi - 128);
+    mbar_init(&part_ready[0], kTcEpi - 128);
+    mbar_init(&part_ready[1], kTcEpi - 128);
     fence_barrier_init();
   }
   if (warp == kTcIssueWarp) {
@@ -458,9 +459,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       float* pb = part + (i & 1) * kTcGroups * 128;
       if (grp != 0) {
         pb[grp * 128 + row] = sum;
-        mbar_arrive(part_ready);  // release
+        mbar_arrive(&part_ready[i & 1]);  // release
       } else {
-        if (!mbar_wait_bounded(part_ready, i & 1)) {
+        // one barrier per buffer: an arrival for item i + 1 can never count
+        // toward item i's phase
+        if (!mbar_wait_bounded(&part_ready[i & 1], (i >> 1) & 1)) {
           ok = false;
           break;
         }

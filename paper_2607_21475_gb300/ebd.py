@@ -1,9 +1,11 @@
 """Thin Python binding of libebd (include/ebd.h): argument marshalling only.
 
 Each function carries the name of the C entry point it calls and takes torch
-tensors that already live on the GPU; it checks shapes, dtypes and
-contiguity, passes raw device pointers plus sizes, and raises ``EbdError`` on
-a non-OK status.  Every step of the hot path runs in the library's CUDA
+tensors that already live on the GPU (the eviction calls also take K, V and
+the scores as page-locked CPU tensors: the library then reads the scores and
+only the kept rows from host memory); it checks shapes, dtypes and
+contiguity, passes raw pointers plus sizes, and raises ``EbdError`` on a
+non-OK status.  Every step of the hot path runs in the library's CUDA
 kernels.  PyTorch supplies device memory and the current stream.
 
 If the compiled library is missing the import of any entry point raises: there
@@ -143,13 +145,16 @@ def _dtype_code(t: torch.Tensor) -> int:
     raise TypeError(f"unsupported dtype {t.dtype}; expected float32 or bfloat16")
 
 
-def _ptr(t, dtype=None, shape=None, name="tensor"):
+def _ptr(t, dtype=None, shape=None, name="tensor", host_ok=False):
+    """Address of a contiguous tensor.  host_ok: a page-locked CPU tensor is
+    accepted too (the library reads it from the device over the host link)."""
     if t is None:
         return None
     if not isinstance(t, torch.Tensor):
         raise TypeError(f"{name} must be a torch.Tensor")
-    if not t.is_cuda:
-        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_cuda and not (host_ok and t.is_pinned()):
+        raise ValueError(f"{name} must be a CUDA tensor" +
+                         (" or a page-locked CPU tensor" if host_ok else ""))
     if not t.is_contiguous():
         raise ValueError(f"{name} must be contiguous")
     if dtype is not None and t.dtype != dtype:
@@ -224,7 +229,7 @@ def ebd_compute_pi(design: EbdDesign, scores: torch.Tensor, pi: torch.Tensor,
                    certain_mask=None, dev_status=None, stream=None):
     shp = (design.batch, design.n_kv_heads, design.n_ctx)
     _check("ebd_compute_pi", lib().ebd_compute_pi(
-        ctypes.byref(design), _ptr(scores, torch.float32, shp, "scores"),
+        ctypes.byref(design), _ptr(scores, torch.float32, shp, "scores", True),
         _ptr(pi, torch.float32, shp, "pi"), _ptr(certain_mask, torch.uint8, shp, "certain_mask"),
         _ptr(dev_status, torch.int32, (1,), "dev_status"), _stream(stream)))
     return pi
@@ -271,9 +276,11 @@ def ebd_evict(design: EbdDesign, K: torch.Tensor, V: torch.Tensor, scores, q_obs
     ws, wsb = (None, 0)
     if scores is None:
         ws, wsb = _workspace(ebd_evict_workspace_bytes(design, n_obs), K.device, workspace)
+    host_ok = scores is not None  # K, V, scores may stay in page-locked host memory
     _check("ebd_evict", lib().ebd_evict(
-        ctypes.byref(design), dt, _ptr(K, K.dtype, (B, H, N, d), "K"),
-        _ptr(V, K.dtype, (B, H, N, d), "V"), _ptr(scores, torch.float32, (B, H, N), "scores"),
+        ctypes.byref(design), dt, _ptr(K, K.dtype, (B, H, N, d), "K", host_ok),
+        _ptr(V, K.dtype, (B, H, N, d), "V", True),
+        _ptr(scores, torch.float32, (B, H, N), "scores", True),
         _ptr(q_obs, K.dtype, None if q_obs is None else (B, H, n_obs, d), "q_obs"), n_obs,
         _ptr(out.K_c, K.dtype, (B, H, cap, d), "K_c"), _ptr(out.V_c, K.dtype, (B, H, cap, d), "V_c"),
         _ptr(out.logw_c, torch.float32, (B, H, cap), "logw_c"),
@@ -288,7 +295,7 @@ def ebd_select(design: EbdDesign, scores: torch.Tensor, out: CompactCache, strea
     B, H, N = design.batch, design.n_kv_heads, design.n_ctx
     cap = out.capacity
     _check("ebd_select", lib().ebd_select(
-        ctypes.byref(design), _ptr(scores, torch.float32, (B, H, N), "scores"),
+        ctypes.byref(design), _ptr(scores, torch.float32, (B, H, N), "scores", True),
         _ptr(out.idx_c, torch.int32, (B, H, cap), "idx_c"),
         _ptr(out.logw_c, torch.float32, (B, H, cap), "logw_c"),
         _ptr(out.n_kept, torch.int32, (B, H), "n_kept"), cap,
@@ -302,8 +309,9 @@ def ebd_gather(design: EbdDesign, K: torch.Tensor, V: torch.Tensor, out: Compact
     B, H, N, d = design.batch, design.n_kv_heads, design.n_ctx, design.head_dim
     cap = out.capacity
     _check("ebd_gather", lib().ebd_gather(
-        ctypes.byref(design), _dtype_code(K), _ptr(K, K.dtype, (B, H, N, d), "K"),
-        _ptr(V, K.dtype, (B, H, N, d), "V"), _ptr(out.idx_c, torch.int32, (B, H, cap), "idx_c"),
+        ctypes.byref(design), _dtype_code(K), _ptr(K, K.dtype, (B, H, N, d), "K", True),
+        _ptr(V, K.dtype, (B, H, N, d), "V", True),
+        _ptr(out.idx_c, torch.int32, (B, H, cap), "idx_c"),
         _ptr(out.n_kept, torch.int32, (B, H), "n_kept"), cap,
         _ptr(out.K_c, K.dtype, (B, H, cap, d), "K_c"), _ptr(out.V_c, K.dtype, (B, H, cap, d), "V_c"),
         _stream(stream)))

@@ -228,6 +228,48 @@ def test_evict_pipelined_chunks_match_single_stream_and_oracle(E, B, H, N, d, dt
                            Kb[b, h], Vb[b, h], cap)
 
 
+def test_evict_from_page_locked_host_memory_matches_device(E):
+    """K, V and the scores left in page-locked host memory: the select reads the
+    scores and the gather only the kept rows over the host link; the outputs
+    equal those of the same call on device copies.  Pageable host memory is
+    refused before any launch."""
+    import ctypes
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    B, H, N, d, cap = 24, 8, 2048, 128, 384   # more units than SMs: pipelined chunks
+    assert B * H > sms
+    g = torch.Generator().manual_seed(5)
+    K = torch.randn((B, H, N, d), generator=g).to(torch.bfloat16)
+    V = torch.randn((B, H, N, d), generator=g).to(torch.bfloat16)
+    s = torch.exp(1.5 * torch.randn((B, H, N), generator=g))
+    des = _design(E, B, H, 4, d, N, 1, 9, N // 50, N // 10)
+    dev = E.alloc_compact(B, H, cap, d, torch.bfloat16, DEV)
+    E.ebd_evict(des, K.to(DEV), V.to(DEV), s.to(DEV), None, dev)
+    host = E.alloc_compact(B, H, cap, d, torch.bfloat16, DEV)
+    Kp, Vp, sp = K.pin_memory(), V.pin_memory(), s.pin_memory()
+    E.ebd_evict(des, Kp, Vp, sp, None, host)
+    sel = E.alloc_compact(B, H, cap, d, torch.bfloat16, DEV)   # the two halves alone
+    E.ebd_select(des, sp, sel)
+    E.ebd_gather(des, Kp, Vp, sel)
+    torch.cuda.synchronize()
+    for cc in (host, sel):
+        assert cc.dev_status.item() == 0
+        assert torch.equal(cc.n_kept, dev.n_kept)
+        for b in range(B):
+            for h in range(H):
+                n = min(int(dev.n_kept[b, h]), cap)
+                for f in ("idx_c", "logw_c", "K_c", "V_c"):
+                    assert torch.equal(getattr(cc, f)[b, h, :n], getattr(dev, f)[b, h, :n]), f
+    # pageable memory: the binding refuses it, and so does the C entry point
+    with pytest.raises(ValueError):
+        E.ebd_gather(des, K, V, sel)
+    st = E.lib().ebd_gather(ctypes.byref(des), E.EBD_BF16, ctypes.c_void_p(K.data_ptr()),
+                            ctypes.c_void_p(V.data_ptr()), ctypes.c_void_p(sel.idx_c.data_ptr()),
+                            ctypes.c_void_p(sel.n_kept.data_ptr()), cap,
+                            ctypes.c_void_p(sel.K_c.data_ptr()), ctypes.c_void_p(sel.V_c.data_ptr()),
+                            ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    assert st == 1  # EBD_ERR_INVALID
+
+
 def test_evict_capacity_overflow_is_flagged_and_bounded(E):
     B, H, N, d = 1, 2, 2000, 64
     cap = 64  # far below the ~400 kept tokens
