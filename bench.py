@@ -69,6 +69,12 @@ def parse_args():
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--batch", type=int, default=0,
                    help="override the workload's batch (smaller cases for profiling)")
+    p.add_argument("--sweep", action="store_true",
+                   help="instead of the step: the batch x context x budget sweep on the 28/4 "
+                        "GQA shape, one JSON line per point (decode GB/s and roofline "
+                        "fraction, pipelined eviction Mtokens/s)")
+    p.add_argument("--sweep-filter", default="",
+                   help="only sweep points whose name contains this string")
     p.add_argument("--rows", action="store_true",
                    help="instead of the step: time the added rows (append/re-eviction cadence, "
                         "certificate aggregation, systematic select, observation queries, "
@@ -828,11 +834,77 @@ def run_rows(args):
     return lines
 
 
+def run_sweep(args):
+    """Batch {1,8,32,64} x N {4k,16k,64k,128k} x budget {5,10,25,50}% on the
+    28/4-head, d=128, bf16 shape with log-normal scores: one layer per point,
+    eviction (ebd_evict, pipelined) and certified decode each captured in a
+    CUDA graph and timed alone (median of `--steps` runs, L2 flushed before
+    each).  One JSON line per point."""
+    from paper_2607_21475_gb300 import ebd
+    from paper_2607_21475_gb300.workloads import sweep_workloads
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    hbm_peak, peak_kind, _ = measured_peaks()
+    time_us = _timer(dev, max(args.steps, 5))
+    for w in sweep_workloads():
+        if args.sweep_filter and args.sweep_filter not in w.name:
+            continue
+        B, H, G, d, N = w.batch, w.n_kv_heads, w.group, w.head_dim, w.n_ctx
+        inp = make_layer_inputs(w, 0, dev)
+        des = ebd.design_for(batch=B, n_kv_heads=H, group=G, head_dim=d, n_ctx=N, layer=0,
+                             seed=w.philox_seed, n_sink=w.n_sink, n_recent=w.n_recent,
+                             k_head=w.k_head, budget_tokens=w.budget_tokens,
+                             bisect_iters=w.bisect_iters, eps=w.eps)
+        cc = ebd.alloc_compact(B, H, w.capacity, d, w.torch_dtype, dev)
+        Hq = H * G
+        y = torch.empty((B, Hq, d), dtype=torch.float32, device=dev)
+        o4 = [torch.empty((B, Hq), dtype=torch.float32, device=dev) for _ in range(4)]
+        ws = torch.empty(max(1, ebd.ebd_decode_workspace_bytes(ebd.EBD_BF16, B, H, G, d,
+                                                               w.capacity)),
+                         dtype=torch.uint8, device=dev)
+
+        def evict():
+            ebd.ebd_evict(des, inp["K"], inp["V"], inp["scores"], None, cc)
+
+        def decode():
+            ebd.ebd_certified_decode(inp["Q"], cc.K_c, cc.V_c, cc.logw_c, cc.n_kept, y, *o4,
+                                     workspace=ws)
+
+        evict()
+        decode()
+        torch.cuda.synchronize()
+        if cc.dev_status.item():
+            raise RuntimeError(f"{w.name}: device status {cc.dev_status.item()}")
+        graphs = {}
+        for name, fn in (("evict", evict), ("decode", decode)):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                fn()
+            graphs[name] = g
+        ev_us = time_us(graphs["evict"].replay)
+        dec_us = time_us(graphs["decode"].replay)
+        n_kept = [torch.clamp(cc.n_kept, max=w.capacity).cpu().numpy()]
+        dbytes = decode_bytes(w, n_kept)
+        gbs = dbytes / (dec_us * 1e-6) / 1e9
+        print(json.dumps({
+            "point": w.name, "batch": B, "n_ctx": N, "budget": w.budget,
+            "q_heads": Hq, "kv_heads": H, "head_dim": d, "kv_dtype": w.dtype,
+            "decode_us": dec_us, "decode_bytes": dbytes, "decode_gbs": gbs,
+            "decode_frac_of_measured_hbm": gbs / hbm_peak, "decode_pct_of_8tbs": gbs / 80.0,
+            "evict_us": ev_us, "evict_mtok_s": B * N / (ev_us * 1e-6) / 1e6,
+            "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"}))
+        del inp, cc, y, o4, ws, graphs
+        torch.cuda.empty_cache()
+
+
 def main():
     args = parse_args()
     world, rank, local = dist_setup(args)
     if args.impl == "reference":
         run_reference(args, world, rank)
+    elif args.sweep:
+        if rank == 0:
+            run_sweep(args)
     elif args.rows:
         if rank == 0:
             run_rows(args)

@@ -141,12 +141,88 @@ __device__ __forceinline__ float tail_pi(float s, int mode, float c, float eps) 
   return fminf(1.f, fmaxf(eps, c * s));
 }
 
-__global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs a) {
-  extern __shared__ uint32_t cert_bits[];  // bit i set <=> token i in A
-  __shared__ BlockScratch sh;
-  __shared__ unsigned hist[256];
-  __shared__ unsigned sh_prefix, sh_remaining;
-  __shared__ int sh_bad;
+// ---------------------------------------------------------------------------
+// Large contexts (N > 32768): the scores stay in global memory (L2-resident
+// while the unit is worked on).  Every pass walks them in steps of 4096
+// tokens, thread t taking tokens 4t .. 4t + 3 of a step (one float4 load; one
+// Philox call gives the draws of all four), four steps per round so that four
+// loads per thread are in flight.  The certainty set is a bit array in shared
+// memory.  Passes: four radix digits (per-warp histograms for the first), the
+// top-slice pass (with an ordered scan of the ties only when fewer of them are
+// needed than there are), one stats pass, the water-filling solve of Eq. (2)
+// (bisection steps replaced by the exact linear solve of the current partition
+// when it lands in the bracket; 1-5 passes as a rule), one draw + compaction
+// pass with one ordered scan per step.
+// ---------------------------------------------------------------------------
+constexpr int kBigStep = 4 * kSelThreads;  // tokens per step
+constexpr int kBigUnroll = 4;              // steps per round
+
+struct BigScratch {
+  unsigned hist[256];
+  int tot[kSelWarps];
+  float rf[3][kSelWarps];
+  int ri[2][kSelWarps];
+  double res_d;
+  float res_f[2];
+  int res_i[2];
+  float c, lo, hi;  // solve state, updated by thread 0 only
+  int mode, stop;
+  unsigned prefix, remaining, eqcount;
+};
+
+// Scores of tokens i0 .. i0 + 3 (0 at and past N); non-finite values read as 0
+// and reported through `bad`; -0 folded onto +0.
+__device__ __forceinline__ void load4(const float* s, int i0, int N, bool vec4, float (&v)[4],
+                                      bool& bad) {
+  if (vec4 && i0 + 3 < N) {
+    const float4 t = __ldg(reinterpret_cast<const float4*>(s + i0));
+    v[0] = t.x;
+    v[1] = t.y;
+    v[2] = t.z;
+    v[3] = t.w;
+  } else {
+#pragma unroll
+    for (int r = 0; r < 4; ++r) v[r] = i0 + r < N ? __ldg(s + i0 + r) : 0.f;
+  }
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    if (!isfinite(v[r])) {
+      bad = bad || (i0 + r < N);
+      v[r] = 0.f;
+    }
+    v[r] += 0.0f;
+  }
+}
+
+// Exclusive prefix over the block, in thread order, of `cnt`, and the block
+// total; two barriers (sh.tot is free again when it returns).
+__device__ __forceinline__ int big_scan(int cnt, int& total, BigScratch& sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int incl = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int n = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += n;
+  }
+  if (lane == 31) sh.tot[warp] = incl;
+  __syncthreads();
+  int before = 0, tot = 0;
+#pragma unroll 8
+  for (int w = 0; w < kSelWarps; ++w) {
+    const int c = sh.tot[w];
+    before += w < warp ? c : 0;
+    tot += c;
+  }
+  __syncthreads();
+  total = tot;
+  return before + incl - cnt;
+}
+
+__global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs a, int words_pad) {
+  extern __shared__ uint32_t big_smem[];
+  __shared__ BigScratch sh;
+  uint32_t* cert_bits = big_smem;            // bit i set <=> token i in A
+  unsigned* whist = big_smem + words_pad;    // [kSelWarps][256] first-digit histograms
 
   const int unit = a.unit0 + blockIdx.x;
   const int b = unit / a.n_kv_heads;
@@ -154,48 +230,83 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
   const int Nrow = a.n_ctx;
   const int N = a.n_len ? min(max(__ldg(a.n_len + unit), 0), Nrow) : Nrow;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int words = (N + 31) >> 5;
   const float* s = a.scores + (size_t)unit * Nrow;
-
+  const bool vec4 = a.vec4 != 0;
   const int ns = min(a.n_sink, N);
   const int rs = max(N - a.n_recent, 0);  // first protected trailing position
-
-  if (tid == 0) sh_bad = 0;
-  bool bad = false;
-  // protected positions
-  for (int base = 0; base < N; base += kSelThreads) {
-    const int i = base + tid;
-    const bool prot = (i < N) && (i < ns || i >= rs);
-    const unsigned bits = __ballot_sync(0xffffffffu, prot);
-    const int wd = (base >> 5) + warp;
-    if (lane == 0 && wd < words) cert_bits[wd] = bits;
-  }
   const int n_prot = ns + (N - rs) - max(0, ns - rs);
   const int n_cand = N - n_prot;
   const int k = min(max(a.k_head, 0), n_cand);
+  const float eps = a.eps;
+  bool bad = false;
+  auto cand = [&](int i) { return i < N && i >= ns && i < rs; };
+  // the nibble of tokens i0 .. i0 + 3 (i0 % 4 == 0) in the certainty bits
+  auto cert4 = [&](int i0) { return (cert_bits[i0 >> 5] >> (i0 & 31)) & 0xFu; };
+  // the eight threads of a word combine their nibbles; one of them stores it
+  auto put4 = [&](int i0, uint32_t n4, bool assign) {
+    uint32_t v = n4 << (i0 & 31);
+    v |= __shfl_xor_sync(0xffffffffu, v, 1);
+    v |= __shfl_xor_sync(0xffffffffu, v, 2);
+    v |= __shfl_xor_sync(0xffffffffu, v, 4);
+    if ((lane & 7) == 0 && i0 < N) cert_bits[i0 >> 5] = assign ? v : (cert_bits[i0 >> 5] | v);
+  };
+
+  // protected positions
+  for (int base = 0; base < N; base += kBigStep) {
+    const int i0 = base + 4 * tid;
+    uint32_t p4 = 0u;
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+      if (i0 + r < N && !cand(i0 + r)) p4 |= 1u << r;
+    put4(i0, p4, true);
+  }
   __syncthreads();
 
-  // ---- E1: top-k among unprotected tokens ---------------------------------
+  // ---- E1: top-k_head among the unprotected tokens ------------------------
   if (k > 0 && k < n_cand) {
     unsigned prefix = 0u, maskbits = 0u, remaining = (unsigned)k;
+#pragma unroll 1
     for (int shift = 24; shift >= 0; shift -= 8) {
-      for (int j = tid; j < 256; j += kSelThreads) hist[j] = 0u;
+      for (int j = tid; j < 256; j += kSelThreads) sh.hist[j] = 0u;
+      unsigned* wh = whist + warp * 256;
+      if (shift == 24)
+        for (int j = lane; j < 256; j += 32) wh[j] = 0u;
       __syncthreads();
-      for (int i = tid; i < N; i += kSelThreads) {
-        if (i < ns || i >= rs) continue;
-        float v = __ldg(s + i);
-        if (!isfinite(v)) { bad = true; v = 0.f; }
-        const uint32_t key = orderable_key(v);
-        if ((key & maskbits) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+#pragma unroll 1
+      for (int base = 0; base < N; base += kBigStep * kBigUnroll) {
+        float v[kBigUnroll][4];
+#pragma unroll
+        for (int q = 0; q < kBigUnroll; ++q)
+          load4(s, base + q * kBigStep + 4 * tid, N, vec4, v[q], bad);
+#pragma unroll
+        for (int q = 0; q < kBigUnroll; ++q) {
+          const int i0 = base + q * kBigStep + 4 * tid;
+#pragma unroll
+          for (int r = 0; r < 4; ++r) {
+            if (!cand(i0 + r)) continue;
+            const uint32_t key = orderable_key(v[q][r]);
+            if (shift == 24) atomicAdd(&wh[key >> 24], 1u);
+            else if ((key & maskbits) == prefix) atomicAdd(&sh.hist[(key >> shift) & 255u], 1u);
+          }
+        }
       }
       __syncthreads();
+      if (shift == 24) {
+        for (int j = tid; j < 256; j += kSelThreads) {
+          unsigned t = 0u;
+#pragma unroll 8
+          for (int w = 0; w < kSelWarps; ++w) t += whist[w * 256 + j];
+          sh.hist[j] = t;
+        }
+        __syncthreads();
+      }
       if (warp == 0) {
         // lane L owns bins 255-8L .. 248-8L (descending key order)
         unsigned c[8];
         unsigned tot = 0;
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
-          c[q] = hist[255 - 8 * lane - q];
+          c[q] = sh.hist[255 - 8 * lane - q];
           tot += c[q];
         }
         unsigned incl = tot;
@@ -210,8 +321,9 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
 #pragma unroll
           for (int q = 0; q < 8; ++q) {
             if (cum + c[q] >= remaining) {
-              sh_prefix = prefix | ((unsigned)(255 - 8 * lane - q) << shift);
-              sh_remaining = remaining - cum;
+              sh.prefix = prefix | ((unsigned)(255 - 8 * lane - q) << shift);
+              sh.remaining = remaining - cum;
+              sh.eqcount = c[q];  // tokens whose key matches the prefix so far
               break;
             }
             cum += c[q];
@@ -219,32 +331,52 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
         }
       }
       __syncthreads();
-      prefix = sh_prefix;
-      remaining = sh_remaining;
+      prefix = sh.prefix;
+      remaining = sh.remaining;
       maskbits |= 255u << shift;
     }
-    // prefix = k-th largest key; take every key above it and the `remaining`
-    // lowest-index tokens equal to it.
+    // prefix is the k-th largest key: every key above it joins A, and the
+    // `remaining` lowest-index tokens equal to it (all of them, without an
+    // ordered scan, when there are no more than that)
+    const bool all_eq = sh.eqcount <= remaining;
     int taken = 0;
-    for (int base = 0; base < N; base += kSelThreads) {
-      const int i = base + tid;
-      bool eq = false, gt = false;
-      if (i < N && !(i < ns || i >= rs)) {
-        float v = __ldg(s + i);
-        if (!isfinite(v)) v = 0.f;
-        const uint32_t key = orderable_key(v);
-        eq = key == prefix;
-        gt = key > prefix;
+#pragma unroll 1
+    for (int base = 0; base < N; base += kBigStep * kBigUnroll) {
+      float v[kBigUnroll][4];
+#pragma unroll
+      for (int q = 0; q < kBigUnroll; ++q)
+        load4(s, base + q * kBigStep + 4 * tid, N, vec4, v[q], bad);
+#pragma unroll
+      for (int q = 0; q < kBigUnroll; ++q) {
+        const int i0 = base + q * kBigStep + 4 * tid;
+        uint32_t gt4 = 0u, eq4 = 0u;
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          if (!cand(i0 + r)) continue;
+          const uint32_t key = orderable_key(v[q][r]);
+          if (key > prefix) gt4 |= 1u << r;
+          else if (key == prefix) eq4 |= 1u << r;
+        }
+        uint32_t sel4 = gt4;
+        if (all_eq) {
+          sel4 |= eq4;
+        } else {
+          int total;
+          int run = taken + big_scan(__popc(eq4), total, sh);
+#pragma unroll
+          for (int r = 0; r < 4; ++r) {
+            if ((eq4 >> r) & 1u) {
+              if (run < (int)remaining) sel4 |= 1u << r;
+              ++run;
+            }
+          }
+          taken += total;
+        }
+        put4(i0, sel4, false);
       }
-      int total;
-      const int rank = block_rank(eq, total, sh);
-      const bool sel = gt || (eq && taken + rank < (int)remaining);
-      const unsigned bits = __ballot_sync(0xffffffffu, sel);
-      const int wd = (base >> 5) + warp;
-      if (lane == 0 && wd < words) cert_bits[wd] |= bits;
-      taken += total;
     }
   } else if (k > 0) {  // every unprotected token is in the top slice
+    const int words = (N + 31) >> 5;
     for (int wd = tid; wd < words; wd += kSelThreads) {
       unsigned m = 0xffffffffu;
       if (wd == words - 1 && (N & 31)) m = (1u << (N & 31)) - 1u;
@@ -257,110 +389,186 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
   const int n_cert = n_prot + k;
   const int nT = N - n_cert;
   const int m = min(max(a.budget - n_cert, 0), nT);
-  float smax = -INFINITY, sminpos = INFINITY;
-  int npos = 0;
-  for (int i = tid; i < N; i += kSelThreads) {
-    if ((cert_bits[i >> 5] >> (i & 31)) & 1u) continue;
-    float v = __ldg(s + i);
-    if (!isfinite(v)) { bad = true; v = 0.f; }
-    smax = fmaxf(smax, v);
-    if (v > 0.f) {
-      sminpos = fminf(sminpos, v);
-      ++npos;
-    }
-  }
-  smax = block_max_f(smax, sh);
-  sminpos = block_min_f(sminpos, sh);
-  npos = block_sum_i(npos, sh);
-
-  const float eps = a.eps;
-  int mode = kPiLinear;
-  float c = 0.f;
-  if (nT == 0 || (float)m <= eps * (float)nT) {
-    mode = kPiFloor;
-  } else if ((float)m >= (float)npos + eps * (float)(nT - npos)) {
-    mode = kPiAll;
-  } else {
-    float lo = logf(eps / smax), hi = logf(1.f / sminpos);
-    for (int it = 0; it < a.iters; ++it) {
-      const float mid = 0.5f * (lo + hi);
-      const float cm = expf(mid);
-      float g = 0.f;
-      for (int i = tid; i < N; i += kSelThreads) {
-        if ((cert_bits[i >> 5] >> (i & 31)) & 1u) continue;
-        float v = __ldg(s + i);
-        if (!isfinite(v)) v = 0.f;
-        g += fminf(1.f, fmaxf(eps, cm * v));
+  {
+    float smax = -INFINITY, sminpos = INFINITY, spos = 0.f;
+    int npos = 0;
+#pragma unroll 1
+    for (int base = 0; base < N; base += kBigStep * kBigUnroll) {
+      float v[kBigUnroll][4];
+#pragma unroll
+      for (int q = 0; q < kBigUnroll; ++q)
+        load4(s, base + q * kBigStep + 4 * tid, N, vec4, v[q], bad);
+#pragma unroll
+      for (int q = 0; q < kBigUnroll; ++q) {
+        const int i0 = base + q * kBigStep + 4 * tid;
+        const uint32_t c4 = i0 < N ? cert4(i0) : 0xFu;
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          if (i0 + r >= N || ((c4 >> r) & 1u)) continue;
+          smax = fmaxf(smax, v[q][r]);
+          if (v[q][r] > 0.f) {
+            sminpos = fminf(sminpos, v[q][r]);
+            spos += v[q][r];
+            ++npos;
+          }
+        }
       }
-      g = block_sum_f2d(g, sh);
-      if (g < (float)m) lo = mid; else hi = mid;
     }
-    // exact solve inside the partition found at the upper end of the bracket
-    const float cb = expf(hi);
-    int n_hi = 0, n_lo = 0;
-    double smid = 0.0;
-    for (int i = tid; i < N; i += kSelThreads) {
-      if ((cert_bits[i >> 5] >> (i & 31)) & 1u) continue;
-      float v = __ldg(s + i);
-      if (!isfinite(v)) v = 0.f;
-      const float t = cb * v;
-      if (t >= 1.f) ++n_hi;
-      else if (t <= eps) ++n_lo;
-      else smid += (double)v;
+    smax = warp_max(smax);
+    sminpos = warp_min(sminpos);
+    npos = warp_sum(npos);
+    spos = warp_sum(spos);
+    if (lane == 0) {
+      sh.rf[0][warp] = smax;
+      sh.rf[1][warp] = sminpos;
+      sh.rf[2][warp] = spos;
+      sh.ri[0][warp] = npos;
     }
-    n_hi = block_sum_i(n_hi, sh);
-    n_lo = block_sum_i(n_lo, sh);
-    smid = block_sum_d(smid, sh);
-    const double cstar = ((double)m - n_hi - (double)eps * n_lo) / smid;
-    const double clo = exp((double)lo), chi = exp((double)hi);
-    if (smid > 0.0 && cstar >= clo * (1.0 - 1e-6) && cstar <= chi * (1.0 + 1e-6))
-      c = (float)cstar;
-    else
-      c = expf(0.5f * (lo + hi));
+    __syncthreads();
+    if (warp == 0) {
+      float mx = sh.rf[0][lane], mn = sh.rf[1][lane];
+      double sd = (double)sh.rf[2][lane];
+      int np = sh.ri[0][lane];
+      mx = warp_max(mx);
+      mn = warp_min(mn);
+      sd = warp_sum(sd);
+      np = warp_sum(np);
+      if (lane == 0) {
+        // scalar decisions once, by thread 0, and broadcast
+        int md = kPiLinear;
+        if (nT == 0 || (float)m <= eps * (float)nT) md = kPiFloor;
+        else if ((float)m >= (float)np + eps * (float)(nT - np)) md = kPiAll;
+        sh.mode = md;
+        sh.stop = md != kPiLinear;
+        if (md == kPiLinear) {
+          sh.lo = logf(eps / mx);
+          sh.hi = logf(1.f / mn);
+          sh.c = fminf(fmaxf((float)((double)m / sd), expf(sh.lo)), expf(sh.hi));
+        } else {
+          sh.c = 0.f;
+        }
+      }
+    }
+    __syncthreads();
+  }
+  const int mode = sh.mode;
+  float c = sh.c;
+#pragma unroll 1
+  for (int it = 0; it < a.iters && !sh.stop; ++it) {
+    int nhi = 0, nlo = 0;
+    float smid = 0.f;
+#pragma unroll 1
+    for (int base = 0; base < N; base += kBigStep * kBigUnroll) {
+      float v[kBigUnroll][4];
+#pragma unroll
+      for (int q = 0; q < kBigUnroll; ++q)
+        load4(s, base + q * kBigStep + 4 * tid, N, vec4, v[q], bad);
+#pragma unroll
+      for (int q = 0; q < kBigUnroll; ++q) {
+        const int i0 = base + q * kBigStep + 4 * tid;
+        const uint32_t c4 = i0 < N ? cert4(i0) : 0xFu;
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          if (i0 + r >= N || ((c4 >> r) & 1u)) continue;
+          const float t = c * v[q][r];
+          if (t >= 1.f) ++nhi;
+          else if (t <= eps) ++nlo;
+          else smid += v[q][r];
+        }
+      }
+    }
+    nhi = warp_sum(nhi);
+    nlo = warp_sum(nlo);
+    smid = warp_sum(smid);
+    __syncthreads();  // the previous iteration's readers of sh are done
+    if (lane == 0) {
+      sh.ri[0][warp] = nhi;
+      sh.ri[1][warp] = nlo;
+      sh.rf[0][warp] = smid;
+    }
+    __syncthreads();
+    if (warp == 0) {
+      double sd = (double)sh.rf[0][lane];
+      int ah = sh.ri[0][lane], al = sh.ri[1][lane];
+      sd = warp_sum(sd);
+      ah = warp_sum(ah);
+      al = warp_sum(al);
+      if (lane == 0) {
+        const double gval = ah + (double)eps * al + (double)c * sd;
+        float lo = sh.lo, hi = sh.hi;
+        if (gval < (double)m) lo = fmaxf(lo, logf(c));
+        else hi = fminf(hi, logf(c));
+        const double clin = sd > 0.0 ? ((double)m - ah - (double)eps * al) / sd : -1.0;
+        if (clin > 0.0 && fabs(clin - (double)c) <= 1e-6 * (double)c) {
+          sh.c = (float)clin;  // the partition at c reproduces its own solve
+          sh.stop = 1;
+        } else {
+          float next;
+          const float lcl = clin > 0.0 ? logf((float)clin) : -INFINITY;
+          if (clin > 0.0 && lcl > lo && lcl < hi) next = (float)clin;
+          else next = expf(0.5f * (lo + hi));
+          if (next == c) sh.stop = 1;
+          sh.c = next;
+        }
+        sh.lo = lo;
+        sh.hi = hi;
+      }
+    }
+    __syncthreads();
+    c = sh.c;
   }
 
   // ---- E3 + E4a: draws, stable compaction of (index, log 1/pi) -------------
   const bool compact = a.n_kept != nullptr;
   int kept = 0;
-  for (int base = 0; base < N; base += kSelThreads) {
-    const int i = base + tid;
-    bool keep = false;
-    float pi = 1.f;
-    bool cert = false;
-    if (i < N) {
-      cert = (cert_bits[i >> 5] >> (i & 31)) & 1u;
-      if (!cert) {
-        float v = __ldg(s + i);
-        if (!isfinite(v)) { bad = true; v = 0.f; }
-        pi = tail_pi(v, mode, c, eps);
+#pragma unroll 1
+  for (int base = 0; base < N; base += kBigStep * kBigUnroll) {
+    float v[kBigUnroll][4];
+#pragma unroll
+    for (int q = 0; q < kBigUnroll; ++q)
+      load4(s, base + q * kBigStep + 4 * tid, N, vec4, v[q], bad);
+#pragma unroll
+    for (int q = 0; q < kBigUnroll; ++q) {
+      const int i0 = base + q * kBigStep + 4 * tid;
+      const uint32_t c4 = i0 < N ? cert4(i0) : 0xFu;
+      uint4 w = make_uint4(0u, 0u, 0u, 0u);
+      if (compact && i0 < N) w = draw_block(a.seed, a.layer, b, kvh, i0 >> 2);
+      const uint32_t wr[4] = {w.x, w.y, w.z, w.w};
+      float pis[4];
+      uint32_t keep4 = 0u;
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const int i = i0 + r;
+        pis[r] = 1.f;
+        if (i >= N) continue;
+        const bool ct = (c4 >> r) & 1u;
+        const float pi = ct ? 1.f : tail_pi(v[q][r], mode, c, eps);
+        pis[r] = pi;
+        if (a.pi_out) a.pi_out[(size_t)unit * Nrow + i] = pi;
+        if (a.mask_out) a.mask_out[(size_t)unit * Nrow + i] = ct ? 1 : 0;
+        if (compact && (ct || word_to_uniform(wr[r]) < pi)) keep4 |= 1u << r;
       }
-      if (a.pi_out) a.pi_out[(size_t)unit * Nrow + i] = pi;
-      if (a.mask_out) a.mask_out[(size_t)unit * Nrow + i] = cert ? 1 : 0;
       if (compact) {
-        const float u = word_to_uniform(draw_word(a.seed, a.layer, b, kvh, i));
-        keep = cert || (u < pi);
+        int total;
+        int p = kept + big_scan(__popc(keep4), total, sh);
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          if (!((keep4 >> r) & 1u)) continue;
+          if (p < a.cap) {
+            a.idx_c[(size_t)unit * a.cap + p] = i0 + r;
+            a.logw_c[(size_t)unit * a.cap + p] = pis[r] >= 1.f ? 0.f : -logf(pis[r]);
+          }
+          ++p;
+        }
+        kept += total;
       }
     }
-    if (compact) {
-      int total;
-      const int rank = block_rank(keep, total, sh);
-      const int p = kept + rank;
-      if (keep && p < a.cap) {
-        a.idx_c[(size_t)unit * a.cap + p] = i;
-        a.logw_c[(size_t)unit * a.cap + p] = (cert || pi >= 1.f) ? 0.f : -logf(pi);
-      }
-      kept += total;
-    }
   }
-  if (bad) sh_bad = 1;
-  __syncthreads();
-  if (tid == 0) {
-    if (compact) {
-      a.n_kept[unit] = kept;
-      if (kept > a.cap) raise_status(a.dev_status, EBD_DEV_CAPACITY);
-    }
-    if (sh_bad) raise_status(a.dev_status, EBD_DEV_NONFINITE);
+  if (compact && tid == 0) {
+    a.n_kept[unit] = kept;
+    if (kept > a.cap) raise_status(a.dev_status, EBD_DEV_CAPACITY);
   }
+  if (__syncthreads_or(bad) && tid == 0) raise_status(a.dev_status, EBD_DEV_NONFINITE);
 }
 
 // ---------------------------------------------------------------------------
@@ -1029,11 +1237,13 @@ ebd_status launch_select_range(const ebd_design* d, const float* scores, const i
     evict_select_smem_kernel<<<units, kRegThreads, smem, stream>>>(a, groups);
     return launch_status();
   }
-  const size_t smem = (size_t)((d->n_ctx + 31) / 32) * 4;
+  // certainty bits (padded to 16 bytes), then the per-warp first-digit histograms
+  const int words_pad = ((d->n_ctx + 31) / 32 + 3) & ~3;
+  const size_t smem = (size_t)words_pad * 4 + (size_t)kSelWarps * 256 * 4;
   if (cudaFuncSetAttribute(evict_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)smem) != cudaSuccess)
     return EBD_ERR_CUDA;
-  evict_select_kernel<<<units, kSelThreads, smem, stream>>>(a);
+  evict_select_kernel<<<units, kSelThreads, smem, stream>>>(a, words_pad);
   return launch_status();
 }
 

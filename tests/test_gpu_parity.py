@@ -70,6 +70,8 @@ PI_CASES = [
     (6144, 307, 1536, "signed"),      # zero / negative scores sit at the floor
     (32768, 655, 3277, "segments"),
     (70001, 1400, 7000, "lognormal"),  # ragged, beyond one smem tile of bits
+    (50000, 1000, 5000, "ties"),       # large context: ordered scan of the tied top keys
+    (40000, 0, 12000, "pareto"),       # large context, no top slice, clipped tail
 ]
 
 
@@ -137,6 +139,8 @@ EVICT_CASES = [
     (1, 2, 37, 64, torch.float32, 2, 20, 64),
     (2, 2, 4097, 128, torch.bfloat16, 80, 410, 576),
     (1, 1, 1, 64, torch.float32, 2, 1, 64),
+    (1, 2, 40000, 64, torch.float32, 800, 4000, 4480),      # large context (global scores)
+    (2, 1, 65537, 128, torch.bfloat16, 1300, 6500, 7104),   # large, ragged (scalar loads)
 ]
 
 
