@@ -1,0 +1,306 @@
+// Certified decode on thread-block clusters, for requests with few units (at
+// most half as many (batch row, KV head) units as SMs): one cluster of C = 2,
+// 4 or 8 CTAs per unit, C the largest that keeps units * C <= SMs.
+//
+// CTA r of a unit's cluster takes tiles [r T / C, (r + 1) T / C) of the unit's
+// T active 16-token tiles and splits them into eight contiguous ranges, one
+// per warp; every warp streams its range through a private cp.async ring and
+// folds it with the same per-tile step as the split-K kernel (decode_tile.cuh).
+// The partial states then meet without leaving the chip: the eight warps' in
+// shared memory (over the ring), where warp g combines query head g; the
+// cluster's CTAs' in the shared memory of CTA 0, written through distributed
+// shared memory; after one cluster barrier CTA 0 combines them and writes
+// y_hat, log N_hat, V_hat, b_t and r_t (Eq. 3, Theorem 2, Eq. 4).  One launch,
+// no workspace, no merge kernel.  Combination rule: w-terms (l, o, cmax,
+// umax) scale by e^(M_part - M), u-terms (U, A2, A1) by its square.
+#include <cuda_runtime.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "decode.cuh"
+#include "decode_tile.cuh"
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ebd {
+
+struct ClusterArgs {
+  const __nv_bfloat16* Q;   // [units * G, D]
+  const __nv_bfloat16* Kc;  // [units, cap, D]
+  const __nv_bfloat16* Vc;
+  const float* logw;        // [units, cap]
+  const int32_t* n_kept;    // [units]
+  int cap;
+  int group;
+  int csize;                // CTAs per cluster (per unit)
+  int lw_off;               // shared-memory layout, bytes: log(1/pi) stages
+  int lead_off;             // CTA records gathered in CTA 0: [csize][G][rec_floats(D)]
+  float* y;
+  float* lse;
+  float* var;
+  float* b_t;
+  float* radius;
+  float log_inv_delta;
+  float eps0;
+  bool exact;               // b_t / radius come from the exact range pass
+};
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t cluster_map(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void st_cluster4(uint32_t addr, float a, float b, float c, float d) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(a), "f"(b),
+               "f"(c), "f"(d)
+               : "memory");
+}
+// Every thread of every CTA of the cluster; writes before it are visible to
+// reads after it across the cluster.
+__device__ __forceinline__ void cluster_barrier() {
+  asm volatile(
+      "barrier.cluster.arrive.release.aligned;\n\t"
+      "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Combine n <= NMAX records (stride rec_floats(D) floats) of one query head;
+// lane holds columns PER * lane .. + PER - 1 of o and A1.
+template <int D>
+struct HeadSum {
+  static constexpr int PER = D / 32;
+  float M, l, U, A2, cm, um;
+  float o[PER], a1[PER];
+  template <int NMAX>
+  __device__ __forceinline__ void combine(const float* recs, int n, size_t stride, int lane) {
+    M = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < NMAX; ++k)
+      if (k < n) M = fmaxf(M, recs[k * stride + kRecM]);
+    l = U = A2 = cm = um = 0.f;
+#pragma unroll
+    for (int e = 0; e < PER; ++e) o[e] = a1[e] = 0.f;
+#pragma unroll
+    for (int k = 0; k < NMAX; ++k) {
+      if (k >= n) break;
+      const float* R = recs + k * stride;
+      const float Mk = R[kRecM];
+      if (Mk == -INFINITY) continue;
+      const float f = expf(Mk - M), f2 = f * f;
+      l = fmaf(f, R[kRecL], l);
+      U = fmaf(f2, R[kRecU], U);
+      A2 = fmaf(f2, R[kRecA2], A2);
+      cm = fmaxf(cm, f * R[kRecCmax]);
+      um = fmaxf(um, f * R[kRecUmax]);
+#pragma unroll
+      for (int e = 0; e < PER; ++e) {
+        o[e] = fmaf(f, R[kRecHead + PER * lane + e], o[e]);
+        a1[e] = fmaf(f2, R[kRecHead + D + PER * lane + e], a1[e]);
+      }
+    }
+  }
+};
+
+template <int D, int S>
+__global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterArgs a) {
+  using L = MmaTileLayout<D>;
+  constexpr int REC = rec_floats(D);
+  constexpr int PER = D / 32;
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem =
+      (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);  // swizzle atoms
+  float* lw_s = reinterpret_cast<float*>(smem + a.lw_off);
+  float* lead = reinterpret_cast<float*>(smem + a.lead_off);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int C = a.csize, G = a.group;
+  const uint32_t rank = cluster_rank();
+  const int unit = blockIdx.x / C;
+  const int n_u = min(max(__ldg(a.n_kept + unit), 0), a.cap);
+  const int T = (n_u + kMmaTile - 1) / kMmaTile;
+  const int c0 = (int)((long long)rank * T / C), c1 = (int)((long long)(rank + 1) * T / C);
+  const int tb = c0 + (int)((long long)warp * (c1 - c0) / kMmaConsumers);
+  const int te = c0 + (int)((long long)(warp + 1) * (c1 - c0) / kMmaConsumers);
+  const float kscale = kLog2e * rsqrtf((float)D);
+  const size_t row_base = (size_t)unit * a.cap;
+
+  TileAcc<D> st;
+  tile_acc_begin<D>(st, a.Q, unit, G, lane);
+  int issued = 0;
+  auto issue_next = [&]() {
+    const int t = tb + issued;
+    if (t < te) {
+      const int stage = warp * S + issued % S;
+      tile_copy<D>(smem + (size_t)stage * L::kStageBytes, lw_s + stage * kMmaTile, a.Kc, a.Vc,
+                   a.logw, row_base + (size_t)t * kMmaTile, lane);
+    }
+    cp_async_commit();
+    ++issued;
+  };
+#pragma unroll
+  for (int p = 0; p < S - 1; ++p) issue_next();
+  int j = 0;
+  for (int t = tb; t < te; ++t, ++j) {
+    issue_next();  // tile j + S - 1 into the stage tile j - 1 left
+    const int s = warp * S + j % S;
+    cp_async_wait<S - 1>();  // this lane's copies of tile j are done
+    __syncwarp();            // and every lane's
+    tile_consume<D>(st, smem_u32(smem + (size_t)s * L::kStageBytes), lw_s + s * kMmaTile,
+                    min(kMmaTile, n_u - t * kMmaTile), lane, kscale);
+  }
+  cp_async_wait<0>();
+  __syncthreads();  // the ring is free: the warps' records go over it
+
+  float* wrec = reinterpret_cast<float*>(smem);  // [warps][G][REC]
+  tile_acc_store<D>(st, wrec + (size_t)warp * G * REC, G, lane);
+  __syncthreads();
+  if (warp < G) {  // this CTA's part of query head `warp`, sent to CTA 0
+    HeadSum<D> h;
+    h.combine<kMmaConsumers>(wrec + (size_t)warp * REC, kMmaConsumers, (size_t)G * REC, lane);
+    const uint32_t dst = cluster_map(smem_u32(lead + ((size_t)rank * G + warp) * REC), 0);
+    if (lane == 0) {
+      st_cluster4(dst + 4 * kRecM, h.M, h.l, h.U, h.A2);
+      st_cluster4(dst + 4 * kRecCmax, h.cm, h.um, 0.f, 0.f);
+    }
+    if constexpr (PER == 4) {  // 16-byte stores: lane holds columns 4 lane .. + 3
+      st_cluster4(dst + 4 * (kRecHead + 4 * lane), h.o[0], h.o[1], h.o[2], h.o[3]);
+      st_cluster4(dst + 4 * (kRecHead + D + 4 * lane), h.a1[0], h.a1[1], h.a1[2], h.a1[3]);
+    } else {  // lanes 2k and 2k + 1 hold columns 4k .. 4k + 3: even lanes store both
+      const float o2 = __shfl_down_sync(0xffffffffu, h.o[0], 1);
+      const float o3 = __shfl_down_sync(0xffffffffu, h.o[1], 1);
+      const float b2 = __shfl_down_sync(0xffffffffu, h.a1[0], 1);
+      const float b3 = __shfl_down_sync(0xffffffffu, h.a1[1], 1);
+      if ((lane & 1) == 0) {
+        st_cluster4(dst + 4 * (kRecHead + 2 * lane), h.o[0], h.o[1], o2, o3);
+        st_cluster4(dst + 4 * (kRecHead + D + 2 * lane), h.a1[0], h.a1[1], b2, b3);
+      }
+    }
+  }
+  cluster_barrier();
+  if (rank != 0 || warp >= G) return;
+
+  HeadSum<D> h;
+  h.combine<8>(lead + (size_t)warp * REC, C, (size_t)G * REC, lane);
+  const long long hq = (long long)unit * G + warp;
+  if (h.M == -INFINITY) {  // no retained row: y = 0, lse = -inf, zero certificate
+#pragma unroll
+    for (int e = 0; e < PER; ++e) a.y[hq * D + PER * lane + e] = 0.f;
+    if (lane == 0) {
+      a.lse[hq] = -INFINITY;
+      a.var[hq] = 0.f;
+      a.b_t[hq] = 0.f;
+      a.radius[hq] = 0.f;
+    }
+    return;
+  }
+  float yy = 0.f, ya = 0.f;
+#pragma unroll
+  for (int e = 0; e < PER; ++e) {
+    const float yv = h.o[e] / h.l;
+    a.y[hq * D + PER * lane + e] = yv;
+    yy = fmaf(yv, yv, yy);
+    ya = fmaf(yv, h.a1[e], ya);
+  }
+  yy = warp_sum(yy);
+  ya = warp_sum(ya);
+  if (lane == 0) {
+    const float ynorm = sqrtf(yy);
+    const float var = fmaxf(0.f, (h.A2 - 2.f * ya + yy * h.U) / (h.l * h.l));
+    a.lse[hq] = h.M + logf(h.l);
+    a.var[hq] = var;
+    if (a.exact) {
+      a.b_t[hq] = 0.f;  // filled by the exact range pass
+    } else {
+      const float bt = (h.cm + ynorm * h.um) / h.l;
+      a.b_t[hq] = bt;
+      a.radius[hq] = (sqrtf(2.f * var * a.log_inv_delta) + bt * a.log_inv_delta) / (ynorm + a.eps0);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+template <int D, int S>
+static ebd_status launch_cluster_t(const DecodeArgs& d, const ReduceArgs& r, int units, int C,
+                                   cudaStream_t s) {
+  using L = MmaTileLayout<D>;
+  ClusterArgs a;
+  a.Q = reinterpret_cast<const __nv_bfloat16*>(d.Q);
+  a.Kc = reinterpret_cast<const __nv_bfloat16*>(d.Kc);
+  a.Vc = reinterpret_cast<const __nv_bfloat16*>(d.Vc);
+  a.logw = d.logw;
+  a.n_kept = d.n_kept;
+  a.cap = d.cap;
+  a.group = d.group;
+  a.csize = C;
+  a.lw_off = kMmaConsumers * S * L::kStageBytes;
+  a.lead_off = (int)align_up((size_t)a.lw_off + (size_t)kMmaConsumers * S * kMmaTile * 4, 16);
+  a.y = r.y;
+  a.lse = r.lse;
+  a.var = r.var;
+  a.b_t = r.b_t;
+  a.radius = r.radius;
+  a.log_inv_delta = r.log_inv_delta;
+  a.eps0 = r.eps0;
+  a.exact = r.exact;
+  const size_t smem = (size_t)a.lead_off + (size_t)C * d.group * rec_floats(D) * 4 + 1024;
+  if (cudaFuncSetAttribute(decode_cluster_kernel<D, S>,
+                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+    return EBD_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(units * C));
+  cfg.blockDim = dim3(kMmaThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cuda_status(cudaLaunchKernelEx(&cfg, decode_cluster_kernel<D, S>, a));
+}
+
+// Shared memory of a cluster CTA with S ring stages.
+static size_t cluster_smem(int D, int S, int C, int G) {
+  const size_t stage = (size_t)2 * (D / 64) * kMmaTile * 128;
+  const size_t lw = align_up((size_t)kMmaConsumers * S * stage + kMmaConsumers * S * kMmaTile * 4, 16);
+  return lw + (size_t)C * G * rec_floats(D) * 4 + 1024;
+}
+
+int cluster_decode_size(int units, int cap) {
+  const int sms = sm_count();
+  if (units < 1 || 2 * units > sms) return 0;
+  int C = 2;
+  while (C < 8 && 2 * C * units <= sms) C *= 2;
+  // measured: the on-chip combine pays off only when the clusters cover most
+  // SMs and every CTA streams a long range (at least 48 tiles at capacity);
+  // otherwise the split-K kernels over every SM are faster
+  if (4 * units * C < 3 * sms) return 0;
+  if ((cap / kMmaTile) / C < 48) return 0;
+  return C;
+}
+
+ebd_status launch_cluster_decode(int head_dim, const DecodeArgs& d, const ReduceArgs& r,
+                                 int units, cudaStream_t s) {
+  const int C = cluster_decode_size(units, d.cap);
+  if (C == 0) return EBD_ERR_UNSUPPORTED;
+  const size_t max_smem = 227 * 1024;
+  const bool three = cluster_smem(head_dim, 3, C, d.group) <= max_smem;
+  if (head_dim == 128)
+    return three ? launch_cluster_t<128, 3>(d, r, units, C, s)
+                 : launch_cluster_t<128, 2>(d, r, units, C, s);
+  if (head_dim == 64)
+    return three ? launch_cluster_t<64, 3>(d, r, units, C, s)
+                 : launch_cluster_t<64, 2>(d, r, units, C, s);
+  return EBD_ERR_UNSUPPORTED;
+}
+
+}  // namespace ebd

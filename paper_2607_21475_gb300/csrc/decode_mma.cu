@@ -17,17 +17,8 @@
 // the head's records over its warps, combines them in shared memory and
 // writes y_hat, lse, V_hat, b_t and r_t.
 //
-// Per tile and warp:
-//   S[16 x 16]  = Qpad[16 x d] . K_tile^T       (rows 0..G-1 = query heads,
-//                                                rows 8..15 = 0; 2 x d/16 mma)
-//   w = 2^(S log2e/sqrt(d) + log2e log(1/pi) - M), u = (1 - pi) w^2
-//   P[16 x 16]  = [w (rows 0..7); u (rows 8..15)] as bf16 hi + bf16 lo parts
-//   acc[16 x d] += P_hi . V_tile + P_lo . V_tile   (rows 0..7: o, rows 8..15: A1)
-// The hi/lo split keeps ~16 mantissa bits of the weights on bf16 tensor
-// cores.  ||v||^2 per token comes from the same V fragments (squares summed
-// over the lanes that hold one token).  The running maximum is updated
-// lazily: accumulators are rescaled only when a row's maximum grows by more
-// than 2^8, so weights stay below 2^8 and u below 2^16.
+// The per-tile step (Q K^T, weights, [w; u] V on mma.sync with hi/lo weight
+// parts, ||v||^2, lazy rescale) lives in decode_tile.cuh.
 //
 // Each warp streams its own tiles: all 32 lanes issue 16-byte cp.async copies
 // of K, V (into the 128-byte-swizzled layout ldmatrix reads) and log(1/pi) for
@@ -43,25 +34,20 @@
 
 #include "common.cuh"
 #include "decode.cuh"
+#include "decode_tile.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 
 namespace ebd {
 
-constexpr int kMmaTile = 16;
-constexpr int kMmaConsumers = 8;  // warps per CTA
 constexpr int kMmaStagesPerWarp = 3;
 constexpr int kMmaStages = kMmaConsumers * kMmaStagesPerWarp;
-constexpr int kMmaThreads = kMmaConsumers * 32;
-constexpr float kRescaleLog2 = 8.f;
 constexpr int kMinTilesPerWarp = 4;
 constexpr int kLocalUnits = 4096;  // tile prefix kept in shared memory up to this many units
 
 template <int D>
 struct MmaLayout {
-  static constexpr int kHalves = D / 64;                 // 64-column (128-byte) boxes per row
-  static constexpr int kBoxBytes = kMmaTile * 128;      // one box: 16 rows x 128 B
-  static constexpr int kStageBytes = 2 * kHalves * kBoxBytes;
+  static constexpr int kStageBytes = MmaTileLayout<D>::kStageBytes;
   static constexpr int kLogwOff = kMmaStages * kStageBytes;
   static constexpr int kScanOff = kLogwOff + kMmaStages * kMmaTile * 4;  // [kMmaConsumers] ints
   static constexpr int kPlanOff = kScanOff + 64;                  // [kLocalUnits + 1] ints
@@ -238,33 +224,19 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
   const int tb = (int)(gw * Ta / W);
   const int te = (int)((gw + 1) * Ta / W);
   const int G = a.group;
-  const int g = lane >> 2, q = lane & 3;
   const float kscale = kLog2e * rsqrtf((float)D);
 
-  // copies: the warp walks its tiles with one cursor; every lane copies 16-byte
-  // chunks of K and V into the 128-byte-swizzled stage layout (chunk ch of row
-  // r of a 64-column half at r * 128 + ((ch ^ (r & 7)) << 4)) and lanes 0-3 the
-  // tile's log(1/pi); one commit group per tile (empty past the range)
+  // copies: the warp walks its tiles with one cursor, one commit group per
+  // tile (empty past the range)
   int pf_t = tb, pf_u = unit_of_tile(toff, units, tb);
   int pf_lo = toff[pf_u], pf_hi = toff[pf_u + 1];
   int issued = 0;
   auto issue_next = [&]() {
     if (pf_t < te) {
-      constexpr int CPR = D / 8;                   // 16-byte chunks per row
-      constexpr int PER = kMmaTile * CPR / 32;     // chunks per lane per tile (K or V)
       const int stage = warp * kMmaStagesPerWarp + issued % kMmaStagesPerWarp;
       const size_t row0 = (size_t)pf_u * a.cap + (size_t)(pf_t - pf_lo) * kMmaTile;
-      unsigned char* st = smem + (size_t)stage * L::kStageBytes;
-#pragma unroll
-      for (int i = 0; i < PER; ++i) {
-        const int c = lane + 32 * i;
-        const int r = c / CPR, ch = c - r * CPR;
-        const int off = (ch >> 3) * L::kBoxBytes + r * 128 + (((ch & 7) ^ (r & 7)) << 4);
-        const size_t src = (row0 + r) * D + ch * 8;
-        cp_async16(st + off, a.Kc + src);
-        cp_async16(st + L::kHalves * L::kBoxBytes + off, a.Vc + src);
-      }
-      if (lane < kMmaTile / 4) cp_async16(lw_s + stage * kMmaTile + 4 * lane, a.logw + row0 + 4 * lane);
+      tile_copy<D>(smem + (size_t)stage * L::kStageBytes, lw_s + stage * kMmaTile, a.Kc, a.Vc,
+                   a.logw, row0, lane);
       ++pf_t;
       if (pf_t < te && pf_t == pf_hi) {
         pf_u = next_unit(toff, pf_u);
@@ -276,55 +248,17 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     ++issued;
   };
 
-  float acc[D / 8][4];
-  float M2 = -INFINITY, l = 0.f, U = 0.f, A2 = 0.f, cmax = 0.f, umax = 0.f;
-  uint32_t qa[D / 16][2];
+  TileAcc<D> st;
   int u = pf_u;
   int seg_end = 0, n_u = 0, seg_start = 0;
-
   auto begin_segment = [&]() {
     seg_start = toff[u];
     seg_end = toff[u + 1];
     n_u = min(__ldg(a.n_kept + u), a.cap);
-    const uint32_t* qrow =
-        reinterpret_cast<const uint32_t*>(a.Q + ((size_t)u * G + (g < G ? g : 0)) * D);
-#pragma unroll
-    for (int kk = 0; kk < D / 16; ++kk) {
-      qa[kk][0] = g < G ? __ldg(qrow + 8 * kk + q) : 0u;
-      qa[kk][1] = g < G ? __ldg(qrow + 8 * kk + 4 + q) : 0u;
-    }
-#pragma unroll
-    for (int j = 0; j < D / 8; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
-    M2 = -INFINITY;
-    l = U = A2 = cmax = umax = 0.f;
+    tile_acc_begin<D>(st, a.Q, u, G, lane);
   };
-
   auto flush_segment = [&]() {
-#pragma unroll
-    for (int o = 1; o <= 2; o <<= 1) {
-      l += __shfl_xor_sync(0xffffffffu, l, o);
-      U += __shfl_xor_sync(0xffffffffu, U, o);
-      A2 += __shfl_xor_sync(0xffffffffu, A2, o);
-      cmax = fmaxf(cmax, __shfl_xor_sync(0xffffffffu, cmax, o));
-      umax = fmaxf(umax, __shfl_xor_sync(0xffffffffu, umax, o));
-    }
-    if (g < G) {
-      float* rec = a.part + ((size_t)(u + gw) * G + g) * REC;
-      if (q == 0) {
-        rec[kRecM] = M2 == -INFINITY ? -INFINITY : M2 * kLn2;
-        rec[kRecL] = l;
-        rec[kRecU] = U;
-        rec[kRecA2] = A2;
-        rec[kRecCmax] = cmax;
-        rec[kRecUmax] = umax;
-      }
-#pragma unroll
-      for (int j = 0; j < D / 8; ++j) {
-        *reinterpret_cast<float2*>(rec + kRecHead + 8 * j + 2 * q) = make_float2(acc[j][0], acc[j][1]);
-        *reinterpret_cast<float2*>(rec + kRecHead + D + 8 * j + 2 * q) =
-            make_float2(acc[j][2], acc[j][3]);
-      }
-    }
+    tile_acc_store<D>(st, a.part + (size_t)(u + gw) * G * REC, G, lane);
   };
 
   // prologue: the first stages of the ring
@@ -344,124 +278,8 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     const int s = warp * kMmaStagesPerWarp + j % kMmaStagesPerWarp;
     cp_async_wait<kMmaStagesPerWarp - 1>();  // this lane's copies of tile j are done
     __syncwarp();                             // and every lane's
-    const uint32_t kbase = smem_u32(smem + (size_t)s * L::kStageBytes);
-    const uint32_t vbase = kbase + L::kHalves * L::kBoxBytes;
-
-    // ---- S = Q K^T ---------------------------------------------------------
-    float sc0[4] = {0.f, 0.f, 0.f, 0.f}, sc1[4] = {0.f, 0.f, 0.f, 0.f};
-    {
-      const int tok = ((lane >> 4) << 3) + (lane & 7);
-      const int half_sel = (lane >> 3) & 1;
-#pragma unroll
-      for (int kk = 0; kk < D / 16; ++kk) {
-        const int chunk = 2 * kk + half_sel;
-        const uint32_t addr = kbase + (chunk >> 3) * L::kBoxBytes + tok * 128 +
-                              (((chunk & 7) ^ (tok & 7)) << 4);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(addr, b0, b1, b2, b3);
-        mma_bf16_16816(sc0, qa[kk][0], 0u, qa[kk][1], 0u, b0, b1);
-        mma_bf16_16816(sc1, qa[kk][0], 0u, qa[kk][1], 0u, b2, b3);
-      }
-    }
-
-    // ---- weights -----------------------------------------------------------
-    const float2 lwa = *reinterpret_cast<const float2*>(lw_s + s * kMmaTile + 2 * q);
-    const float2 lwb = *reinterpret_cast<const float2*>(lw_s + s * kMmaTile + 8 + 2 * q);
-    const float lwv[4] = {lwa.x, lwa.y, lwb.x, lwb.y};
-    const int tk[4] = {2 * q, 2 * q + 1, 8 + 2 * q, 9 + 2 * q};
-    const float sv[4] = {sc0[0], sc0[1], sc1[0], sc1[1]};
-    float x[4];
-    float mx = -INFINITY;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      x[i] = tk[i] < n_valid ? fmaf(sv[i], kscale, lwv[i] * kLog2e) : -INFINITY;
-      mx = fmaxf(mx, x[i]);
-    }
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-    if (mx > M2 + kRescaleLog2) {
-      const float f = exp2f(M2 - mx), f2 = f * f;
-#pragma unroll
-      for (int jj = 0; jj < D / 8; ++jj) {
-        acc[jj][0] *= f;
-        acc[jj][1] *= f;
-        acc[jj][2] *= f2;
-        acc[jj][3] *= f2;
-      }
-      l *= f;
-      U *= f2;
-      A2 *= f2;
-      cmax *= f;
-      umax *= f;
-      M2 = mx;
-    }
-    float wv[4], uv[4], suv[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const bool val = tk[i] < n_valid;
-      wv[i] = exp2f(x[i] - M2);
-      const float omp = val ? one_minus_exp_neg(lwv[i]) : 0.f;  // 1 - pi
-      uv[i] = omp * wv[i] * wv[i];
-      suv[i] = sqrtf(omp) * wv[i];
-      umax = fmaxf(umax, suv[i]);
-    }
-    const uint32_t h0 = pack_bf16(wv[0], wv[1]), h1 = pack_bf16(uv[0], uv[1]);
-    const uint32_t h2 = pack_bf16(wv[2], wv[3]), h3 = pack_bf16(uv[2], uv[3]);
-    const uint32_t r0 = pack_bf16(wv[0] - bf16_lo(h0), wv[1] - bf16_hi(h0));
-    const uint32_t r1 = pack_bf16(uv[0] - bf16_lo(h1), uv[1] - bf16_hi(h1));
-    const uint32_t r2 = pack_bf16(wv[2] - bf16_lo(h2), wv[3] - bf16_hi(h2));
-    const uint32_t r3 = pack_bf16(uv[2] - bf16_lo(h3), uv[3] - bf16_hi(h3));
-    // The scalar sums use exactly the weights the tensor cores multiply with
-    // (hi + lo), so that V_hat = (A2 - 2 y.A1 + |y|^2 U) / l^2 cancels
-    // consistently when y_hat sits close to the retained values.
-    const float wt[4] = {bf16_lo(h0) + bf16_lo(r0), bf16_hi(h0) + bf16_hi(r0),
-                         bf16_lo(h2) + bf16_lo(r2), bf16_hi(h2) + bf16_hi(r2)};
-    const float ut[4] = {bf16_lo(h1) + bf16_lo(r1), bf16_hi(h1) + bf16_hi(r1),
-                         bf16_lo(h3) + bf16_lo(r3), bf16_hi(h3) + bf16_hi(r3)};
-    l += (wt[0] + wt[1]) + (wt[2] + wt[3]);
-    U += (ut[0] + ut[1]) + (ut[2] + ut[3]);
-
-    // ---- acc += P V, ||v||^2 -------------------------------------------------
-    const uint32_t m01 = (tk[0] < n_valid ? 0x0000ffffu : 0u) | (tk[1] < n_valid ? 0xffff0000u : 0u);
-    const uint32_t m23 = (tk[2] < n_valid ? 0x0000ffffu : 0u) | (tk[3] < n_valid ? 0xffff0000u : 0u);
-    float2 vn01 = make_float2(0.f, 0.f), vn23 = make_float2(0.f, 0.f);
-    {
-      const int tok = ((lane >> 3) & 1) * 8 + (lane & 7);
-      const int chunk_sel = lane >> 4;
-#pragma unroll
-      for (int jp = 0; jp < D / 16; ++jp) {
-        const int chunk = 2 * jp + chunk_sel;
-        const uint32_t addr = vbase + (chunk >> 3) * L::kBoxBytes + tok * 128 +
-                              (((chunk & 7) ^ (tok & 7)) << 4);
-        uint32_t v0, v1, v2, v3;
-        ldsm_x4_trans(addr, v0, v1, v2, v3);
-        v0 &= m01;
-        v2 &= m01;
-        v1 &= m23;
-        v3 &= m23;
-        const float2 f0 = make_float2(bf16_lo(v0), bf16_hi(v0));
-        const float2 f1 = make_float2(bf16_lo(v1), bf16_hi(v1));
-        const float2 f2 = make_float2(bf16_lo(v2), bf16_hi(v2));
-        const float2 f3 = make_float2(bf16_lo(v3), bf16_hi(v3));
-        vn01 = __ffma2_rn(f0, f0, __ffma2_rn(f2, f2, vn01));
-        vn23 = __ffma2_rn(f1, f1, __ffma2_rn(f3, f3, vn23));
-        mma_bf16_16816(acc[2 * jp], h0, h1, h2, h3, v0, v1);
-        mma_bf16_16816(acc[2 * jp], r0, r1, r2, r3, v0, v1);
-        mma_bf16_16816(acc[2 * jp + 1], h0, h1, h2, h3, v2, v3);
-        mma_bf16_16816(acc[2 * jp + 1], r0, r1, r2, r3, v2, v3);
-      }
-    }
-    // every lane's reads of this stage are done before it is refilled
-    __syncwarp();
-    float vn[4] = {vn01.x, vn01.y, vn23.x, vn23.y};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      vn[i] += __shfl_xor_sync(0xffffffffu, vn[i], 4);
-      vn[i] += __shfl_xor_sync(0xffffffffu, vn[i], 8);
-      vn[i] += __shfl_xor_sync(0xffffffffu, vn[i], 16);
-      A2 = fmaf(ut[i], vn[i], A2);
-      cmax = fmaxf(cmax, suv[i] * sqrtf(vn[i]));
-    }
+    tile_consume<D>(st, smem_u32(smem + (size_t)s * L::kStageBytes), lw_s + s * kMmaTile,
+                    n_valid, lane, kscale);
   }
   flush_segment();
   cp_async_wait<0>();
@@ -735,6 +553,12 @@ ebd_status launch_fast_decode(ebd_dtype dtype, int head_dim, const DecodePlan& p
                               const DecodeArgs& a, const ReduceArgs& r, int units, void* ws,
                               cudaStream_t stream) {
   if (dtype != EBD_BF16) return EBD_ERR_UNSUPPORTED;
+  // few units: one cluster of CTAs per unit, combined on chip (decode_cluster.cu);
+  // should that launch be refused, the split-K kernels below take the request
+  if (cluster_decode_size(units, a.cap) > 0) {
+    if (launch_cluster_decode(head_dim, a, r, units, stream) == EBD_OK) return EBD_OK;
+    cudaGetLastError();
+  }
   if (head_dim == 128) return launch_fast_t<128>(plan, a, r, units, ws, stream);
   if (head_dim == 64) return launch_fast_t<64>(plan, a, r, units, ws, stream);
   return EBD_ERR_UNSUPPORTED;

@@ -327,6 +327,12 @@ DECODE_CASES = [
     (2, 3, 5, 128, 1000, torch.bfloat16, "random"),  # capacity not a multiple of 16: CUDA cores
     (1, 64, 4, 128, 256, torch.bfloat16, "random"),  # more warps than tiles
     (1, 1, 8, 128, 32768, torch.bfloat16, "full"),    # one unit, hundreds of partial records
+    # cluster kernel (units * C covering most SMs, long per-CTA ranges)
+    (16, 4, 7, 128, 1600, torch.bfloat16, "edges"),   # 64 units, clusters of 2, empty units
+    (8, 8, 8, 64, 1600, torch.bfloat16, "random"),    # head_dim 64, G = 8
+    # split-K with more units than half the SMs
+    (8, 12, 4, 128, 256, torch.bfloat16, "edges"),    # 96 units
+    (10, 10, 8, 64, 160, torch.bfloat16, "random"),   # 100 units, head_dim 64
 ]
 
 
