@@ -280,11 +280,11 @@ int cluster_decode_size(int units, int cap) {
   if (units < 1 || 2 * units > sms) return 0;
   int C = 2;
   while (C < 8 && 2 * C * units <= sms) C *= 2;
-  // measured: the on-chip combine pays off only when the clusters cover most
-  // SMs and every CTA streams a long range (at least 48 tiles at capacity);
+  // measured: the on-chip combine pays off when the clusters cover most SMs
+  // and every CTA has a few tiles to stream (at least 8 at capacity);
   // otherwise the split-K kernels over every SM are faster
   if (4 * units * C < 3 * sms) return 0;
-  if ((cap / kMmaTile) / C < 48) return 0;
+  if ((cap / kMmaTile) / C < 8) return 0;
   return C;
 }
 
