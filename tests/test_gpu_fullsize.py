@@ -167,3 +167,33 @@ def test_fullsize_sweep_points(E, B, N, beta):
     assert decoded >= 1
     del inp, cc, out
     _cleanup()
+
+
+@pytest.mark.parametrize("N", [1 << 20, (1 << 20) - 3])
+def test_maximum_context_eviction(E, N):
+    """The largest context the library takes (2^20 tokens; and a ragged one
+    just below, read with scalar loads): certainty set, pi, draws and
+    compaction against the oracle, on one unit with head_dim 64."""
+    d, k_head, budget = 64, round(0.02 * N), round(0.10 * N)
+    cap = (budget + int(8 * budget ** 0.5) + 64 + 63) // 64 * 64
+    g = torch.Generator().manual_seed(N % 997)
+    K = torch.randn((1, 1, N, d), generator=g)
+    V = torch.randn((1, 1, N, d), generator=g)
+    s = torch.exp(1.5 * torch.randn((1, 1, N), generator=g))
+    des = E.design_for(batch=1, n_kv_heads=1, group=1, head_dim=d, n_ctx=N, layer=1, seed=5,
+                       k_head=k_head, budget_tokens=budget)
+    cc = E.alloc_compact(1, 1, cap, d, torch.float32, DEV)
+    E.ebd_evict(des, K.to(DEV), V.to(DEV), s.to(DEV), None, cc)
+    torch.cuda.synchronize()
+    assert cc.dev_status.item() == 0
+    ref = O.evict_unit(K[0, 0].double().numpy(), V[0, 0].double().numpy(), s[0, 0].numpy(),
+                       n_sink=4, n_recent=32, k_head=k_head, budget_tokens=budget, eps=1e-6,
+                       seed=5, layer=1, b=0, kvh=0, capacity=cap)
+    n = int(cc.n_kept[0, 0])
+    kg = min(n, cap)
+    compare_evict_unit(ref, n, cc.idx_c[0, 0, :kg].cpu().numpy(),
+                       cc.logw_c[0, 0, :kg].cpu().double().numpy(),
+                       bits(cc.K_c[0, 0, :kg]), bits(cc.V_c[0, 0, :kg]), bits(K[0, 0]),
+                       bits(V[0, 0]), cap)
+    del K, V, s, cc
+    _cleanup()
