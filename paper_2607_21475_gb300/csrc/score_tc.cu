@@ -10,7 +10,9 @@
 // epilogue thread that owns a lane keeps that row's running
 // (max, sum 2^(x - max)) without any cross-thread traffic.  Two accumulators
 // (256 columns each) alternate so the MMA of tile j + 1 overlaps the epilogue
-// of tile j.  Output: the base-2 log-sum-exp of every row (workspace).
+// of tile j; three shared-memory stages of K let the copy of tile j + 2 start
+// when the MMA of tile j - 1 is done.  Output: the base-2 log-sum-exp of
+// every row (workspace).
 // Pass 2, score_col_tc_kernel: the transposed product S^T = K Q^T, keys as M
 // (one key per lane), all R query rows as N (split in two halves of <= 256
 // columns, one per accumulator), so key j's thread sums 2^(x_rj - lse_r) over
@@ -57,8 +59,11 @@ struct Tc1Layout {
   static constexpr int kQBox = kTcRows1 * 128;       // 16 KB
   static constexpr int kKBox = kTcKeys1 * 128;       // 32 KB
   static constexpr int kKOff = kHalves * kQBox;
-  static constexpr int kPartOff = kKOff + 2 * kHalves * kKBox;  // [groups][128][2] f32
-  static constexpr int kBarOff = kPartOff + kTcGroups * 128 * 2 * 4;
+  static constexpr int kStages = 3;                  // K tiles in flight
+  static constexpr int kBarOff = kKOff + kStages * kHalves * kKBox;
+  // [groups][128][2] f32 of the final combine, over the K stages (all MMAs
+  // have completed by then)
+  static constexpr int kPartOff = kKOff;
   static constexpr int kBytes = kBarOff + 16 * 8 + 1024;  // + alignment slack
 };
 
@@ -107,25 +112,30 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   using L = Tc1Layout<D>;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = align1024(smem_raw);
+  constexpr int KS = L::kStages;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::kBarOff);
   uint64_t* q_full = bars;
-  uint64_t* k_full = bars + 1;     // [2]
-  uint64_t* k_empty = bars + 3;    // [2]
-  uint64_t* acc_full = bars + 5;   // [2]
-  uint64_t* acc_empty = bars + 7;  // [2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 9);
+  uint64_t* k_full = bars + 1;          // [KS]
+  uint64_t* k_empty = k_full + KS;      // [KS]
+  uint64_t* acc_full = k_empty + KS;    // [2]
+  uint64_t* acc_empty = acc_full + 2;   // [2]
+  uint64_t* mma_done = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int unit = blockIdx.x / a.mtiles, mt = blockIdx.x - unit * a.mtiles;
   const int nk = (a.n_ctx + kTcKeys1 - 1) / kTcKeys1;
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < KS; ++s) {
       mbar_init(&k_full[s], 1);
       mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
       mbar_init(&acc_full[s], 1);
       mbar_init(&acc_empty[s], kTcEpi);
     }
+    mbar_init(mma_done, 1);
     fence_barrier_init();
   }
   if (warp == kTcIssueWarp) {
@@ -149,28 +159,27 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int h = 0; h < L::kHalves; ++h)
         tma_load_2d(smem + h * L::kQBox, &tmQ, h * 64, unit * a.n_obs + mt * kTcRows1, q_full);
       auto load_k = [&](int j) {
-        const int s = j & 1;
+        const int s = j % KS;
         mbar_arrive_expect_tx(&k_full[s], L::kHalves * L::kKBox);
 #pragma unroll
         for (int h = 0; h < L::kHalves; ++h)
           tma_load_2d(smem + L::kKOff + (s * L::kHalves + h) * L::kKBox, &tmK, h * 64,
                       krow0 + j * kTcKeys1, &k_full[s]);
       };
-      load_k(0);
-      ok = mbar_wait_bounded(q_full, 0);
+      int issued = 0, consumed = 0;
+      for (; issued < nk && issued < KS; ++issued) load_k(issued);
+      const bool q_ok = mbar_wait_bounded(q_full, 0);
+      ok = q_ok;
       const uint32_t idesc = umma_idesc_bf16_f32(128, kTcKeys1);
       const uint32_t qbase = smem_u32(smem);
       for (int j = 0; ok && j < nk; ++j) {
-        const int s = j & 1;
-        if (j + 1 < nk) {  // next key tile into the other stage once its MMAs are done
-          if (j >= 1 && !mbar_wait_bounded(&k_empty[s ^ 1], ((j - 1) >> 1) & 1)) {
-            ok = false;
-            break;
-          }
-          load_k(j + 1);
+        const int s = j % KS, b = j & 1;  // K stage, accumulator
+        if (!mbar_wait_bounded(&k_full[s], (j / KS) & 1)) {
+          ok = false;
+          break;
         }
-        if (!mbar_wait_bounded(&k_full[s], (j >> 1) & 1) ||
-            (j >= 2 && !mbar_wait_bounded(&acc_empty[s], ((j - 2) >> 1) & 1))) {
+        ++consumed;
+        if (j >= 2 && !mbar_wait_bounded(&acc_empty[b], ((j - 2) >> 1) & 1)) {
           ok = false;
           break;
         }
@@ -181,11 +190,25 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           const uint32_t off = (uint32_t)((kk & 3) * 32);
           const uint64_t ad = umma_desc_k_sw128(qbase + (kk >> 2) * L::kQBox + off);
           const uint64_t bd = umma_desc_k_sw128(kbase + (kk >> 2) * L::kKBox + off);
-          umma_bf16(tmem + s * kTcKeys1, ad, bd, idesc, kk > 0);
+          umma_bf16(tmem + b * kTcKeys1, ad, bd, idesc, kk > 0);
         }
         umma_commit(&k_empty[s]);
-        umma_commit(&acc_full[s]);
+        umma_commit(&acc_full[b]);
+        // the stage of tile j - 1 takes tile j - 1 + KS once its MMAs are done
+        // (MMA j is queued behind them meanwhile)
+        if (j >= 1 && issued < nk) {
+          if (!mbar_wait_bounded(&k_empty[(j - 1) % KS], ((j - 1) / KS) & 1)) {
+            ok = false;
+            break;
+          }
+          load_k(issued++);
+        }
       }
+      // unwind: copies still in flight, then every MMA issued
+      if (!q_ok) mbar_wait_bounded(q_full, 0);
+      for (int t = consumed; t < issued; ++t) mbar_wait_bounded(&k_full[t % KS], (t / KS) & 1);
+      umma_commit(mma_done);
+      mbar_wait_bounded(mma_done, 0);
     }
     __syncwarp();
   } else {
@@ -200,27 +223,31 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
       tc_fence_after();
       const int kvalid = a.n_ctx - j * kTcKeys1;  // keys of this tile inside the unit
-#pragma unroll 1
-      for (int c = grp; c < kTcKeys1 / 32 && c * 32 < kvalid; c += kTcGroups) {
-        uint32_t r[32];
-        tmem_ld32(tmem + lane_base + b * kTcKeys1 + c * 32, r);
+      // this warp's two 32-key chunks (grp and grp + 4) loaded together, one
+      // wait, one running-max update and one pass of exponentials over 64 keys
+      const int nv0 = kvalid - grp * 32, nv1 = nv0 - 4 * 32;
+      if (nv0 > 0) {
+        uint32_t r[64];
+        tmem_ld32(tmem + lane_base + b * kTcKeys1 + grp * 32,
+                  *reinterpret_cast<uint32_t(*)[32]>(r));
+        tmem_ld32(tmem + lane_base + b * kTcKeys1 + (grp + 4) * 32,
+                  *reinterpret_cast<uint32_t(*)[32]>(r + 32));
         tmem_ld_wait();
-        float x[32];
-        const int nv = kvalid - c * 32;
-        if (nv >= 32) {
+        if (nv0 < 32 || nv1 < 32) {  // the unit's last keys: the rest belongs to the next unit
 #pragma unroll
-          for (int i = 0; i < 32; ++i) x[i] = __uint_as_float(r[i]);
-        } else {  // the unit's last keys: the rest of the chunk is another unit's
-#pragma unroll
-          for (int i = 0; i < 32; ++i) x[i] = i < nv ? __uint_as_float(r[i]) : -INFINITY;
+          for (int i = 0; i < 64; ++i) {
+            const bool in = i < 32 ? i < nv0 : i - 32 < nv1;
+            if (!in) r[i] = __float_as_uint(-INFINITY);
+          }
         }
-        float m4[4] = {x[0], x[1], x[2], x[3]};
+        float m4[4] = {__uint_as_float(r[0]), __uint_as_float(r[1]), __uint_as_float(r[2]),
+                       __uint_as_float(r[3])};
 #pragma unroll
-        for (int i = 4; i < 32; i += 8) {
-          m4[0] = fmax3(m4[0], x[i], x[i + 1]);
-          m4[1] = fmax3(m4[1], x[i + 2], x[i + 3]);
-          m4[2] = fmax3(m4[2], x[i + 4], x[i + 5]);
-          m4[3] = fmax3(m4[3], x[i + 6], x[i + 7]);
+        for (int i = 4; i < 64; i += 8) {
+          m4[0] = fmax3(m4[0], __uint_as_float(r[i]), __uint_as_float(r[i + 1]));
+          m4[1] = fmax3(m4[1], __uint_as_float(r[i + 2]), __uint_as_float(r[i + 3]));
+          m4[2] = fmax3(m4[2], __uint_as_float(r[i + 4]), __uint_as_float(r[i + 5]));
+          m4[3] = fmax3(m4[3], __uint_as_float(r[i + 6]), __uint_as_float(r[i + 7]));
         }
         const float cm = fmaxf(fmax3(m4[0], m4[1], m4[2]), m4[3]);
         if (cm > m) {
@@ -231,9 +258,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const float2 sc2 = make_float2(sc, sc), nmc = make_float2(-m * sc, -m * sc);
         float2 s2a = make_float2(0.f, 0.f), s2b = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int i = 0; i < 32; i += 4) {
-          const float2 ea = __ffma2_rn(make_float2(x[i], x[i + 1]), sc2, nmc);
-          const float2 eb = __ffma2_rn(make_float2(x[i + 2], x[i + 3]), sc2, nmc);
+        for (int i = 0; i < 64; i += 4) {
+          const float2 ea = __ffma2_rn(make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])),
+                                       sc2, nmc);
+          const float2 eb = __ffma2_rn(
+              make_float2(__uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])), sc2, nmc);
           s2a = __fadd2_rn(s2a, make_float2(exp2f(ea.x), exp2f(ea.y)));
           s2b = __fadd2_rn(s2b, make_float2(exp2f(eb.x), exp2f(eb.y)));
         }
