@@ -407,21 +407,31 @@ def e2e_run(path: Path, steps: int, in_place: bool, n_kept_layers=None):
     inside the timed region.
 
     in_place=False: K, V, Q and the scores (or the observation queries) are
-    copied to the device first.  in_place=True (workloads with given scores):
-    only Q is copied; ebd_evict reads K, V and the scores where they are, in
-    host memory, so the select reads every score and the gather only the kept
-    rows over the host link.  Returns (ms per step, H2D bytes, D2H bytes), the
-    H2D bytes being what crosses the link: the copies, plus for in_place the
-    scores and the kept K/V rows the kernels read."""
+    copied to the device first.  in_place=True: what the kernels read in full
+    is copied (Q; with attention scoring also K and the observation queries,
+    since scoring reads every key), the rest stays in host memory where
+    ebd_evict reads it (the select reads every score, the gather only the
+    kept rows).  Returns (ms per step, H2D bytes, D2H bytes), the H2D bytes
+    being what crosses the link: the copies, plus for in_place the scores and
+    the kept rows the kernels read in place."""
     ebd, w, dev = path.ebd, path.w, path.dev
     keys = ["K", "V", "Q"] + (["q_obs"] if path.scored else ["scores"])
     host_in = [{k: inp[k].cpu().pin_memory() for k in keys} for inp in path.inputs]
     host_out = [{k: v.cpu().pin_memory() for k, v in o.items()} for o in path.out]
-    copied = ["Q"] if in_place else keys
+    if not in_place:
+        copied = keys
+    elif path.scored:
+        copied = ["K", "Q", "q_obs"]   # V stays on the host: only its kept rows move
+    else:
+        copied = ["Q"]                 # K, V and the scores stay on the host
     h2d = sum(hi[k].numel() * hi[k].element_size() for hi in host_in for k in copied)
     if in_place:
-        h2d += sum(hi["scores"].numel() * 4 for hi in host_in)
-        h2d += sum(int(nk.sum()) * 2 * w.head_dim * w.elem_bytes for nk in n_kept_layers)
+        rows = sum(int(nk.sum()) for nk in n_kept_layers)
+        if path.scored:
+            h2d += rows * w.head_dim * w.elem_bytes            # kept V rows
+        else:
+            h2d += sum(hi["scores"].numel() * 4 for hi in host_in)
+            h2d += rows * 2 * w.head_dim * w.elem_bytes        # kept K and V rows
     d2h = sum(t.numel() * t.element_size() for ho in host_out for t in ho.values())
     ev_ws = None
     if path.scored:
@@ -433,10 +443,11 @@ def e2e_run(path: Path, steps: int, in_place: bool, n_kept_layers=None):
             inp, hi = path.inputs[l], host_in[l]
             for k in copied:
                 inp[k].copy_(hi[k], non_blocking=True)
-            src = hi if in_place else inp
+            def src(k):
+                return inp[k] if k in copied else hi[k]
             cc, o = path.cc[l], path.out[l]
-            ebd.ebd_evict(path.designs[l], src["K"], src["V"],
-                          None if path.scored else src["scores"],
+            ebd.ebd_evict(path.designs[l], src("K"), src("V"),
+                          None if path.scored else src("scores"),
                           inp["q_obs"] if path.scored else None, cc, workspace=ev_ws)
             ebd.ebd_certified_decode(inp["Q"], cc.K_c, cc.V_c, cc.logw_c, cc.n_kept, o["y"],
                                      o["lse"], o["var"], o["b"], o["r"], workspace=path.dec_ws)
@@ -626,11 +637,14 @@ def run_ours(args, world, rank, local):
             return {"value": whole_job_rate(dbytes, world, ms * 1e-3) / 1e9, "unit": "GB/s",
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms}
         e2e_copy = e2e_line(False)
-        e2e_copy["inputs"] = "K, V, Q and the scores copied to the device each step"
+        e2e_copy["inputs"] = ("K, V, Q and the " + ("observation queries" if path.scored else
+                              "scores") + " copied to the device each step")
+        e2e = e2e_line(True)
         if path.scored:
-            e2e = e2e_copy  # scoring reads every key: the cache goes to the device
+            e2e["inputs"] = ("K, Q and the observation queries copied (scoring reads every key); "
+                             "V read in place from page-locked host memory (the gather reads "
+                             "only the kept rows)")
         else:
-            e2e = e2e_line(True)
             e2e["inputs"] = ("K, V and the scores read in place from page-locked host memory "
                              "(the select reads every score, the gather only the kept rows); "
                              "Q copied")

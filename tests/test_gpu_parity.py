@@ -274,6 +274,32 @@ def test_evict_from_page_locked_host_memory_matches_device(E):
     assert st == 1  # EBD_ERR_INVALID
 
 
+def test_scored_eviction_with_host_resident_values_matches_device(E):
+    """Attention scoring reads every key, so K and the observation queries
+    stay in device memory, but V may be page-locked host memory (only the kept
+    rows are read); the outputs equal the all-device call.  A host-resident K
+    is refused on this path."""
+    B, H, G, N, d, R, cap = 2, 2, 4, 2048, 128, 256, 576
+    g = torch.Generator().manual_seed(8)
+    K = torch.randn((B, H, N, d), generator=g).to(torch.bfloat16)
+    V = torch.randn((B, H, N, d), generator=g).to(torch.bfloat16)
+    q = torch.randn((B, H, R, d), generator=g).to(torch.bfloat16)
+    des = _design(E, B, H, G, d, N, 0, 3, N // 50, N // 5)
+    ref = E.alloc_compact(B, H, cap, d, torch.bfloat16, DEV)
+    E.ebd_evict(des, K.to(DEV), V.to(DEV), None, q.to(DEV), ref)
+    out = E.alloc_compact(B, H, cap, d, torch.bfloat16, DEV)
+    E.ebd_evict(des, K.to(DEV), V.pin_memory(), None, q.to(DEV), out)
+    torch.cuda.synchronize()
+    assert out.dev_status.item() == 0 and torch.equal(out.n_kept, ref.n_kept)
+    for b in range(B):
+        for h in range(H):
+            n = min(int(ref.n_kept[b, h]), cap)
+            for f in ("idx_c", "logw_c", "K_c", "V_c"):
+                assert torch.equal(getattr(out, f)[b, h, :n], getattr(ref, f)[b, h, :n]), f
+    with pytest.raises(ValueError):
+        E.ebd_evict(des, K.pin_memory(), V.pin_memory(), None, q.to(DEV), out)
+
+
 def test_evict_capacity_overflow_is_flagged_and_bounded(E):
     B, H, N, d = 1, 2, 2000, 64
     cap = 64  # far below the ~400 kept tokens
