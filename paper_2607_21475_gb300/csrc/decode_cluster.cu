@@ -117,6 +117,10 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
   float* lw_s = reinterpret_cast<float*>(smem + a.lw_off);
   float* lead = reinterpret_cast<float*>(smem + a.lead_off);
 
+  // launched as a programmatic dependent: wait for the predecessor's outputs
+  // before the first read; let a following dependent launch early
+  grid_dependency_wait();
+  grid_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int C = a.csize, G = a.group;
   const uint32_t rank = cluster_rank();
@@ -258,13 +262,15 @@ static ebd_status launch_cluster_t(const DecodeArgs& d, const ReduceArgs& r, int
   cfg.blockDim = dim3(kMmaThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = (unsigned)C;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cuda_status(cudaLaunchKernelEx(&cfg, decode_cluster_kernel<D, S>, a));
 }
 

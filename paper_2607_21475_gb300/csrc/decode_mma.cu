@@ -15,7 +15,9 @@
 // The merge kernel (one CTA per query head, launched as a programmatic
 // dependent of the decode so its launch overlaps the decode's tail) spreads
 // the head's records over its warps, combines them in shared memory and
-// writes y_hat, lse, V_hat, b_t and r_t.
+// writes y_hat, lse, V_hat, b_t and r_t.  The decode kernel is itself launched
+// as a programmatic dependent of whatever precedes it (a previous layer's
+// merge, say), waiting before its first memory access.
 //
 // The per-tile step (Q K^T, weights, [w; u] V on mma.sync with hi/lo weight
 // parts, ||v||^2, lazy rescale) lives in decode_tile.cuh.
@@ -84,15 +86,6 @@ struct MergeArgs {
   float eps0;
   bool exact;                // b_t / radius come from the exact range pass
 };
-
-// Programmatic dependent launch: the decode lets the merge grid launch early;
-// the merge waits for the whole decode grid (and its memory) before reading.
-__device__ __forceinline__ void grid_launch_dependents() {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-__device__ __forceinline__ void grid_dependency_wait() {
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-}
 
 // Working warps of a decode over Ta active tiles (each gets >= kMinTilesPerWarp).
 __host__ __device__ __forceinline__ long long decode_working_warps(long long Ta, long long Wall) {
@@ -201,6 +194,10 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
       (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);  // swizzle atoms
   float* lw_s = reinterpret_cast<float*>(smem + L::kLogwOff);
 
+  // launched as a programmatic dependent: the previous kernel's outputs
+  // (the compact cache, Q) are visible after this wait; nothing is read or
+  // written before it
+  grid_dependency_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int units = a.units;
   const int32_t* toff = a.tile_off;
@@ -301,6 +298,7 @@ __global__ void __launch_bounds__(MW * 32) decode_merge_kernel(MergeArgs a) {
   __shared__ __align__(16) float sh_o[MW][D];
   __shared__ __align__(16) float sh_a[MW][D];
   grid_dependency_wait();
+  grid_launch_dependents();  // a following dependent grid may launch now
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = a.group;
@@ -515,9 +513,22 @@ static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, con
   if (cudaFuncSetAttribute(decode_mma_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            smem) != cudaSuccess)
     return EBD_ERR_CUDA;
-  decode_mma_kernel<D><<<plan.ctas, kMmaThreads, smem, s>>>(f);
-  ebd_status st = launch_status();
-  if (st != EBD_OK) return st;
+  {
+    // programmatic dependent of whatever precedes it in the stream: its launch
+    // overlaps that kernel's tail (the kernel waits before touching memory)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)plan.ctas);
+    cfg.blockDim = dim3(kMmaThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const ebd_status st = cuda_status(cudaLaunchKernelEx(&cfg, decode_mma_kernel<D>, f));
+    if (st != EBD_OK) return st;
+  }
 
   MergeArgs m;
   m.tile_off = tile_off;

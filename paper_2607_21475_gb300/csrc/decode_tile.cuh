@@ -35,6 +35,17 @@ constexpr int kMmaConsumers = 8;  // warps per CTA
 constexpr int kMmaThreads = kMmaConsumers * 32;
 constexpr float kRescaleLog2 = 8.f;
 
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialization may start while its predecessor in the stream runs; it must
+// wait before reading the predecessor's outputs or writing anything.  A
+// kernel lets its own dependents launch early with launch_dependents.
+__device__ __forceinline__ void grid_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 template <int D>
 struct MmaTileLayout {
   static constexpr int kHalves = D / 64;             // 64-column (128-byte) boxes per row

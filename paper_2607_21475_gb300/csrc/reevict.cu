@@ -23,6 +23,9 @@ __global__ void __launch_bounds__(kAppendWarps * 32)
                   int cap, uint4* __restrict__ K_c, uint4* __restrict__ V_c,
                   float* __restrict__ logw_c, int32_t* __restrict__ idx_c,
                   int32_t* __restrict__ n_kept, int32_t* dev_status) {
+  // a decode launched next as a programmatic dependent may start its launch
+  // now; it waits for this kernel's writes before reading the cache
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int unit = blockIdx.x * kAppendWarps + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (unit >= units) return;
