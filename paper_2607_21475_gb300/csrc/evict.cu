@@ -4,19 +4,26 @@
 //   E1  certainty set A: protected positions (sinks, recency window) plus the
 //       top-k_head unprotected tokens by score, equal scores to the lower index
 //       (Section 3.3 and Appendix B of the paper).  Exact selection by an
-//       MSB-first 8-bit radix select over order-preserving score keys, then an
-//       ordered scan among the tokens equal to the k-th key.
+//       MSB-first 8-bit radix select over order-preserving score keys; an
+//       ordered scan among the tokens equal to the k-th key only when fewer of
+//       them are needed than there are.
 //   E2  inclusion probabilities on the tail T (Eq. 2): pi_i = clip(c s_i, eps, 1)
-//       with c solving sum_T pi_i = m (clip-saturated tokens join A), found by
-//       a fixed number of bisection steps on log c, then one exact linear solve
-//       inside the partition (clipped-high / linear / floor) the bisection ends in.
-//   E3  Poisson draw: keep_i = (u_i < pi_i) with u_i from Philox4x32-10 keyed by
-//       the seed, counter (token, kvh, layer, b).
+//       with c solving sum_T pi_i = m (clip-saturated tokens join A): bisection
+//       on log c whose steps take the exact linear solve of the current
+//       partition (clipped-high / linear / floor) when it lands in the bracket,
+//       stopping once the partition reproduces its own solve.
+//   E3  Poisson draw: keep_i = (u_i < pi_i), u_i from word i % 4 of Philox4x32-10
+//       keyed by the seed at counter (i / 4, kvh, layer, b); or the systematic
+//       design at the same pi (one uniform per unit, fixed-point cumulative sums).
 //   E4  stable compaction: an ordered block scan of the keep flags writes the
 //       token index and log(1/pi_i) of every kept token; a second, HBM-bound
 //       kernel then copies the kept K and V rows with 16-byte loads.
-// The certainty set lives in shared memory as a bitmask (N/8 bytes).  Scores
-// are re-read from global memory (L2-resident) by each pass.
+// Two select kernels: up to 32768 tokens the unit's scores sit in shared
+// memory (one float4 per thread per 4096-token group); beyond, they stay in
+// global memory (L2-resident while the unit is worked on) and every pass reads
+// them in 4096-token steps.  ebd_evict pipelines chunks of one SM count of
+// units over streams so that the copy of one select wave overlaps the next.
+// K, V and the scores may be page-locked host memory (read over the host link).
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
@@ -54,83 +61,6 @@ struct SelectArgs {
   int systematic;       // tail design: 0 Poisson, 1 systematic at the same pi
   int unit0;            // first unit of this launch (CTA x handles unit unit0 + x)
 };
-
-struct BlockScratch {
-  float f[kSelWarps];
-  double d[kSelWarps];
-  int i[kSelWarps];
-};
-
-__device__ __forceinline__ float block_sum_f2d(float v, BlockScratch& sh) {
-  // per-thread float partials, combined across the block in double
-  v = warp_sum(v);
-  __syncthreads();
-  if ((threadIdx.x & 31) == 0) sh.d[threadIdx.x >> 5] = (double)v;
-  __syncthreads();
-  double r = 0.0;
-#pragma unroll 8
-  for (int w = 0; w < kSelWarps; ++w) r += sh.d[w];
-  return (float)r;
-}
-__device__ __forceinline__ double block_sum_d(double v, BlockScratch& sh) {
-  v = warp_sum(v);
-  __syncthreads();
-  if ((threadIdx.x & 31) == 0) sh.d[threadIdx.x >> 5] = v;
-  __syncthreads();
-  double r = 0.0;
-#pragma unroll 8
-  for (int w = 0; w < kSelWarps; ++w) r += sh.d[w];
-  return r;
-}
-__device__ __forceinline__ int block_sum_i(int v, BlockScratch& sh) {
-  v = warp_sum(v);
-  __syncthreads();
-  if ((threadIdx.x & 31) == 0) sh.i[threadIdx.x >> 5] = v;
-  __syncthreads();
-  int r = 0;
-#pragma unroll 8
-  for (int w = 0; w < kSelWarps; ++w) r += sh.i[w];
-  return r;
-}
-__device__ __forceinline__ float block_max_f(float v, BlockScratch& sh) {
-  v = warp_max(v);
-  __syncthreads();
-  if ((threadIdx.x & 31) == 0) sh.f[threadIdx.x >> 5] = v;
-  __syncthreads();
-  float r = sh.f[0];
-#pragma unroll 8
-  for (int w = 1; w < kSelWarps; ++w) r = fmaxf(r, sh.f[w]);
-  return r;
-}
-__device__ __forceinline__ float block_min_f(float v, BlockScratch& sh) {
-  v = warp_min(v);
-  __syncthreads();
-  if ((threadIdx.x & 31) == 0) sh.f[threadIdx.x >> 5] = v;
-  __syncthreads();
-  float r = sh.f[0];
-#pragma unroll 8
-  for (int w = 1; w < kSelWarps; ++w) r = fminf(r, sh.f[w]);
-  return r;
-}
-
-// Ordered count: exclusive prefix of `flag` over the block in thread order and
-// the block total.  Two barriers.
-__device__ __forceinline__ int block_rank(bool flag, int& total, BlockScratch& sh) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const unsigned bal = __ballot_sync(0xffffffffu, flag);
-  __syncthreads();
-  if (lane == 0) sh.i[warp] = __popc(bal);
-  __syncthreads();
-  int before = 0, tot = 0;
-#pragma unroll 8
-  for (int w = 0; w < kSelWarps; ++w) {
-    const int c = sh.i[w];
-    before += (w < warp) ? c : 0;
-    tot += c;
-  }
-  total = tot;
-  return before + __popc(bal & ((1u << lane) - 1u));
-}
 
 enum PiMode : int { kPiFloor = 0, kPiAll = 1, kPiLinear = 2 };
 
