@@ -66,6 +66,10 @@ def parse_args():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
+    p.add_argument("--no-all-cores", action="store_true",
+                   help="skip the oracle timing on every host core")
+    p.add_argument("--all-core-units", type=int, default=64,
+                   help="units of layer 0 in the all-core oracle sample")
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--batch", type=int, default=0,
                    help="override the workload's batch (smaller cases for profiling)")
@@ -504,6 +508,90 @@ def oracle_sample(w: Workload, inputs, seconds: float, max_units=None):
     return units, t_ev, t_dec, dbytes
 
 
+def _to_f64(a):
+    """float32 numpy, or bfloat16 bit patterns as int16 numpy -> float64."""
+    if a.dtype == np.int16:
+        return (a.astype(np.int32).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    return a.astype(np.float64)
+
+
+def _host_array(t):
+    """A tensor's values for a pool worker: bf16 as its int16 bit patterns."""
+    t = t.contiguous()
+    return (t.view(torch.int16) if t.dtype == torch.bfloat16 else t.float()).cpu().numpy()
+
+
+def _oracle_evict_task(task):
+    """Pool worker: eviction of one unit (E0 first for attention scores); its
+    own compute time only (the unpacking of the inputs is not timed)."""
+    from oracle import ebd_oracle as O
+    p, u, K16, V16, s, qo16 = task
+    K, V = _to_f64(K16), _to_f64(V16)
+    b, h = divmod(u, p["H"])
+    t = time.perf_counter()
+    if s is None:
+        s = O.accumulated_attention_scores(_to_f64(qo16), K).astype(np.float32)
+    r = O.evict_unit(K, V, s, n_sink=p["n_sink"], n_recent=p["n_recent"], k_head=p["k_head"],
+                     budget_tokens=p["budget"], eps=p["eps"], seed=p["seed"], layer=0, b=b,
+                     kvh=h, capacity=p["cap"])
+    dt = time.perf_counter() - t
+    return os.getpid(), dt, r.idx, r.logw
+
+
+def _oracle_decode_task(task):
+    """Pool worker: certified decode of one unit over its kept rows."""
+    from oracle import ebd_oracle as O
+    Q16, Kc16, Vc16, logw = task
+    Q, Kc, Vc = _to_f64(Q16), _to_f64(Kc16), _to_f64(Vc16)
+    t = time.perf_counter()
+    O.hajek_decode(Q, Kc, Vc, logw)
+    return os.getpid(), time.perf_counter() - t
+
+
+def oracle_all_cores(w: Workload, inputs, max_units: int, processes=None):
+    """The float64 oracle on every host core: a spawn-started process pool runs
+    the eviction of a sample of units, then their decode; each phase's time is
+    the largest per-process sum of task compute times (start-up and the
+    transfer of inputs not counted)."""
+    import multiprocessing as mp
+    B, H, G, d = w.batch, w.n_kv_heads, w.group, w.head_dim
+    cores = processes or (len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity")
+                          else os.cpu_count())
+    U = min(B * H, max_units)
+    p = {"H": H, "n_sink": w.n_sink, "n_recent": w.n_recent, "k_head": w.k_head,
+         "budget": w.budget_tokens, "eps": w.eps, "seed": w.philox_seed, "cap": w.capacity}
+
+    i16 = _host_array
+    ev_tasks = []
+    for u in range(U):
+        b, h = divmod(u, H)
+        s = inputs["scores"][b, h].cpu().numpy() if "scores" in inputs else None
+        qo = i16(inputs["q_obs"][b, h]) if s is None else None
+        ev_tasks.append((p, u, i16(inputs["K"][b, h]), i16(inputs["V"][b, h]), s, qo))
+    with mp.get_context("spawn").Pool(cores) as pool:
+        pool.map(_to_f64, [np.zeros(1, np.int16)] * cores)  # start every worker
+        res = pool.map(_oracle_evict_task, ev_tasks, chunksize=1)
+        t_ev = {}
+        for pid, dt, _, _ in res:
+            t_ev[pid] = t_ev.get(pid, 0.0) + dt
+        dec_tasks, dbytes = [], 0
+        for u, (_, _, idx, logw) in enumerate(res):
+            b, h = divmod(u, H)
+            dec_tasks.append((i16(inputs["Q"][b, h * G:(h + 1) * G]), ev_tasks[u][2][idx],
+                              ev_tasks[u][3][idx], logw))
+            n = min(len(idx), w.capacity)
+            dbytes += n * (2 * d * w.elem_bytes + 4) + G * d * w.elem_bytes + G * (d + 4) * 4
+        t_dec = {}
+        for pid, dt in pool.map(_oracle_decode_task, dec_tasks, chunksize=1):
+            t_dec[pid] = t_dec.get(pid, 0.0) + dt
+    wall_ev, wall_dec = max(t_ev.values()), max(t_dec.values())
+    return {"value": dbytes / wall_dec / 1e9, "unit": "GB/s", "cores": cores, "kind": "oracle",
+            "evict_mtok_s": U * w.n_ctx / wall_ev / 1e6,
+            "sample": f"{U} of {B * H} (batch row, kv head) units of layer 0 on {cores} "
+                      f"processes: eviction {wall_ev:.2f} s, decode {wall_dec:.3f} s "
+                      f"(largest per-process compute time)"}
+
+
 def config_of(w: Workload):
     return {"workload": w.name, "layers": w.n_layers, "batch": w.batch, "n_ctx": w.n_ctx,
             "q_heads": w.n_q_heads, "kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
@@ -656,6 +744,11 @@ def run_ours(args, world, rank, local):
                "sample": f"{u} of {w.batch * w.n_kv_heads} (batch row, kv head) units of "
                          f"layer 0: eviction + certified decode ({t_ev + t_dec:.1f} s)",
                "evict_mtok_s": u * w.n_ctx / t_ev / 1e6}
+        if not args.no_all_cores:
+            try:
+                cpu["all_cores"] = oracle_all_cores(w, path.inputs[0], args.all_core_units)
+            except Exception as e:  # a host without spawn or enough memory: say so
+                cpu["all_cores"] = {"unavailable": f"{type(e).__name__}: {e}"[:200]}
 
     launches = args.steps * sum(path.launches[p] * L for p in path.phases)
     line = {
