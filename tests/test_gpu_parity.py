@@ -375,7 +375,8 @@ def _synthetic_cache(B, H, cap, d, dtype, pattern, seed):
     elif pattern == "full":
         n = torch.full((units,), cap)
     else:
-        base = [0, 1, cap, cap - 1, 63, 65, cap // 2 + 3]
+        # an overflowed unit (n_kept > cap: the decode reads the cap rows it has)
+        base = [0, 1, cap, cap - 1, 63, 65, cap // 2 + 3, cap + 5]
         n = torch.tensor([base[i % len(base)] for i in range(units)])
     return Kc, Vc, logw, n.view(B, H).int()
 
