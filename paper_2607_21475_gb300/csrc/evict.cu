@@ -25,6 +25,7 @@
 // units over streams so that the copy of one select wave overlaps the next.
 // K, V and the scores may be page-locked host memory (read over the host link).
 #include <cuda_runtime.h>
+#include <float.h>
 #include <math.h>
 #include <stdint.h>
 
@@ -64,11 +65,39 @@ struct SelectArgs {
 
 enum PiMode : int { kPiFloor = 0, kPiAll = 1, kPiLinear = 2 };
 
-
-__device__ __forceinline__ float tail_pi(float s, int mode, float c, float eps) {
-  if (mode == kPiFloor) return eps;
-  if (mode == kPiAll) return s > 0.f ? 1.f : eps;
+// pi of a tail token, Eq. (2): min(1, max(eps, c s)).  The two saturated
+// regimes are the same formula at an extreme c: a budget at or below the
+// floor (every tail token at eps) is c = 0, and a budget that covers every
+// positive score (those at 1, the rest at eps) is c = FLT_MAX, for which
+// c s >= 1 at every normal s > 0.
+__device__ __forceinline__ float tail_pi(float s, float c, float eps) {
   return fminf(1.f, fmaxf(eps, c * s));
+}
+
+__device__ __forceinline__ float saturated_c(int mode) { return mode == kPiAll ? FLT_MAX : 0.f; }
+
+// One water-filling step of Eq. (2), taken by one thread.  Given the partition
+// at the current scale c (nh tail tokens clipped at 1, nl at eps, the others
+// summing to smid), narrow the bisection bracket [lo, hi] on log c and return
+// the next c: the exact linear solve of this partition when it lies inside the
+// bracket, else the bracket's midpoint.  `stop` is set once the partition
+// reproduces its own solve (or the step no longer moves c).  float32
+// throughout: the sums it takes are float32 partial sums, and on this GPU the
+// fp64 pipe would make this serial step the longest part of an iteration.
+__device__ __forceinline__ float water_fill_step(int m, int nh, int nl, float smid, float eps,
+                                                 float c, float& lo, float& hi, int& stop) {
+  const float gval = (float)nh + eps * (float)nl + c * smid;
+  if (gval < (float)m) lo = fmaxf(lo, logf(c));
+  else hi = fminf(hi, logf(c));
+  const float clin = smid > 0.f ? ((float)(m - nh) - eps * (float)nl) / smid : -1.f;
+  if (clin > 0.f && fabsf(clin - c) <= 1e-6f * c) {
+    stop = 1;  // the partition at c reproduces its own solve
+    return clin;
+  }
+  const float lcl = clin > 0.f ? logf(clin) : -INFINITY;
+  const float next = (clin > 0.f && lcl > lo && lcl < hi) ? clin : expf(0.5f * (lo + hi));
+  if (next == c) stop = 1;
+  return next;
 }
 
 // ---------------------------------------------------------------------------
@@ -92,11 +121,8 @@ struct BigScratch {
   int tot[kSelWarps];
   float rf[3][kSelWarps];
   int ri[2][kSelWarps];
-  double res_d;
-  float res_f[2];
-  int res_i[2];
   float c, lo, hi;  // solve state, updated by thread 0 only
-  int mode, stop;
+  int stop;
   unsigned prefix, remaining, eqcount;
 };
 
@@ -357,7 +383,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
     __syncthreads();
     if (warp == 0) {
       float mx = sh.rf[0][lane], mn = sh.rf[1][lane];
-      double sd = (double)sh.rf[2][lane];
+      float sd = sh.rf[2][lane];
       int np = sh.ri[0][lane];
       mx = warp_max(mx);
       mn = warp_min(mn);
@@ -368,20 +394,18 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
         int md = kPiLinear;
         if (nT == 0 || (float)m <= eps * (float)nT) md = kPiFloor;
         else if ((float)m >= (float)np + eps * (float)(nT - np)) md = kPiAll;
-        sh.mode = md;
         sh.stop = md != kPiLinear;
         if (md == kPiLinear) {
           sh.lo = logf(eps / mx);
           sh.hi = logf(1.f / mn);
-          sh.c = fminf(fmaxf((float)((double)m / sd), expf(sh.lo)), expf(sh.hi));
+          sh.c = fminf(fmaxf((float)m / sd, expf(sh.lo)), expf(sh.hi));
         } else {
-          sh.c = 0.f;
+          sh.c = saturated_c(md);
         }
       }
     }
     __syncthreads();
   }
-  const int mode = sh.mode;
   float c = sh.c;
 #pragma unroll 1
   for (int it = 0; it < a.iters && !sh.stop; ++it) {
@@ -410,7 +434,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
     nhi = warp_sum(nhi);
     nlo = warp_sum(nlo);
     smid = warp_sum(smid);
-    __syncthreads();  // the previous iteration's readers of sh are done
+    // (the barrier closing the previous iteration ordered its reads of sh)
     if (lane == 0) {
       sh.ri[0][warp] = nhi;
       sh.ri[1][warp] = nlo;
@@ -418,28 +442,16 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
     }
     __syncthreads();
     if (warp == 0) {
-      double sd = (double)sh.rf[0][lane];
+      float sd = sh.rf[0][lane];
       int ah = sh.ri[0][lane], al = sh.ri[1][lane];
       sd = warp_sum(sd);
       ah = warp_sum(ah);
       al = warp_sum(al);
       if (lane == 0) {
-        const double gval = ah + (double)eps * al + (double)c * sd;
         float lo = sh.lo, hi = sh.hi;
-        if (gval < (double)m) lo = fmaxf(lo, logf(c));
-        else hi = fminf(hi, logf(c));
-        const double clin = sd > 0.0 ? ((double)m - ah - (double)eps * al) / sd : -1.0;
-        if (clin > 0.0 && fabs(clin - (double)c) <= 1e-6 * (double)c) {
-          sh.c = (float)clin;  // the partition at c reproduces its own solve
-          sh.stop = 1;
-        } else {
-          float next;
-          const float lcl = clin > 0.0 ? logf((float)clin) : -INFINITY;
-          if (clin > 0.0 && lcl > lo && lcl < hi) next = (float)clin;
-          else next = expf(0.5f * (lo + hi));
-          if (next == c) sh.stop = 1;
-          sh.c = next;
-        }
+        int stop = 0;
+        sh.c = water_fill_step(m, ah, al, sd, eps, c, lo, hi, stop);
+        sh.stop = stop;
         sh.lo = lo;
         sh.hi = hi;
       }
@@ -472,7 +484,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
         pis[r] = 1.f;
         if (i >= N) continue;
         const bool ct = (c4 >> r) & 1u;
-        const float pi = ct ? 1.f : tail_pi(v[q][r], mode, c, eps);
+        const float pi = ct ? 1.f : tail_pi(v[q][r], c, eps);
         pis[r] = pi;
         if (a.pi_out) a.pi_out[(size_t)unit * Nrow + i] = pi;
         if (a.mask_out) a.mask_out[(size_t)unit * Nrow + i] = ct ? 1 : 0;
@@ -506,8 +518,15 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
 // 1024 threads; thread t owns tokens g*4096 + 4t + r (g < JG, r < 4): the four
 // tokens that share one Philox call live in one thread, and its scores sit in
 // shared memory as one float4 per group (read once from HBM).  Membership is
-// a 64-bit mask per thread (bit 4g + r).  Loops over groups stay rolled so the
+// a 32-bit mask per thread (bit 4g + r).  Loops over groups stay rolled so the
 // kernel stays small in the instruction cache.
+// The top slice is an MSB-first radix select over 8-bit digits of the
+// order-preserving keys: the load builds the first digit's histogram, one
+// pass over every candidate settles the first digit (and builds the second
+// digit's histogram), and later passes touch only the tokens still in
+// contention.  A token leaves contention either into the top slice or into
+// the tail, and the tail statistics that Eq. (2) starts from are taken as it
+// leaves, so no separate pass gathers them.
 // The scale c of Eq. (2) is found by bisection on log c whose steps are
 // replaced by the exact linear solve inside the current partition whenever
 // that solve lands inside the bracket (water-filling); it stops once the
@@ -517,6 +536,9 @@ constexpr int kRegThreads = 1024;
 constexpr int kRegWarps = kRegThreads / 32;
 constexpr int kRegMaxGroups = 8;
 constexpr int kGroupTokens = 4 * kRegThreads;
+// Per-warp histograms sit 257 words apart, so that the lanes of the reduce,
+// which read one bin from four warps' histograms at once, hit distinct banks.
+constexpr int kHistStride = 257;
 
 struct RegScratch {
   long long ll[kRegWarps];  // systematic design: per-warp prefix totals
@@ -525,24 +547,21 @@ struct RegScratch {
   int off[kRegMaxGroups][kRegWarps];
   float rf[3][kRegWarps];
   int ri[2][kRegWarps];
-  double res_d;
-  float res_f[2];
+  float res_f[3];
   int res_i[2];
   float c, lo, hi;  // solve state, updated by thread 0 only
-  int mode, stop;
+  int stop;
   unsigned prefix, remaining, eqcount;
   int total;
 };
 
 // Cross-warp combine of per-warp partials written to sh.rf / sh.ri by lane 0
-// of every warp: warp 0 reduces the kRegWarps entries (the float sum in
-// double, so that only 32 lanes touch the slow fp64 pipe) and publishes
-// res_*.  Callers bracket it with barriers.
+// of every warp: warp 0 reduces the kRegWarps entries and publishes res_*.
+// Callers bracket it with barriers.
 __device__ __forceinline__ void combine_stats(RegScratch& sh) {
   const int lane = threadIdx.x & 31;
   if ((threadIdx.x >> 5) == 0) {
-    float mx = sh.rf[0][lane], mn = sh.rf[1][lane];
-    double sd = (double)sh.rf[2][lane];
+    float mx = sh.rf[0][lane], mn = sh.rf[1][lane], sd = sh.rf[2][lane];
     int n = sh.ri[0][lane];
     mx = warp_max(mx);
     mn = warp_min(mn);
@@ -551,7 +570,7 @@ __device__ __forceinline__ void combine_stats(RegScratch& sh) {
     if (lane == 0) {
       sh.res_f[0] = mx;
       sh.res_f[1] = mn;
-      sh.res_d = sd;
+      sh.res_f[2] = sd;
       sh.res_i[0] = n;
     }
   }
@@ -560,51 +579,69 @@ __device__ __forceinline__ void combine_stats(RegScratch& sh) {
 __device__ __forceinline__ void combine_partition(RegScratch& sh) {
   const int lane = threadIdx.x & 31;
   if ((threadIdx.x >> 5) == 0) {
-    double sd = (double)sh.rf[0][lane];
+    float sd = sh.rf[0][lane];
     int a = sh.ri[0][lane], b = sh.ri[1][lane];
     sd = warp_sum(sd);
     a = warp_sum(a);
     b = warp_sum(b);
     if (lane == 0) {
-      sh.res_d = sd;
+      sh.res_f[2] = sd;
       sh.res_i[0] = a;
       sh.res_i[1] = b;
     }
   }
 }
 
-// Exclusive prefix, over the lanes of this warp, of the number of set bits in
-// 4-bit group g of `flags`.
-__device__ __forceinline__ int lane_prefix(uint32_t flags, int g) {
-  const int lane = threadIdx.x & 31;
-  const int c = __popc((flags >> (4 * g)) & 0xFu);
-  int incl = c;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int n = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += n;
-  }
-  return incl - c;
+// Per-group counts of the set bits of `flags` (group g = bits 4g .. 4g + 3),
+// one byte per group: groups 0-3 in `lo`, groups 4-7 in `hi`.
+__device__ __forceinline__ void group_counts(uint32_t flags, uint32_t& lo, uint32_t& hi) {
+  uint32_t x = flags - ((flags >> 1) & 0x55555555u);
+  x = (x & 0x33333333u) + ((x >> 2) & 0x33333333u);  // each nibble holds its count
+  uint32_t l = x & 0xFFFFu, h = x >> 16;
+  l = (l | (l << 8)) & 0x00FF00FFu;
+  l = (l | (l << 4)) & 0x0F0F0F0Fu;
+  h = (h | (h << 8)) & 0x00FF00FFu;
+  h = (h | (h << 4)) & 0x0F0F0F0Fu;
+  lo = l;
+  hi = h;
+}
+
+__device__ __forceinline__ int group_byte(uint32_t lo, uint32_t hi, int g) {
+  return (int)(((g < 4 ? lo : hi) >> (8 * (g & 3))) & 0xFFu);
 }
 
 // Ordered count of the set bits of `flags` (bit 4g + r <-> token
-// g*4096 + 4*tid + r): afterwards sh.off[g][w] is the number of set bits at
-// tokens before warp w's slice of group g; returns the block total.  The rank
-// of a token is sh.off[g][warp] + lane_prefix(flags, g) + its rank in the thread.
-__device__ __forceinline__ int ordered_scan(uint32_t flags, int JG, RegScratch& sh) {
+// g*4096 + 4*tid + r).  One warp scan of the packed per-group counts (a warp's
+// count in one group is at most 128, so the bytes never carry) gives every
+// lane its exclusive prefix in all groups at once (`below_lo`, `below_hi`);
+// afterwards sh.off[g][w] is the number of set bits at tokens before warp w's
+// slice of group g.  Returns the block total.  The rank of a token is
+// sh.off[g][warp] + group_byte(below, g) + its rank within the thread's group.
+__device__ __forceinline__ int ordered_scan(uint32_t flags, int JG, RegScratch& sh,
+                                            uint32_t& below_lo, uint32_t& below_hi) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  __syncthreads();  // previous readers of sh.off / sh.total are done
-#pragma unroll 1
-  for (int g = 0; g < JG; ++g) {
-    const int c = __popc((flags >> (4 * g)) & 0xFu);
-    const int tot = warp_sum(c);
-    if (lane == 0) sh.tot[g][warp] = tot;
+  uint32_t lo, hi;
+  group_counts(flags, lo, hi);
+  uint32_t il = lo, ih = hi;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t nl = __shfl_up_sync(0xffffffffu, il, o);
+    const uint32_t nh = __shfl_up_sync(0xffffffffu, ih, o);
+    if (lane >= o) {
+      il += nl;
+      ih += nh;
+    }
   }
+  below_lo = il - lo;
+  below_hi = ih - hi;
+  const uint32_t tl = __shfl_sync(0xffffffffu, il, 31);
+  const uint32_t th = __shfl_sync(0xffffffffu, ih, 31);
+  __syncthreads();  // previous readers of sh.tot / sh.off / sh.total are done
+  if (lane < JG) sh.tot[lane][warp] = group_byte(tl, th, lane);
   __syncthreads();
   if (warp == 0) {
     const int E = JG * kRegWarps;               // <= 256
     const int PER = (E + 31) / 32;              // <= 8
-
     int local = 0;
 #pragma unroll 1
     for (int q = 0; q < PER; ++q) {
@@ -633,11 +670,65 @@ __device__ __forceinline__ int ordered_scan(uint32_t flags, int JG, RegScratch& 
   return sh.total;
 }
 
+// One radix-select step: the per-warp histograms of the current digit are
+// summed into sh.hist, then warp 0 finds, from
+// the top, the digit value holding the `remaining`-th largest key still in
+// contention and publishes it (sh.prefix), the rank left inside it
+// (sh.remaining) and its count (sh.eqcount).  Three barriers.
+__device__ __forceinline__ void choose_digit(const unsigned* whist, RegScratch& sh,
+                                             unsigned remaining) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  __syncthreads();  // every per-warp histogram is complete
+  {
+    // warp w sums bins 8w .. 8w + 7: lane l takes bin 8w + (l & 7) over warps
+    // 8(l >> 3) .. 8(l >> 3) + 7, then four lanes combine by shuffles
+    const int j = 8 * warp + (lane & 7), q = lane >> 3;
+    unsigned t = 0u;
+#pragma unroll
+    for (int w = 0; w < kRegWarps / 4; ++w) t += whist[(q * (kRegWarps / 4) + w) * kHistStride + j];
+    t += __shfl_xor_sync(0xffffffffu, t, 8);
+    t += __shfl_xor_sync(0xffffffffu, t, 16);
+    if (lane < 8) sh.hist[j] = t;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    unsigned c[8];
+    unsigned tot = 0;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      c[q] = sh.hist[255 - 8 * lane - q];
+      tot += c[q];
+    }
+    unsigned incl = tot;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const unsigned n = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += n;
+    }
+    const unsigned excl = incl - tot;
+    if (excl < remaining && incl >= remaining) {
+      unsigned cum = excl;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (cum + c[q] >= remaining) {
+          sh.prefix = (unsigned)(255 - 8 * lane - q);  // the chosen digit
+          sh.remaining = remaining - cum;
+          sh.eqcount = c[q];  // keys in contention with this digit
+          break;
+        }
+        cum += c[q];
+      }
+    }
+  }
+  __syncthreads();
+}
+
 __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(SelectArgs a, int JG) {
   extern __shared__ float4 s4[];  // [JG][1024]: scores of thread t, group g at s4[g*1024 + t]
-  // followed by the per-warp top-digit histograms [kRegWarps][256]
+  // followed by the per-warp radix histograms [kRegWarps][kHistStride]
   unsigned* whist = reinterpret_cast<unsigned*>(s4 + JG * kRegThreads);
   __shared__ RegScratch sh;
+  const float* sflat = reinterpret_cast<const float*>(s4);
   const int unit = a.unit0 + blockIdx.x;
   const int b = unit / a.n_kv_heads;
   const int kvh = unit - b * a.n_kv_heads;
@@ -651,148 +742,139 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
   const int n_cand = N - n_prot;
   const int k = min(max(a.k_head, 0), n_cand);
   const float eps = a.eps;
+  const bool radix = k > 0 && k < n_cand;
+  unsigned* wh = whist + warp * kHistStride;
   auto tok = [&](int g, int r) { return g * kGroupTokens + 4 * tid + r; };
-  auto is_cand = [&](int i) { return i < N && i >= ns && i < rs; };
+  auto is_cand = [&](int i) { return i >= ns && i < rs; };  // for i < N
+  auto score_of = [&](int bitpos) {  // bit 4g + r of the membership masks
+    return sflat[((bitpos >> 2) * kRegThreads + tid) * 4 + (bitpos & 3)];
+  };
+  auto zero_hist = [&]() {
+    for (int j = lane; j < 256; j += 32) wh[j] = 0u;
+    __syncwarp();
+  };
+
+  // statistics of the tail tokens this thread has met (the start of Eq. 2)
+  float smax = -INFINITY, sminpos = INFINITY, spos = 0.f;
+  int npos = 0;
+  auto add_tail = [&](float v) {
+    smax = fmaxf(smax, v);
+    if (v > 0.f) {
+      sminpos = fminf(sminpos, v);
+      spos += v;
+      ++npos;
+    }
+  };
 
   // ---- load: sanitise, fold -0 onto +0, protected positions -------------------
+  // every group's load is issued before the first is used
+  if (radix) zero_hist();
   bool bad = false;
   uint32_t cert = 0u, valid = 0u;
-  // every group's load in flight before the first use
+  float4 raw[kRegMaxGroups];
+#pragma unroll
+  for (int g = 0; g < kRegMaxGroups; ++g) {
+    raw[g] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (g < JG) {
+      const int i0 = tok(g, 0);
+      if (a.vec4 && i0 + 3 < N) {
+        raw[g] = __ldg(reinterpret_cast<const float4*>(sp + i0));
+      } else {
+        if (i0 < N) raw[g].x = __ldg(sp + i0);
+        if (i0 + 1 < N) raw[g].y = __ldg(sp + i0 + 1);
+        if (i0 + 2 < N) raw[g].z = __ldg(sp + i0 + 2);
+        if (i0 + 3 < N) raw[g].w = __ldg(sp + i0 + 3);
+      }
+    }
+  }
 #pragma unroll
   for (int g = 0; g < kRegMaxGroups; ++g) {
     if (g >= JG) break;
-    const int i0 = tok(g, 0);
-    float v[4];
-    if (a.vec4 && i0 + 3 < N) {
-      const float4 v4 = __ldg(reinterpret_cast<const float4*>(sp + i0));
-      v[0] = v4.x;
-      v[1] = v4.y;
-      v[2] = v4.z;
-      v[3] = v4.w;
-    } else {
-#pragma unroll
-      for (int r = 0; r < 4; ++r) v[r] = (i0 + r < N) ? __ldg(sp + i0 + r) : 0.f;
-    }
+    float v[4] = {raw[g].x, raw[g].y, raw[g].z, raw[g].w};
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
-      const int i = i0 + r;
+      const int i = tok(g, r);
       if (!isfinite(v[r])) {
         bad = bad || (i < N);
         v[r] = 0.f;
       }
       v[r] += 0.0f;
-      if (i < N) valid |= 1u << (4 * g + r);
-      if (i < N && !is_cand(i)) cert |= 1u << (4 * g + r);  // protected
+      if (i >= N) continue;
+      const uint32_t bit = 1u << (4 * g + r);
+      valid |= bit;
+      if (!is_cand(i)) cert |= bit;  // protected
+      else if (radix) atomicAdd(&wh[orderable_key(v[r]) >> 24], 1u);  // first digit
+      else if (k == 0) add_tail(v[r]);  // no top slice: every candidate is tail
     }
     s4[g * kRegThreads + tid] = make_float4(v[0], v[1], v[2], v[3]);
   }
 
-
   // ---- E1: top-k_head among the unprotected tokens ------------------------
-  // MSB-first radix select over 8-bit digits of the order-preserving keys.
-  // `live` holds the tokens whose key still matches the chosen prefix; after
-  // each digit, tokens above it join the certainty set and tokens below it
-  // drop out, so later passes touch only the few tokens still in contention.
-  if (k > 0 && k < n_cand) {
-    uint32_t live = valid & ~cert;  // the unprotected tokens
+  if (radix) {
+    uint32_t live = valid & ~cert;  // candidates whose keys match the chosen digits
     unsigned remaining = (unsigned)k;
+    bool done = false;
 #pragma unroll 1
-    for (int shift = 24; shift >= 0; shift -= 8) {
-      for (int j = tid; j < 256; j += kRegThreads) sh.hist[j] = 0u;
-      __syncthreads();
+    for (int shift = 24;; shift -= 8) {
+      choose_digit(whist, sh, remaining);
+      const unsigned digit = sh.prefix;
+      remaining = sh.remaining;
+      done = sh.eqcount == remaining;  // every key with this digit is in the slice
+      const bool last = done || shift == 0;
+      const int nshift = last ? 0 : shift - 8;
+      if (!last) zero_hist();
+      // a token with a higher digit joins the slice, a lower one the tail; an
+      // equal one stays in contention and counts toward the next digit
+      auto settle = [&](int bitpos, float v) {
+        const uint32_t key = orderable_key(v);
+        const unsigned d = (key >> shift) & 255u;
+        const uint32_t bit = 1u << bitpos;
+        if (d > digit || (d == digit && done)) {
+          cert |= bit;
+          live &= ~bit;
+        } else if (d < digit) {
+          live &= ~bit;
+          add_tail(v);
+        } else if (!last) {
+          atomicAdd(&wh[(key >> nshift) & 255u], 1u);
+        }
+      };
       if (shift == 24) {
-        // every candidate takes part: per-warp private histograms keep the
-        // crowded top bins of skewed scores from serialising across warps
-        unsigned* wh = whist + warp * 256;
-        for (int j = lane; j < 256; j += 32) wh[j] = 0u;
-        __syncwarp();
+        // every candidate is still in contention
 #pragma unroll 1
         for (int g = 0; g < JG; ++g) {
+          const uint32_t l4 = (live >> (4 * g)) & 0xFu;
+          if (!l4) continue;
           const float4 v4 = s4[g * kRegThreads + tid];
           const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
 #pragma unroll
           for (int r = 0; r < 4; ++r)
-            if ((live >> (4 * g + r)) & 1u) atomicAdd(&wh[orderable_key(vv[r]) >> 24], 1u);
-        }
-        __syncthreads();
-        for (int j = tid; j < 256; j += kRegThreads) {
-          unsigned t = 0u;
-#pragma unroll 8
-          for (int w = 0; w < kRegWarps; ++w) t += whist[w * 256 + j];
-          sh.hist[j] = t;
+            if ((l4 >> r) & 1u) settle(4 * g + r, vv[r]);
         }
       } else {
         for (uint32_t m = live; m; m &= m - 1) {
           const int bitpos = __ffs(m) - 1;
-          const float4 v4 = s4[(bitpos >> 2) * kRegThreads + tid];
-          const int r = bitpos & 3;
-          const float v = r == 0 ? v4.x : (r == 1 ? v4.y : (r == 2 ? v4.z : v4.w));
-          atomicAdd(&sh.hist[(orderable_key(v) >> shift) & 255u], 1u);
+          settle(bitpos, score_of(bitpos));
         }
       }
-      __syncthreads();
-      if (warp == 0) {
-        unsigned c[8];
-        unsigned tot = 0;
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          c[q] = sh.hist[255 - 8 * lane - q];
-          tot += c[q];
-        }
-        unsigned incl = tot;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const unsigned n = __shfl_up_sync(0xffffffffu, incl, o);
-          if (lane >= o) incl += n;
-        }
-        const unsigned excl = incl - tot;
-        if (excl < remaining && incl >= remaining) {
-          unsigned cum = excl;
-#pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            if (cum + c[q] >= remaining) {
-              sh.prefix = (unsigned)(255 - 8 * lane - q);  // the chosen digit
-              sh.remaining = remaining - cum;
-              sh.eqcount = c[q];  // live tokens with this digit
-              break;
-            }
-            cum += c[q];
-          }
-        }
-      }
-      __syncthreads();
-      const unsigned digit = sh.prefix;
-      remaining = sh.remaining;
-      for (uint32_t m = live; m; m &= m - 1) {
-        const int bitpos = __ffs(m) - 1;
-        const float4 v4 = s4[(bitpos >> 2) * kRegThreads + tid];
-        const int r = bitpos & 3;
-        const float v = r == 0 ? v4.x : (r == 1 ? v4.y : (r == 2 ? v4.z : v4.w));
-        const unsigned d = (orderable_key(v) >> shift) & 255u;
-        if (d != digit) {
-          live &= ~(1u << bitpos);
-          if (d > digit) cert |= 1u << bitpos;
-        }
-      }
+      if (last) break;
     }
-    // `live` now holds exactly the tokens whose key equals the k-th largest;
-    // the `remaining` lowest-index ones complete the top slice (all of them,
-    // without an ordered scan, when there are no more than that)
-    const uint32_t eq = live;
-    if (sh.eqcount <= remaining) {
-      cert |= eq;
-    } else {
-      ordered_scan(eq, JG, sh);
+    if (!done) {
+      // `live` holds the tokens whose key equals the k-th largest, more of
+      // them than are needed: the `remaining` lowest-index ones join the slice
+      uint32_t bl, bh;
+      ordered_scan(live, JG, sh, bl, bh);
 #pragma unroll 1
       for (int g = 0; g < JG; ++g) {
-        int run = sh.off[g][warp] + lane_prefix(eq, g);
+        const uint32_t e4 = (live >> (4 * g)) & 0xFu;
+        if (!e4) continue;
+        int run = sh.off[g][warp] + group_byte(bl, bh, g);
 #pragma unroll
         for (int r = 0; r < 4; ++r) {
-          const uint32_t bit = 1u << (4 * g + r);
-          if (eq & bit) {
-            if (run < (int)remaining) cert |= bit;
-            ++run;
-          }
+          if (!((e4 >> r) & 1u)) continue;
+          if (run < (int)remaining) cert |= 1u << (4 * g + r);
+          else add_tail(score_of(4 * g + r));
+          ++run;
         }
       }
     }
@@ -806,23 +888,6 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
   const int n_cert = n_prot + k;
   const int nT = N - n_cert;
   const int m = min(max(a.budget - n_cert, 0), nT);
-  float smax = -INFINITY, sminpos = INFINITY, spos = 0.f;
-  int npos = 0;
-#pragma unroll 1
-  for (int g = 0; g < JG; ++g) {
-    const float4 v4 = s4[g * kRegThreads + tid];
-    const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
-#pragma unroll
-    for (int r = 0; r < 4; ++r) {
-      if (!is_tail(g, r)) continue;
-      smax = fmaxf(smax, vv[r]);
-      if (vv[r] > 0.f) {
-        sminpos = fminf(sminpos, vv[r]);
-        spos += vv[r];
-        ++npos;
-      }
-    }
-  }
   smax = warp_max(smax);
   sminpos = warp_min(sminpos);
   npos = warp_sum(npos);
@@ -837,26 +902,23 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
   __syncthreads();
   combine_stats(sh);
   __syncthreads();
-  // Scalar decisions are taken once, by thread 0, and broadcast: the fp64
-  // arithmetic they use would otherwise run on every thread.
+  // Scalar decisions are taken once, by thread 0, and broadcast.
   if (tid == 0) {
     const float smax_b = sh.res_f[0], sminpos_b = sh.res_f[1];
     const int npos_b = sh.res_i[0];
     int md = kPiLinear;
     if (nT == 0 || (float)m <= eps * (float)nT) md = kPiFloor;
     else if ((float)m >= (float)npos_b + eps * (float)(nT - npos_b)) md = kPiAll;
-    sh.mode = md;
     sh.stop = md != kPiLinear;
     if (md == kPiLinear) {
       sh.lo = logf(eps / smax_b);
       sh.hi = logf(1.f / sminpos_b);
-      sh.c = fminf(fmaxf((float)((double)m / sh.res_d), expf(sh.lo)), expf(sh.hi));
+      sh.c = fminf(fmaxf((float)m / sh.res_f[2], expf(sh.lo)), expf(sh.hi));
     } else {
-      sh.c = 0.f;
+      sh.c = saturated_c(md);
     }
   }
   __syncthreads();
-  const int mode = sh.mode;
   float c = sh.c;
 #pragma unroll 1
   for (int it = 0; it < a.iters && !sh.stop; ++it) {
@@ -878,7 +940,7 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
     nhi = warp_sum(nhi);
     nlo = warp_sum(nlo);
     smid = warp_sum(smid);
-    __syncthreads();
+    // (the barrier closing the previous iteration ordered its reads of sh)
     if (lane == 0) {
       sh.ri[0][warp] = nhi;
       sh.ri[1][warp] = nlo;
@@ -887,24 +949,10 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
     __syncthreads();
     combine_partition(sh);
     if (tid == 0) {
-      const int nh = sh.res_i[0], nl = sh.res_i[1];
-      const double smid_d = sh.res_d;
-      const double gval = nh + (double)eps * nl + (double)c * smid_d;
       float lo = sh.lo, hi = sh.hi;
-      if (gval < (double)m) lo = fmaxf(lo, logf(c));
-      else hi = fminf(hi, logf(c));
-      const double clin = smid_d > 0.0 ? ((double)m - nh - (double)eps * nl) / smid_d : -1.0;
-      if (clin > 0.0 && fabs(clin - (double)c) <= 1e-6 * (double)c) {
-        sh.c = (float)clin;  // the partition at c reproduces its own solve
-        sh.stop = 1;
-      } else {
-        float next;
-        const float lcl = clin > 0.0 ? logf((float)clin) : -INFINITY;
-        if (clin > 0.0 && lcl > lo && lcl < hi) next = (float)clin;
-        else next = expf(0.5f * (lo + hi));
-        if (next == c) sh.stop = 1;
-        sh.c = next;
-      }
+      int stop = 0;
+      sh.c = water_fill_step(m, sh.res_i[0], sh.res_i[1], sh.res_f[2], eps, c, lo, hi, stop);
+      sh.stop = stop;
       sh.lo = lo;
       sh.hi = hi;
     }
@@ -914,7 +962,7 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
 
   // ---- E3 + E4a: draws and ordered compaction of (index, log 1/pi) --------
   const bool compact = a.n_kept != nullptr;
-  uint32_t keep = 0u;
+  uint32_t keep = cert;
   if (compact && a.systematic) {
     // Fixed-size systematic sampling at the same pi (Hajek 1964): the tail in
     // token order, cumulative sums C_i of pi in units of 2^-32 (each pi rounded
@@ -942,13 +990,12 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
       if (t4) atomicOr(&tailbits[i0 >> 5], t4 << (i0 & 31));
     }
     __syncthreads();
-    const float* sflat = reinterpret_cast<const float*>(s4);
     auto score_at = [&](int i) {  // token i of the load layout
       return sflat[((i >> 12) * kRegThreads + ((i & 4095) >> 2)) * 4 + (i & 3)];
     };
     // pi in units of 2^-32 (mod 2^32: pi = 1 adds 0 to the fraction)
     auto units32 = [&](float sv, bool& full) {
-      const float p = tail_pi(sv, mode, c, eps);
+      const float p = tail_pi(sv, c, eps);
       full = p >= 1.f;
       return full ? 0u : __float2uint_rn(p * 4294967296.f);
     };
@@ -984,8 +1031,8 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
         }
         const uint32_t after = frac + incl, before = after - v;
         const bool sel = is_t && (full || after < before);  // a carry: an integer crossed
-        const uint32_t m = __ballot_sync(0xffffffffu, sel);
-        if (lane == 0) keepbits[i >> 5] = m;
+        const uint32_t mk = __ballot_sync(0xffffffffu, sel);
+        if (lane == 0) keepbits[i >> 5] = mk;
         frac += __shfl_sync(0xffffffffu, incl, 31);
       }
     }
@@ -993,48 +1040,57 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
 #pragma unroll 1
     for (int g = 0; g < JG; ++g) {
       const int i0 = tok(g, 0);
-      const uint32_t k4 = (keepbits[i0 >> 5] >> (i0 & 31)) & 0xFu;
-      keep |= (k4 | ((cert & valid) >> (4 * g) & 0xFu)) << (4 * g);
+      keep |= ((keepbits[i0 >> 5] >> (i0 & 31)) & 0xFu) << (4 * g);
     }
-  }
-#pragma unroll 1
-  for (int g = 0; g < JG; ++g) {
-    const float4 v4 = s4[g * kRegThreads + tid];
-    const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
-    const bool any_tail = ((tail >> (4 * g)) & 0xFu) != 0u;
-    uint4 w = make_uint4(0u, 0u, 0u, 0u);
-    if (compact && !a.systematic && __any_sync(0xffffffffu, any_tail))
-      w = draw_block(a.seed, a.layer, b, kvh, g * kRegThreads + tid);
-    const uint32_t wr[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-    for (int r = 0; r < 4; ++r) {
-      const int i = tok(g, r);
-      if (!((valid >> (4 * g + r)) & 1u)) continue;
-      const bool ct = (cert >> (4 * g + r)) & 1u;
-      const float pi = ct ? 1.f : tail_pi(vv[r], mode, c, eps);
-      if (a.pi_out) a.pi_out[(size_t)unit * Nrow + i] = pi;
-      if (a.mask_out) a.mask_out[(size_t)unit * Nrow + i] = ct ? 1 : 0;
-      if (compact && !a.systematic && (ct || word_to_uniform(wr[r]) < pi))
-        keep |= 1u << (4 * g + r);
-    }
-  }
-  if (compact) {
-    const int total = ordered_scan(keep, JG, sh);
+  } else if (compact) {
+    // Poisson design: keep a tail token when its uniform falls below pi
 #pragma unroll 1
     for (int g = 0; g < JG; ++g) {
-      int p = sh.off[g][warp] + lane_prefix(keep, g);
+      const uint32_t t4 = (tail >> (4 * g)) & 0xFu;
+      if (!__any_sync(0xffffffffu, t4 != 0u)) continue;
+      const uint4 w = draw_block(a.seed, a.layer, b, kvh, g * kRegThreads + tid);
+      if (!t4) continue;
+      const float4 v4 = s4[g * kRegThreads + tid];
+      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+      const uint32_t wr[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+        if (((t4 >> r) & 1u) && word_to_uniform(wr[r]) < tail_pi(vv[r], c, eps))
+          keep |= 1u << (4 * g + r);
+    }
+  }
+  if (a.pi_out || a.mask_out) {
+#pragma unroll 1
+    for (int g = 0; g < JG; ++g) {
       const float4 v4 = s4[g * kRegThreads + tid];
       const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
 #pragma unroll
       for (int r = 0; r < 4; ++r) {
-        const uint32_t bit = 1u << (4 * g + r);
-        if (!(keep & bit)) continue;
+        const int i = tok(g, r);
+        if (!((valid >> (4 * g + r)) & 1u)) continue;
+        const bool ct = (cert >> (4 * g + r)) & 1u;
+        if (a.pi_out) a.pi_out[(size_t)unit * Nrow + i] = ct ? 1.f : tail_pi(vv[r], c, eps);
+        if (a.mask_out) a.mask_out[(size_t)unit * Nrow + i] = ct ? 1 : 0;
+      }
+    }
+  }
+  if (compact) {
+    uint32_t bl, bh;
+    const int total = ordered_scan(keep, JG, sh, bl, bh);
+    int32_t* idx_row = a.idx_c + (size_t)unit * a.cap;
+    float* logw_row = a.logw_c + (size_t)unit * a.cap;
+#pragma unroll 1
+    for (int g = 0; g < JG; ++g) {
+      // one store per kept token, group by group so that a warp's stores fall
+      // close together
+      int p = sh.off[g][warp] + group_byte(bl, bh, g);
+      for (uint32_t k4 = (keep >> (4 * g)) & 0xFu; k4; k4 &= k4 - 1, ++p) {
+        const int bitpos = 4 * g + __ffs(k4) - 1;
         if (p < a.cap) {
-          const float pi = (cert & bit) ? 1.f : tail_pi(vv[r], mode, c, eps);
-          a.idx_c[(size_t)unit * a.cap + p] = tok(g, r);
-          a.logw_c[(size_t)unit * a.cap + p] = pi >= 1.f ? 0.f : -logf(pi);
+          const float pi = ((cert >> bitpos) & 1u) ? 1.f : tail_pi(score_of(bitpos), c, eps);
+          idx_row[p] = g * kGroupTokens + 4 * tid + (bitpos & 3);
+          logw_row[p] = pi >= 1.f ? 0.f : -logf(pi);
         }
-        ++p;
       }
     }
     if (tid == 0) {
@@ -1160,7 +1216,7 @@ ebd_status launch_select_range(const ebd_design* d, const float* scores, const i
   if (groups <= kRegMaxGroups) {
     // the limit is set on every launch: with the kernel's static shared memory
     // even 48 KB of dynamic memory is above the default
-    const size_t smem = (size_t)groups * kRegThreads * sizeof(float4) + kRegWarps * 256 * 4;
+    const size_t smem = (size_t)groups * kRegThreads * sizeof(float4) + kRegWarps * kHistStride * 4;
     if (cudaFuncSetAttribute(evict_select_smem_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem) != cudaSuccess)
       return EBD_ERR_CUDA;
