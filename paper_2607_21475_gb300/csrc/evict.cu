@@ -960,6 +960,21 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
     c = sh.c;
   }
 
+  if (a.pi_out || a.mask_out) {
+#pragma unroll 1
+    for (int g = 0; g < JG; ++g) {
+      const float4 v4 = s4[g * kRegThreads + tid];
+      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const int i = tok(g, r);
+        if (!((valid >> (4 * g + r)) & 1u)) continue;
+        const bool ct = (cert >> (4 * g + r)) & 1u;
+        if (a.pi_out) a.pi_out[(size_t)unit * Nrow + i] = ct ? 1.f : tail_pi(vv[r], c, eps);
+        if (a.mask_out) a.mask_out[(size_t)unit * Nrow + i] = ct ? 1 : 0;
+      }
+    }
+  }
   // ---- E3 + E4a: draws and ordered compaction of (index, log 1/pi) --------
   const bool compact = a.n_kept != nullptr;
   uint32_t keep = cert;
@@ -1040,7 +1055,17 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
 #pragma unroll 1
     for (int g = 0; g < JG; ++g) {
       const int i0 = tok(g, 0);
-      keep |= ((keepbits[i0 >> 5] >> (i0 & 31)) & 0xFu) << (4 * g);
+      const uint32_t k4 = (keepbits[i0 >> 5] >> (i0 & 31)) & 0xFu;
+      if (!k4) continue;
+      keep |= k4 << (4 * g);
+      float4& slot = s4[g * kRegThreads + tid];
+      float vv[4] = {slot.x, slot.y, slot.z, slot.w};
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const float pi = tail_pi(vv[r], c, eps);
+        if ((k4 >> r) & 1u) vv[r] = pi >= 1.f ? 0.f : -logf(pi);
+      }
+      slot = make_float4(vv[0], vv[1], vv[2], vv[3]);
     }
   } else if (compact) {
     // Poisson design: keep a tail token when its uniform falls below pi
@@ -1050,27 +1075,21 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
       if (!__any_sync(0xffffffffu, t4 != 0u)) continue;
       const uint4 w = draw_block(a.seed, a.layer, b, kvh, g * kRegThreads + tid);
       if (!t4) continue;
-      const float4 v4 = s4[g * kRegThreads + tid];
-      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+      float4& slot = s4[g * kRegThreads + tid];
+      float vv[4] = {slot.x, slot.y, slot.z, slot.w};
       const uint32_t wr[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-      for (int r = 0; r < 4; ++r)
-        if (((t4 >> r) & 1u) && word_to_uniform(wr[r]) < tail_pi(vv[r], c, eps))
-          keep |= 1u << (4 * g + r);
-    }
-  }
-  if (a.pi_out || a.mask_out) {
-#pragma unroll 1
-    for (int g = 0; g < JG; ++g) {
-      const float4 v4 = s4[g * kRegThreads + tid];
-      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+      uint32_t k4 = 0u;
 #pragma unroll
       for (int r = 0; r < 4; ++r) {
-        const int i = tok(g, r);
-        if (!((valid >> (4 * g + r)) & 1u)) continue;
-        const bool ct = (cert >> (4 * g + r)) & 1u;
-        if (a.pi_out) a.pi_out[(size_t)unit * Nrow + i] = ct ? 1.f : tail_pi(vv[r], c, eps);
-        if (a.mask_out) a.mask_out[(size_t)unit * Nrow + i] = ct ? 1 : 0;
+        const float pi = tail_pi(vv[r], c, eps);
+        if (((t4 >> r) & 1u) && word_to_uniform(wr[r]) < pi) {
+          k4 |= 1u << r;
+          vv[r] = pi >= 1.f ? 0.f : -logf(pi);  // the score is not needed again
+        }
+      }
+      if (k4) {
+        slot = make_float4(vv[0], vv[1], vv[2], vv[3]);
+        keep |= k4 << (4 * g);
       }
     }
   }
@@ -1087,9 +1106,9 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
       for (uint32_t k4 = (keep >> (4 * g)) & 0xFu; k4; k4 &= k4 - 1, ++p) {
         const int bitpos = 4 * g + __ffs(k4) - 1;
         if (p < a.cap) {
-          const float pi = ((cert >> bitpos) & 1u) ? 1.f : tail_pi(score_of(bitpos), c, eps);
+          // a kept tail token's slot holds its log(1/pi) by now
           idx_row[p] = g * kGroupTokens + 4 * tid + (bitpos & 3);
-          logw_row[p] = pi >= 1.f ? 0.f : -logf(pi);
+          logw_row[p] = ((cert >> bitpos) & 1u) ? 0.f : score_of(bitpos);
         }
       }
     }
