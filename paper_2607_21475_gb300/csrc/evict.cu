@@ -31,6 +31,7 @@
 
 #include "common.cuh"
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace ebd {
 
@@ -553,6 +554,12 @@ struct RegScratch {
   int stop;
   unsigned prefix, remaining, eqcount;
   int total;
+  // published for the other CTAs of a unit's cluster (two buffers: an
+  // exchange reuses the buffer of the one before the last)
+  unsigned hist_x[2][256];
+  float xf[2][3];
+  int xi[2][2];
+  int xres[2];
 };
 
 // Cross-warp combine of per-warp partials written to sh.rf / sh.ri by lane 0
@@ -670,13 +677,42 @@ __device__ __forceinline__ int ordered_scan(uint32_t flags, int JG, RegScratch& 
   return sh.total;
 }
 
+// Exclusive prefix over the ranks of a unit's cluster of a per-CTA count `v`
+// (the same in every thread of the CTA), and the cluster total; every thread
+// gets both.  Without a cluster (C == 1) that is (0, v).
+__device__ __forceinline__ int cluster_scan(int v, RegScratch& sh, int C, int crank, int& xpar,
+                                            int& total) {
+  if (C == 1) {
+    total = v;
+    return 0;
+  }
+  if (threadIdx.x == 0) sh.xi[xpar][0] = v;
+  cluster_barrier();
+  if (threadIdx.x == 0) {
+    const uint32_t addr = smem_u32(&sh.xi[xpar][0]);
+    unsigned below = 0u, tot = 0u;  // unsigned: the systematic walk sums modulo 2^32
+    for (int q = 0; q < C; ++q) {
+      const unsigned x = ld_cluster_u32(cluster_map(addr, (uint32_t)q));
+      if (q < crank) below += x;
+      tot += x;
+    }
+    sh.xres[0] = (int)below;
+    sh.xres[1] = (int)tot;
+  }
+  __syncthreads();
+  xpar ^= 1;
+  total = sh.xres[1];
+  return sh.xres[0];
+}
+
 // One radix-select step: the per-warp histograms of the current digit are
-// summed into sh.hist, then warp 0 finds, from
+// summed into sh.hist (over every CTA of the unit's cluster when C > 1), then
+// warp 0 finds, from
 // the top, the digit value holding the `remaining`-th largest key still in
 // contention and publishes it (sh.prefix), the rank left inside it
 // (sh.remaining) and its count (sh.eqcount).  Three barriers.
 __device__ __forceinline__ void choose_digit(const unsigned* whist, RegScratch& sh,
-                                             unsigned remaining) {
+                                             unsigned remaining, int C, int dpar) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   __syncthreads();  // every per-warp histogram is complete
   {
@@ -688,7 +724,17 @@ __device__ __forceinline__ void choose_digit(const unsigned* whist, RegScratch& 
     for (int w = 0; w < kRegWarps / 4; ++w) t += whist[(q * (kRegWarps / 4) + w) * kHistStride + j];
     t += __shfl_xor_sync(0xffffffffu, t, 8);
     t += __shfl_xor_sync(0xffffffffu, t, 16);
-    if (lane < 8) sh.hist[j] = t;
+    if (lane < 8) (C > 1 ? sh.hist_x[dpar][j] : sh.hist[j]) = t;
+  }
+  if (C > 1) {
+    // the cluster's histogram: every CTA sums all CTAs' histograms
+    cluster_barrier();
+    if (tid < 256) {
+      const uint32_t addr = smem_u32(&sh.hist_x[dpar][tid]);
+      unsigned t = 0u;
+      for (int q = 0; q < C; ++q) t += ld_cluster_u32(cluster_map(addr, (uint32_t)q));
+      sh.hist[tid] = t;
+    }
   }
   __syncthreads();
   if (warp == 0) {
@@ -729,7 +775,9 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
   unsigned* whist = reinterpret_cast<unsigned*>(s4 + JG * kRegThreads);
   __shared__ RegScratch sh;
   const float* sflat = reinterpret_cast<const float*>(s4);
-  const int unit = a.unit0 + blockIdx.x;
+  const int C = (int)cluster_size();      // CTAs per unit: 1 without a cluster launch
+  const int crank = (int)cluster_rank();  // this CTA's slice of the unit
+  const int unit = a.unit0 + (int)blockIdx.x / C;
   const int b = unit / a.n_kv_heads;
   const int kvh = unit - b * a.n_kv_heads;
   const int Nrow = a.n_ctx;
@@ -744,7 +792,10 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
   const float eps = a.eps;
   const bool radix = k > 0 && k < n_cand;
   unsigned* wh = whist + warp * kHistStride;
-  auto tok = [&](int g, int r) { return g * kGroupTokens + 4 * tid + r; };
+  const int t0 = crank * JG * kGroupTokens;  // first token of this CTA's slice
+  auto ltok = [&](int g, int r) { return g * kGroupTokens + 4 * tid + r; };  // within the slice
+  auto tok = [&](int g, int r) { return t0 + ltok(g, r); };
+  int xpar = 0;  // cluster exchange buffer (cluster-uniform)
   auto is_cand = [&](int i) { return i >= ns && i < rs; };  // for i < N
   auto score_of = [&](int bitpos) {  // bit 4g + r of the membership masks
     return sflat[((bitpos >> 2) * kRegThreads + tid) * 4 + (bitpos & 3)];
@@ -816,7 +867,7 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
     bool done = false;
 #pragma unroll 1
     for (int shift = 24;; shift -= 8) {
-      choose_digit(whist, sh, remaining);
+      choose_digit(whist, sh, remaining, C, (shift >> 3) & 1);
       const unsigned digit = sh.prefix;
       remaining = sh.remaining;
       done = sh.eqcount == remaining;  // every key with this digit is in the slice
@@ -863,12 +914,13 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
       // `live` holds the tokens whose key equals the k-th largest, more of
       // them than are needed: the `remaining` lowest-index ones join the slice
       uint32_t bl, bh;
-      ordered_scan(live, JG, sh, bl, bh);
+      int ties_all;
+      const int lower = cluster_scan(ordered_scan(live, JG, sh, bl, bh), sh, C, crank, xpar, ties_all);
 #pragma unroll 1
       for (int g = 0; g < JG; ++g) {
         const uint32_t e4 = (live >> (4 * g)) & 0xFu;
         if (!e4) continue;
-        int run = sh.off[g][warp] + group_byte(bl, bh, g);
+        int run = lower + sh.off[g][warp] + group_byte(bl, bh, g);
 #pragma unroll
         for (int r = 0; r < 4; ++r) {
           if (!((e4 >> r) & 1u)) continue;
@@ -902,6 +954,31 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
   __syncthreads();
   combine_stats(sh);
   __syncthreads();
+  if (C > 1) {
+    // the cluster's statistics, combined in rank order (the same in every CTA)
+    if (tid == 0) {
+      sh.xf[xpar][0] = sh.res_f[0];
+      sh.xf[xpar][1] = sh.res_f[1];
+      sh.xf[xpar][2] = sh.res_f[2];
+      sh.xi[xpar][0] = sh.res_i[0];
+    }
+    cluster_barrier();
+    if (tid == 0) {
+      float mx = -INFINITY, mn = INFINITY, sd = 0.f;
+      int n = 0;
+      for (int q = 0; q < C; ++q) {
+        mx = fmaxf(mx, ld_cluster_f32(cluster_map(smem_u32(&sh.xf[xpar][0]), (uint32_t)q)));
+        mn = fminf(mn, ld_cluster_f32(cluster_map(smem_u32(&sh.xf[xpar][1]), (uint32_t)q)));
+        sd += ld_cluster_f32(cluster_map(smem_u32(&sh.xf[xpar][2]), (uint32_t)q));
+        n += (int)ld_cluster_u32(cluster_map(smem_u32(&sh.xi[xpar][0]), (uint32_t)q));
+      }
+      sh.res_f[0] = mx;
+      sh.res_f[1] = mn;
+      sh.res_f[2] = sd;
+      sh.res_i[0] = n;
+    }
+    xpar ^= 1;
+  }
   // Scalar decisions are taken once, by thread 0, and broadcast.
   if (tid == 0) {
     const float smax_b = sh.res_f[0], sminpos_b = sh.res_f[1];
@@ -948,6 +1025,27 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
     }
     __syncthreads();
     combine_partition(sh);
+    if (C > 1) {
+      if (tid == 0) {
+        sh.xf[xpar][0] = sh.res_f[2];
+        sh.xi[xpar][0] = sh.res_i[0];
+        sh.xi[xpar][1] = sh.res_i[1];
+      }
+      cluster_barrier();
+      if (tid == 0) {
+        float sd = 0.f;
+        int nh = 0, nl = 0;
+        for (int q = 0; q < C; ++q) {
+          sd += ld_cluster_f32(cluster_map(smem_u32(&sh.xf[xpar][0]), (uint32_t)q));
+          nh += (int)ld_cluster_u32(cluster_map(smem_u32(&sh.xi[xpar][0]), (uint32_t)q));
+          nl += (int)ld_cluster_u32(cluster_map(smem_u32(&sh.xi[xpar][1]), (uint32_t)q));
+        }
+        sh.res_f[2] = sd;
+        sh.res_i[0] = nh;
+        sh.res_i[1] = nl;
+      }
+      xpar ^= 1;
+    }
     if (tid == 0) {
       float lo = sh.lo, hi = sh.hi;
       int stop = 0;
@@ -1001,7 +1099,7 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
 #pragma unroll 1
     for (int g = 0; g < JG; ++g) {
       const uint32_t t4 = (tail >> (4 * g)) & 0xFu;
-      const int i0 = tok(g, 0);
+      const int i0 = ltok(g, 0);
       if (t4) atomicOr(&tailbits[i0 >> 5], t4 << (i0 & 31));
     }
     __syncthreads();
@@ -1028,7 +1126,12 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
     for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
     if (lane == 0) sh.ll[warp] = (long long)part;
     __syncthreads();
-    uint32_t frac = 0u - u32;  // fractional part of C - u before this warp's tokens
+    uint32_t cta_part = 0u;
+#pragma unroll 8
+    for (int w2 = 0; w2 < kRegWarps; ++w2) cta_part += (uint32_t)sh.ll[w2];
+    int parts_all;
+    // fractional part of C - u before this warp's tokens
+    uint32_t frac = 0u - u32 + (uint32_t)cluster_scan((int)cta_part, sh, C, crank, xpar, parts_all);
 #pragma unroll 8
     for (int w2 = 0; w2 < kRegWarps; ++w2) frac += w2 < warp ? (uint32_t)sh.ll[w2] : 0u;
     if (wbase < ntok) {
@@ -1054,7 +1157,7 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
     __syncthreads();
 #pragma unroll 1
     for (int g = 0; g < JG; ++g) {
-      const int i0 = tok(g, 0);
+      const int i0 = ltok(g, 0);
       const uint32_t k4 = (keepbits[i0 >> 5] >> (i0 & 31)) & 0xFu;
       if (!k4) continue;
       keep |= k4 << (4 * g);
@@ -1073,7 +1176,7 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
     for (int g = 0; g < JG; ++g) {
       const uint32_t t4 = (tail >> (4 * g)) & 0xFu;
       if (!__any_sync(0xffffffffu, t4 != 0u)) continue;
-      const uint4 w = draw_block(a.seed, a.layer, b, kvh, g * kRegThreads + tid);
+      const uint4 w = draw_block(a.seed, a.layer, b, kvh, (t0 >> 2) + g * kRegThreads + tid);
       if (!t4) continue;
       float4& slot = s4[g * kRegThreads + tid];
       float vv[4] = {slot.x, slot.y, slot.z, slot.w};
@@ -1095,29 +1198,31 @@ __global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(Selec
   }
   if (compact) {
     uint32_t bl, bh;
-    const int total = ordered_scan(keep, JG, sh, bl, bh);
+    int total;
+    const int lower = cluster_scan(ordered_scan(keep, JG, sh, bl, bh), sh, C, crank, xpar, total);
     int32_t* idx_row = a.idx_c + (size_t)unit * a.cap;
     float* logw_row = a.logw_c + (size_t)unit * a.cap;
 #pragma unroll 1
     for (int g = 0; g < JG; ++g) {
       // one store per kept token, group by group so that a warp's stores fall
       // close together
-      int p = sh.off[g][warp] + group_byte(bl, bh, g);
+      int p = lower + sh.off[g][warp] + group_byte(bl, bh, g);
       for (uint32_t k4 = (keep >> (4 * g)) & 0xFu; k4; k4 &= k4 - 1, ++p) {
         const int bitpos = 4 * g + __ffs(k4) - 1;
         if (p < a.cap) {
           // a kept tail token's slot holds its log(1/pi) by now
-          idx_row[p] = g * kGroupTokens + 4 * tid + (bitpos & 3);
+          idx_row[p] = tok(g, bitpos & 3);
           logw_row[p] = ((cert >> bitpos) & 1u) ? 0.f : score_of(bitpos);
         }
       }
     }
-    if (tid == 0) {
+    if (tid == 0 && crank == 0) {
       a.n_kept[unit] = total;
       if (total > a.cap) raise_status(a.dev_status, EBD_DEV_CAPACITY);
     }
   }
   if (__syncthreads_or(bad) && tid == 0) raise_status(a.dev_status, EBD_DEV_NONFINITE);
+  if (C > 1) cluster_barrier();  // no CTA leaves while another may read its shared memory
 }
 
 // E4b: copy kept K and V rows (16-byte chunks, `cpr` chunks per row).
@@ -1201,10 +1306,27 @@ ebd_status check_design(const ebd_design* d) {
   return EBD_OK;
 }
 
+// CTAs per unit for the shared-memory select: as many as the unit's scores
+// need (32768 tokens per CTA), then more, up to a cluster of 8, while the
+// request would leave SMs idle and every CTA keeps at least 4096 tokens.
+// 0: the context is too long for a cluster (the global-memory kernel takes it).
+constexpr int kMaxSelectCluster = 8;
+int select_cluster_size(int n_ctx, int units) {
+  const int per_cta = kRegMaxGroups * kGroupTokens;
+  const int need = (n_ctx + per_cta - 1) / per_cta;
+  if (need > kMaxSelectCluster) return 0;
+  int C = need;
+  const long long sms = sm_count();
+  while (2 * C <= kMaxSelectCluster && (long long)units * 2 * C <= sms &&
+         n_ctx >= 2 * C * kGroupTokens)
+    C *= 2;
+  return C;
+}
+
 ebd_status launch_select_range(const ebd_design* d, const float* scores, const int32_t* n_len,
                                float* pi, uint8_t* mask, int32_t* idx_c, float* logw_c,
                                int32_t* n_kept, int cap, int32_t* dev_status, int unit0,
-                               int n_units, cudaStream_t stream) {
+                               int n_units, cudaStream_t stream, int ctas_per_unit) {
   SelectArgs a;
   a.scores = scores;
   a.n_ctx = d->n_ctx;
@@ -1230,8 +1352,32 @@ ebd_status launch_select_range(const ebd_design* d, const float* scores, const i
   a.unit0 = unit0;
   const int units = n_units;
   if (units < 1) return EBD_OK;
+  const int C = ctas_per_unit > 0 ? ctas_per_unit : select_cluster_size(d->n_ctx, units);
+  if (C > 1) {
+    // a cluster of C CTAs per unit, CTA r holding tokens [r S, (r + 1) S)
+    const int per = (d->n_ctx + C - 1) / C;
+    const int jg = (per + kGroupTokens - 1) / kGroupTokens;
+    const size_t smem = (size_t)jg * kRegThreads * sizeof(float4) + kRegWarps * kHistStride * 4;
+    if (cudaFuncSetAttribute(evict_select_smem_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem) != cudaSuccess)
+      return EBD_ERR_CUDA;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(units * C));
+    cfg.blockDim = dim3(kRegThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)C;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, evict_select_smem_kernel, a, jg) == cudaSuccess)
+      return launch_status();
+    (void)cudaGetLastError();  // the cluster could not be placed: one CTA per unit below
+  }
   const int groups = (d->n_ctx + kGroupTokens - 1) / kGroupTokens;
-  if (a.systematic && groups > kRegMaxGroups && idx_c) return EBD_ERR_UNSUPPORTED;
   if (groups <= kRegMaxGroups) {
     // the limit is set on every launch: with the kernel's static shared memory
     // even 48 KB of dynamic memory is above the default
@@ -1242,6 +1388,7 @@ ebd_status launch_select_range(const ebd_design* d, const float* scores, const i
     evict_select_smem_kernel<<<units, kRegThreads, smem, stream>>>(a, groups);
     return launch_status();
   }
+  if (a.systematic && idx_c) return EBD_ERR_UNSUPPORTED;
   // certainty bits (padded to 16 bytes), then the per-warp first-digit histograms
   const int words_pad = ((d->n_ctx + 31) / 32 + 3) & ~3;
   const size_t smem = (size_t)words_pad * 4 + (size_t)kSelWarps * 256 * 4;
@@ -1256,7 +1403,7 @@ ebd_status launch_select(const ebd_design* d, const float* scores, const int32_t
                          float* pi, uint8_t* mask, int32_t* idx_c, float* logw_c, int32_t* n_kept,
                          int cap, int32_t* dev_status, cudaStream_t stream) {
   return launch_select_range(d, scores, n_len, pi, mask, idx_c, logw_c, n_kept, cap, dev_status,
-                             0, d->batch * d->n_kv_heads, stream);
+                             0, d->batch * d->n_kv_heads, stream, 0);
 }
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -1441,13 +1588,17 @@ EvictStreams* evict_streams(cudaStream_t s) {
   return e.ok ? &e : nullptr;
 }
 
-// E1-E4 for every unit: chunks of sm_count() units, pipelined over streams.
+// E1-E4 for every unit: chunks of one select wave of units, pipelined over streams.
 ebd_status select_and_gather(const ebd_design* d, ebd_dtype dtype, const float* scores,
                              const void* K, const void* V, void* K_c, void* V_c, float* logw_c,
                              int32_t* idx_c, int32_t* n_kept, int cap, int32_t* dev_status,
                              cudaStream_t s) {
   const int units = d->batch * d->n_kv_heads;
-  const int chunk = sm_count();
+  // One cluster size for the whole call, so that every chunk splits its units
+  // as one launch over all of them would (the float sums of Eq. 2 follow the
+  // split).  A chunk is one select wave: an SM per CTA.
+  const int C = select_cluster_size(d->n_ctx, units);
+  const int chunk = C > 1 ? (sm_count() / C > 0 ? sm_count() / C : 1) : sm_count();
   EvictStreams* es = units > chunk ? evict_streams(s) : nullptr;
   if (!es) {
     ebd_status st = launch_select(d, scores, nullptr, nullptr, nullptr, idx_c, logw_c, n_kept,
@@ -1471,7 +1622,7 @@ ebd_status select_and_gather(const ebd_design* d, ebd_dtype dtype, const float* 
     const int u0 = c * chunk;
     const int n = units - u0 < chunk ? units - u0 : chunk;
     st = launch_select_range(d, scores, nullptr, nullptr, nullptr, idx_c, logw_c, n_kept, cap,
-                             dev_status, u0, n, cs);
+                             dev_status, u0, n, cs, C);
     if (st == EBD_OK)
       st = launch_gather_range(d, dtype, K, V, idx_c, n_kept, cap, K_c, V_c, u0, n, cs);
   }

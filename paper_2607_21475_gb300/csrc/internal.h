@@ -35,11 +35,18 @@ ebd_status launch_gather(const ebd_design* d, ebd_dtype dtype, const void* K, co
                          const int32_t* idx_c, const int32_t* n_kept, int cap, void* K_c,
                          void* V_c, cudaStream_t s);
 
-// The same for the units [unit0, unit0 + n_units) only.
+// The same for the units [unit0, unit0 + n_units) only.  `ctas_per_unit`:
+// the cluster size of the shared-memory select (0: chosen for this launch's
+// units; a caller that splits one request into several launches passes the
+// size chosen for the whole request, so each unit is split the same way).
 ebd_status launch_select_range(const ebd_design* d, const float* scores, const int32_t* n_len,
                                float* pi, uint8_t* mask, int32_t* idx_c, float* logw_c,
                                int32_t* n_kept, int cap, int32_t* dev_status, int unit0,
-                               int n_units, cudaStream_t stream);
+                               int n_units, cudaStream_t stream, int ctas_per_unit);
+
+// CTAs per unit of the shared-memory select for `units` units of n_ctx
+// tokens (0 when the context is too long for a cluster).
+int select_cluster_size(int n_ctx, int units);
 ebd_status launch_gather_range(const ebd_design* d, ebd_dtype dtype, const void* K,
                                const void* V, const int32_t* idx_c, const int32_t* n_kept,
                                int cap, void* K_c, void* V_c, int unit0, int n_units,

@@ -72,6 +72,8 @@ PI_CASES = [
     (70001, 1400, 7000, "lognormal"),  # ragged, beyond one smem tile of bits
     (50000, 1000, 5000, "ties"),       # large context: ordered scan of the tied top keys
     (40000, 0, 12000, "pareto"),       # large context, no top slice, clipped tail
+    (250000, 5000, 25000, "lognormal"),  # a cluster of eight CTAs per unit
+    (131072, 2600, 13000, "ties"),     # ties ordered across the CTAs of a cluster
 ]
 
 
@@ -141,6 +143,8 @@ EVICT_CASES = [
     (1, 1, 1, 64, torch.float32, 2, 1, 64),
     (1, 2, 40000, 64, torch.float32, 800, 4000, 4480),      # large context (global scores)
     (2, 1, 65537, 128, torch.bfloat16, 1300, 6500, 7104),   # large, ragged (scalar loads)
+    (1, 1, 100003, 64, torch.float32, 2000, 10000, 10496),  # cluster with a ragged and an empty CTA
+    (1, 1, 300007, 64, torch.float32, 6000, 30000, 31232),  # beyond a cluster: global scores
 ]
 
 
@@ -230,6 +234,59 @@ def test_evict_pipelined_chunks_match_single_stream_and_oracle(E, B, H, N, d, dt
                            piped.logw_c[b, h, :kg].cpu().double().numpy(),
                            bits(piped.K_c[b, h, :kg]), bits(piped.V_c[b, h, :kg]),
                            Kb[b, h], Vb[b, h], cap)
+
+
+def test_evict_cluster_chunks_match_single_launch_and_oracle(E):
+    """Contexts over 32768 tokens split each unit over a cluster of CTAs (two
+    here); with more units than one wave of clusters holds, ebd_evict also
+    pipelines chunks of units.  The outputs equal one select and one gather
+    launch, eagerly and replayed from a captured graph, and sampled units
+    (chunk edges) match the oracle."""
+    B, H, N, d, dtype = 20, 8, 33000, 64, torch.bfloat16
+    k_head, budget, cap = N // 50, N // 10, 3712
+    g = torch.Generator(device=DEV).manual_seed(5)
+    Kg = torch.randn((B, H, N, d), generator=g, device=DEV).to(dtype)
+    Vg = torch.randn((B, H, N, d), generator=g, device=DEV).to(dtype)
+    sg = torch.exp(1.5 * torch.randn((B, H, N), generator=g, device=DEV))
+    des = _design(E, B, H, 1, d, N, 5, 99, k_head, budget)
+    ref = E.alloc_compact(B, H, cap, d, dtype, DEV)
+    E.ebd_select(des, sg, ref)
+    E.ebd_gather(des, Kg, Vg, ref)
+    piped = E.alloc_compact(B, H, cap, d, dtype, DEV)
+    E.ebd_evict(des, Kg, Vg, sg, None, piped)
+    graphed = E.alloc_compact(B, H, cap, d, dtype, DEV)
+    torch.cuda.synchronize()
+    gr = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gr):
+        E.ebd_evict(des, Kg, Vg, sg, None, graphed)
+    gr.replay()
+    torch.cuda.synchronize()
+    assert ref.dev_status.item() == 0
+    for cc in (piped, graphed):
+        assert cc.dev_status.item() == 0
+        assert torch.equal(cc.n_kept, ref.n_kept)
+        for b in range(B):
+            for h in range(H):
+                n = min(int(ref.n_kept[b, h]), cap)
+                assert torch.equal(cc.idx_c[b, h, :n], ref.idx_c[b, h, :n])
+                assert torch.equal(cc.logw_c[b, h, :n], ref.logw_c[b, h, :n])
+                assert torch.equal(cc.K_c[b, h, :n], ref.K_c[b, h, :n])
+                assert torch.equal(cc.V_c[b, h, :n], ref.V_c[b, h, :n])
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    wave = sms // 2
+    for u in sorted({0, wave - 1, wave, min(2 * wave, B * H - 1), B * H - 1}):
+        b, h = divmod(u, H)
+        Ku, Vu = Kg[b, h].cpu(), Vg[b, h].cpu()
+        su = sg[b, h].cpu()
+        r = O.evict_unit(Ku.double().numpy(), Vu.double().numpy(), su.numpy(), n_sink=4,
+                         n_recent=32, k_head=k_head, budget_tokens=budget, eps=1e-6, seed=99,
+                         layer=5, b=b, kvh=h, capacity=cap)
+        n = int(piped.n_kept[b, h])
+        kg = min(n, cap)
+        compare_evict_unit(r, n, piped.idx_c[b, h, :kg].cpu().numpy(),
+                           piped.logw_c[b, h, :kg].cpu().double().numpy(),
+                           bits(piped.K_c[b, h, :kg]), bits(piped.V_c[b, h, :kg]),
+                           bits(Ku), bits(Vu), cap)
 
 
 def test_evict_from_page_locked_host_memory_matches_device(E):
@@ -594,7 +651,8 @@ def test_append_then_reevict_then_decode_matches_oracle(E):
 # ------------------------------------------------------- systematic design
 @pytest.mark.parametrize("B,H,N,budget,dist", [(2, 3, 1000, 100, "lognormal"),
                                                (1, 4, 20000, 2000, "pareto"),
-                                               (2, 2, 32768, 3277, "lognormal")])
+                                               (2, 2, 32768, 3277, "lognormal"),
+                                               (1, 2, 70001, 7000, "lognormal")])
 def test_systematic_select_matches_oracle(E, B, H, N, budget, dist):
     g = torch.Generator().manual_seed(N + budget)
     if dist == "lognormal":
