@@ -194,7 +194,9 @@ ebd_status ebd_evict(const ebd_design* design, ebd_dtype dtype, const void* K, c
  *
  * ebd_gather: copies rows K[idx_c[p]], V[idx_c[p]] to K_c[p], V_c[p] for
  * p < min(n_kept, cap) of every unit (16-byte loads; d * elem must be a
- * multiple of 16 bytes and the four tensors 16-byte aligned).
+ * multiple of 16 bytes and the four tensors 16-byte aligned).  A row whose
+ * index lies outside [0, n_ctx) is skipped (its K_c/V_c row is left as it
+ * was), so a corrupt index list cannot make the copy read out of bounds.
  * The scores of ebd_select and K, V of ebd_gather may be page-locked host
  * memory, as for ebd_evict.
  */

@@ -1248,11 +1248,16 @@ __global__ void __launch_bounds__(kGatherThreads) gather_rows_kernel(
 #pragma unroll
     for (int u = 0; u < kGatherUnroll; ++u) {
       const long long it = it0 + u * stride;
-      ok[u] = it < items;
-      if (ok[u]) {
+      const bool live = it < items;
+      ok[u] = false;
+      if (live) {
         const int p = (int)(it / cpr);
         const int ch = (int)(it - (long long)p * cpr);
-        const size_t src = src_base + (size_t)idx[p] * cpr + ch;
+        const int r = idx[p];
+        // a row whose index lies outside the context is read from row 0 and
+        // not stored: the copy never reads out of bounds
+        ok[u] = (unsigned)r < (unsigned)n_ctx;
+        const size_t src = src_base + (size_t)(ok[u] ? r : 0) * cpr + ch;
         dst[u] = dst_base + (size_t)p * cpr + ch;
         kv[u] = __ldg(K + src);
         vv[u] = __ldg(V + src);

@@ -30,7 +30,8 @@ ebd_status launch_select(const ebd_design* d, const float* scores, const int32_t
                          int cap, int32_t* dev_status, cudaStream_t stream);
 
 // E4b for every unit (evict.cu): rows K[idx_c[p]], V[idx_c[p]] (row stride
-// d->n_ctx) to K_c[p], V_c[p] for p < min(n_kept, cap).
+// d->n_ctx) to K_c[p], V_c[p] for p < min(n_kept, cap); rows whose index lies
+// outside [0, n_ctx) are skipped.
 ebd_status launch_gather(const ebd_design* d, ebd_dtype dtype, const void* K, const void* V,
                          const int32_t* idx_c, const int32_t* n_kept, int cap, void* K_c,
                          void* V_c, cudaStream_t s);

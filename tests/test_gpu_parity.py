@@ -455,6 +455,40 @@ def test_decode_matches_oracle_on_synthetic_cache(E, B, H, G, d, cap, dtype, pat
                                  out[4][b, sl], exact)
 
 
+def test_gather_skips_rows_with_out_of_range_indices(E):
+    """ebd_gather copies exactly the rows whose index lies in [0, n_ctx): a row
+    named by a negative or too large index is left as it was (a corrupt index
+    list cannot make the copy read out of bounds), every other row is copied
+    bit for bit."""
+    B, H, N, d, cap = 2, 3, 1000, 128, 64
+    g = torch.Generator().manual_seed(5)
+    K = torch.randn((B, H, N, d), generator=g).to(torch.bfloat16).to(DEV)
+    V = torch.randn((B, H, N, d), generator=g).to(torch.bfloat16).to(DEV)
+    des = _design(E, B, H, 1, d, N, 0, 1, 10, 60)
+    cc = E.alloc_compact(B, H, cap, d, torch.bfloat16, DEV)
+    idx = torch.randint(0, N, (B, H, cap), generator=g).int()
+    bad = torch.rand((B, H, cap), generator=g) < 0.25
+    idx[bad & (torch.rand((B, H, cap), generator=g) < 0.5)] = -3
+    idx[bad & (idx >= 0)] = N + 17
+    cc.idx_c.copy_(idx)
+    n = torch.tensor([[cap, cap - 5, 0], [1, 37, cap]], dtype=torch.int32)
+    cc.n_kept.copy_(n)
+    cc.K_c.fill_(7.0)
+    cc.V_c.fill_(-7.0)
+    E.ebd_gather(des, K, V, cc)
+    torch.cuda.synchronize()
+    Kc, Vc, Kh, Vh = cc.K_c.cpu(), cc.V_c.cpu(), K.cpu(), V.cpu()
+    for b in range(B):
+        for h in range(H):
+            for p in range(cap):
+                r = int(idx[b, h, p])
+                if p < int(n[b, h]) and 0 <= r < N:
+                    assert torch.equal(Kc[b, h, p], Kh[b, h, r])
+                    assert torch.equal(Vc[b, h, p], Vh[b, h, r])
+                else:
+                    assert bool((Kc[b, h, p] == 7.0).all()) and bool((Vc[b, h, p] == -7.0).all())
+
+
 def test_decode_workspace_needs_no_clearing_and_is_deterministic(E):
     """The decode writes every partial record before its merge reads it: a
     workspace full of garbage gives the same bits as a fresh one, call after
