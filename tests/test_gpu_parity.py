@@ -455,6 +455,55 @@ def test_decode_matches_oracle_on_synthetic_cache(E, B, H, G, d, cap, dtype, pat
                                  out[4][b, sl], exact)
 
 
+def _decode_outputs(E, args, B, Hq, d):
+    y = torch.empty((B, Hq, d), dtype=torch.float32, device=DEV)
+    lse, var, bt, r = (torch.empty((B, Hq), dtype=torch.float32, device=DEV) for _ in range(4))
+    E.ebd_certified_decode(*args, y, lse, var, bt, r)
+    torch.cuda.synchronize()
+    return y, lse, var, bt, r
+
+
+@pytest.mark.parametrize("design", ["full_budget", "top_k_only"])
+def test_certain_designs_give_exact_attention_and_zero_certificate(E, design):
+    """Degenerate designs the method fixes exactly, end to end through both
+    calls.  A budget covering the context keeps every token with pi = 1: Eq. 3
+    is then Eq. 1 (full attention) and Theorem 2's (1 - pi) factor makes V_hat,
+    b_t and r_t exactly zero.  A budget of just the certainty set (4 sinks, 32
+    recent, the top slice; no Poisson tail) gives exact attention over the kept
+    rows, again with a zero certificate."""
+    B, H, G, d, N, k_head = 2, 2, 4, 128, 1000, 40
+    budget = N if design == "full_budget" else 4 + 32 + k_head
+    cap = 1008
+    g = torch.Generator().manual_seed(31)
+    K = torch.randn((B, H, N, d), generator=g).to(torch.bfloat16)
+    V = torch.randn((B, H, N, d), generator=g).to(torch.bfloat16)
+    Q = torch.randn((B, H * G, d), generator=g).to(torch.bfloat16)
+    s = torch.exp(1.5 * torch.randn((B, H, N), generator=g))
+    des = _design(E, B, H, G, d, N, 0, 9, k_head, budget)
+    cc = E.alloc_compact(B, H, cap, d, torch.bfloat16, DEV)
+    E.ebd_evict(des, K.to(DEV), V.to(DEV), s.to(DEV), None, cc)
+    y, lse, var, bt, r = _decode_outputs(E, [Q.to(DEV), cc.K_c, cc.V_c, cc.logw_c, cc.n_kept],
+                                         B, H * G, d)
+    assert cc.dev_status.item() == 0
+    n = cc.n_kept.cpu()
+    assert bool((n == budget).all())
+    assert bool((cc.logw_c.cpu()[..., :budget] == 0).all())
+    for t in (var, bt, r):
+        assert bool((t == 0).all())
+    Kd, Vd, Qd = K.double(), V.double(), Q.double()
+    for b in range(B):
+        for h in range(H):
+            rows = cc.idx_c[b, h, :budget].long().cpu()
+            if design == "full_budget":
+                assert torch.equal(rows, torch.arange(N))
+            q = Qd[b, h * G:(h + 1) * G]
+            a = torch.softmax(q @ Kd[b, h, rows].T / math.sqrt(d), dim=-1)
+            ref = a @ Vd[b, h, rows]
+            got = y[b, h * G:(h + 1) * G].double().cpu()
+            scale = ref.abs().max(dim=-1, keepdim=True).values
+            assert bool(((got - ref).abs() <= 2e-3 * scale).all())
+
+
 def test_gather_skips_rows_with_out_of_range_indices(E):
     """ebd_gather copies exactly the rows whose index lies in [0, n_ctx): a row
     named by a negative or too large index is left as it was (a corrupt index
