@@ -73,6 +73,9 @@ def parse_args():
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--batch", type=int, default=0,
                    help="override the workload's batch (smaller cases for profiling)")
+    p.add_argument("--layers", type=int, default=0,
+                   help="override the workload's layer count (a smaller case of the same "
+                        "kernels, e.g. for profiling)")
     p.add_argument("--sweep", action="store_true",
                    help="instead of the step: the batch x context x budget sweep on the 28/4 "
                         "GQA shape, one JSON line per point (decode GB/s and roofline "
@@ -88,7 +91,11 @@ def parse_args():
 
 def workload_of(args) -> Workload:
     w = WORKLOADS[args.workload]
-    return w.with_(batch=args.batch) if args.batch > 0 else w
+    if args.batch > 0:
+        w = w.with_(batch=args.batch)
+    if args.layers > 0:
+        w = w.with_(n_layers=args.layers)
+    return w
 
 
 def dist_setup(args):
@@ -702,7 +709,10 @@ def run_ours(args, world, rank, local):
             v["gbs"] = v["alg_bytes_per_launch"] / (v["ms_per_launch"] * 1e-3) / 1e9
     dom = max(kern, key=lambda k: kern[k]["ms_per_launch"])
     kname = {"select": "evict_select_smem_kernel", "gather": "gather_rows_kernel",
-             "decode": "decode_mma_kernel + decode_merge_kernel",
+             "decode": ("certified decode: decode_mma_kernel + decode_merge_kernel (split-K), "
+                        "decode_cluster_kernel (few units), or decode_generic_kernel + "
+                        "decode_reduce_kernel (float32 or ragged capacity), as the request "
+                        "selects"),
              "score": "score_lse_tc_kernel + score_col_tc_kernel"}[dom]
     if dom == "score":
         # dense bf16 contraction on tcgen05: measured cuBLAS bf16 burst peak
