@@ -125,9 +125,21 @@ def max_over_ranks(x: float, world: int, device: str = "cuda") -> float:
     return float(t.item())
 
 
+def sum_over_ranks(x: float, world: int, device: str = "cuda") -> float:
+    """Every rank's value, all-reduced with SUM (bytes of shards that differ a
+    little in their kept rows)."""
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
 def whole_job_rate(units_per_rank: float, world: int, max_seconds: float) -> float:
-    """Weak scaling: every rank processes the same replica of the workload, so
-    the job processes world * units in the slowest rank's time."""
+    """Weak scaling: every rank processes a shard of the same size (its own B
+    batch rows of the workload's shape), so the job processes world * units in
+    the slowest rank's time."""
     return world * units_per_rank / max_seconds
 
 
@@ -640,6 +652,11 @@ def run_reference(args, world, rank):
 
 def run_ours(args, world, rank, local):
     w = workload_of(args)
+    if rank > 0:
+        # rank r holds its own shard of units: batch rows r B .. (r + 1) B - 1 of
+        # a world x B batch, drawn from their own seeds (rank 0 is the
+        # single-GPU workload itself)
+        w = w.with_(seed=w.seed + 7919 * rank, philox_seed=w.philox_seed + rank)
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     hbm_peak, peak_kind, peaks = measured_peaks()
@@ -689,7 +706,8 @@ def run_ours(args, world, rank, local):
 
     L = w.n_layers
     dbytes = decode_bytes(w, n_kept)
-    value = whole_job_rate(dbytes, world, ph_ms["decode"] * 1e-3) / 1e9
+    dbytes_mean = sum_over_ranks(dbytes, world) / world  # the shards' kept rows differ
+    value = whole_job_rate(dbytes_mean, world, ph_ms["decode"] * 1e-3) / 1e9
     evict_mtok = whole_job_rate(w.batch * w.n_ctx * L, world, ph_ms["evict"] * 1e-3) / 1e6
     # the eviction kernels run back to back, each phase alone (no overlap)
     serial_ms = sum(ph_ms[p] for p in path.kernel_phases)
@@ -732,7 +750,7 @@ def run_ours(args, world, rank, local):
         def e2e_line(in_place):
             ms, h2d, d2h = e2e_run(path, args.steps, in_place, n_kept)
             ms = max_over_ranks(ms, world)
-            return {"value": whole_job_rate(dbytes, world, ms * 1e-3) / 1e9, "unit": "GB/s",
+            return {"value": whole_job_rate(dbytes_mean, world, ms * 1e-3) / 1e9, "unit": "GB/s",
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms}
         e2e_copy = e2e_line(False)
         e2e_copy["inputs"] = ("K, V, Q and the " + ("observation queries" if path.scored else
