@@ -262,11 +262,15 @@ int cluster_decode_size(int units, int cap) {
   if (units < 1 || 2 * units > sms) return 0;
   int C = 2;
   while (C < 8 && 2 * C * units <= sms) C *= 2;
-  // measured: the on-chip combine pays off when the clusters cover most SMs
-  // and every CTA has a few tiles to stream (at least 8 at capacity);
-  // otherwise the split-K kernels over every SM are faster
-  if (4 * units * C < 3 * sms) return 0;
-  if ((cap / kMmaTile) / C < 8) return 0;
+  // measured: the on-chip combine pays off when every CTA has a few tiles to
+  // stream (at least 8 at capacity) and either the clusters cover most SMs or,
+  // with fewer CTAs, each CTA's share stays within what one SM streams quickly
+  // (at most 160 tiles: on 4 units the single launch beats the split-K pair by
+  // up to 20% there, and loses beyond ~250 tiles); otherwise the split-K
+  // kernels over every SM are faster
+  const int per_cta = (cap / kMmaTile) / C;
+  if (per_cta < 8) return 0;
+  if (4 * units * C < 3 * sms && per_cta > 160) return 0;
   return C;
 }
 
