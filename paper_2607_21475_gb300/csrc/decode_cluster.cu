@@ -1,6 +1,7 @@
-// Certified decode on thread-block clusters, for requests with few units (at
-// most half as many (batch row, KV head) units as SMs): one cluster of C = 2,
-// 4 or 8 CTAs per unit, C the largest that keeps units * C <= SMs.
+// Certified decode on thread-block clusters, for requests with at most one
+// (batch row, KV head) unit per SM: one cluster of C = 1, 2, 4 or 8 CTAs per
+// unit, C the largest that keeps units * C <= SMs (C = 1: one CTA holds the
+// whole unit and combines it alone).
 //
 // CTA r of a unit's cluster takes tiles [r T / C, (r + 1) T / C) of the unit's
 // T active 16-token tiles and splits them into eight contiguous ranges, one
@@ -259,8 +260,8 @@ static size_t cluster_smem(int D, int S, int C, int G) {
 
 int cluster_decode_size(int units, int cap) {
   const int sms = sm_count();
-  if (units < 1 || 2 * units > sms) return 0;
-  int C = 2;
+  if (units < 1 || units > sms) return 0;
+  int C = 1;  // one CTA per unit (no partner CTAs) when only one fits per SM
   while (C < 8 && 2 * C * units <= sms) C *= 2;
   // measured: the on-chip combine pays off when every CTA has a few tiles to
   // stream (at least 8 at capacity) and either the clusters cover most SMs or,

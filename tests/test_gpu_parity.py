@@ -413,9 +413,12 @@ DECODE_CASES = [
     # cluster kernel (units * C covering most SMs, long per-CTA ranges)
     (16, 4, 7, 128, 1600, torch.bfloat16, "edges"),   # 64 units, clusters of 2, empty units
     (8, 8, 8, 64, 1600, torch.bfloat16, "random"),    # head_dim 64, G = 8
-    # split-K with more units than half the SMs
+    # one CTA per unit (no partner CTAs) for more units than half the SMs
     (8, 12, 4, 128, 256, torch.bfloat16, "edges"),    # 96 units
     (10, 10, 8, 64, 160, torch.bfloat16, "random"),   # 100 units, head_dim 64
+    # split-K with more units than SMs
+    (20, 10, 4, 128, 256, torch.bfloat16, "edges"),   # 200 units
+    (16, 12, 8, 64, 160, torch.bfloat16, "random"),   # 192 units, head_dim 64, G = 8
 ]
 
 
