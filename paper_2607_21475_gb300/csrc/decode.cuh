@@ -74,9 +74,9 @@ ebd_status launch_fast_decode(ebd_dtype dtype, int head_dim, const DecodePlan& p
                               const DecodeArgs& a, const ReduceArgs& r, int units, void* ws,
                               cudaStream_t stream);
 
-// Cluster path (decode_cluster.cu) for requests with at most as many units
-// as SMs: CTAs per unit (0 when the path does not apply), and the launch (same
-// arguments as the tensor-core path; no workspace).
+// Cluster path (decode_cluster.cu): CTAs per unit (0 when the path does not
+// apply), and the launch (same arguments as the tensor-core path; no
+// workspace).
 int cluster_decode_size(int units, int cap);
 ebd_status launch_cluster_decode(int head_dim, const DecodeArgs& d, const ReduceArgs& r,
                                  int units, cudaStream_t stream);

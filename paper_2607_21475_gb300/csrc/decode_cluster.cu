@@ -1,7 +1,7 @@
-// Certified decode on thread-block clusters, for requests with at most one
-// (batch row, KV head) unit per SM: one cluster of C = 1, 2, 4 or 8 CTAs per
-// unit, C the largest that keeps units * C <= SMs (C = 1: one CTA holds the
-// whole unit and combines it alone).
+// Certified decode on thread-block clusters: one cluster of C = 1, 2, 4 or 8
+// CTAs per (batch row, KV head) unit, C the largest that keeps units * C <=
+// SMs (C = 1: one CTA holds the whole unit and combines it alone; with more
+// units than SMs those CTAs run in waves).
 //
 // CTA r of a unit's cluster takes tiles [r T / C, (r + 1) T / C) of the unit's
 // T active 16-token tiles and splits them into eight contiguous ranges, one
@@ -260,7 +260,16 @@ static size_t cluster_smem(int D, int S, int C, int G) {
 
 int cluster_decode_size(int units, int cap) {
   const int sms = sm_count();
-  if (units < 1 || units > sms) return 0;
+  if (units < 1) return 0;
+  if (units > sms) {
+    // more units than SMs: still one CTA per unit, the later ones starting as
+    // the first finish (the block scheduler hands them to the SMs that are
+    // done first); measured at 256 units faster than the split-K pair while a
+    // unit holds at most 512 tiles (dialogue 32k: 84.4 -> 82.5 us), slower
+    // beyond (wave quantisation)
+    const int tiles = cap / kMmaTile;
+    return tiles >= 8 && tiles <= 512 ? 1 : 0;
+  }
   int C = 1;  // one CTA per unit (no partner CTAs) when only one fits per SM
   while (C < 8 && 2 * C * units <= sms) C *= 2;
   // measured: the on-chip combine pays off when every CTA has a few tiles to
