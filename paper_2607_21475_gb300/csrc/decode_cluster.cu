@@ -264,10 +264,14 @@ int cluster_decode_size(int units, int cap) {
   if (units > sms) {
     // more units than SMs: still one CTA per unit, the later ones starting as
     // the first finish (the block scheduler hands them to the SMs that are
-    // done first); measured at 256 units faster than the split-K pair while a
-    // unit holds at most 512 tiles (dialogue 32k: 84.4 -> 82.5 us), slower
-    // beyond (wave quantisation)
+    // done first).  Measured on the 32k dialogue shape against the split-K
+    // pair: faster when the waves are at least 80% full (256 units, 84%:
+    // 83.3 -> 81.9 us; 288 units, 95%: 90.6 -> 86.2 us), much slower when the
+    // last wave is thin (160 units: 62.0 -> 79.5 us), and slower for units of
+    // more than 512 tiles (the quantisation of long waves)
     const int tiles = cap / kMmaTile;
+    const long long waves = (units + sms - 1) / sms;
+    if (5LL * units < 4LL * waves * sms) return 0;
     return tiles >= 8 && tiles <= 512 ? 1 : 0;
   }
   int C = 1;  // one CTA per unit (no partner CTAs) when only one fits per SM

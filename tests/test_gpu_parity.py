@@ -416,10 +416,11 @@ DECODE_CASES = [
     # one CTA per unit (no partner CTAs) for more units than half the SMs
     (8, 12, 4, 128, 256, torch.bfloat16, "edges"),    # 96 units
     (10, 10, 8, 64, 160, torch.bfloat16, "random"),   # 100 units, head_dim 64
-    # one CTA per unit, in waves, for more units than SMs
-    (20, 10, 4, 128, 256, torch.bfloat16, "edges"),   # 200 units
-    (16, 12, 8, 64, 160, torch.bfloat16, "random"),   # 192 units, head_dim 64, G = 8
-    # split-K with more units than SMs (units too short or too long for waves)
+    # one CTA per unit, in waves at least 80% full, for more units than SMs
+    (32, 8, 4, 128, 256, torch.bfloat16, "edges"),    # 256 units
+    (24, 12, 8, 64, 160, torch.bfloat16, "random"),   # 288 units, head_dim 64, G = 8
+    # split-K with more units than SMs (thin last wave, units too short or long)
+    (20, 10, 4, 128, 256, torch.bfloat16, "edges"),   # 200 units: a 66%-full last wave
     (20, 10, 4, 128, 96, torch.bfloat16, "edges"),    # 200 units of 6 tiles
     (4, 40, 4, 128, 8256, torch.bfloat16, "random"),  # 160 units of 516 tiles
 ]
