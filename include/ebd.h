@@ -223,6 +223,10 @@ ebd_status ebd_gather(const ebd_design* design, ebd_dtype dtype, const void* K, 
  * An empty unit (n_kept = 0) gives y = 0, lse = -inf and a zero certificate.
  * Needs workspace of ebd_decode_workspace_bytes(...) bytes for the split-K
  * partial records.  Supports d in {64, 128} and 1 <= G <= 8.
+ * Results are reproducible bit for bit: a request always takes the same
+ * kernels and the same summation order on a given GPU (the choice depends on
+ * the request's shape and the GPU's SM count, so GPUs with another SM count
+ * may differ in the last bits).
  */
 size_t ebd_decode_workspace_bytes(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads,
                                   int32_t group, int32_t head_dim, int32_t capacity);
