@@ -105,6 +105,18 @@ const char* ebd_status_string(ebd_status status);
 int32_t ebd_abi_version(void);
 
 /*
+ * Failure-path check (no counterpart in the paper, which specifies no
+ * runtime).  Launches one warp that waits, with the same bounded wait the
+ * tensor-core pipelines use, on an mbarrier phase that nothing completes: the
+ * wait gives up after ~2 s, the kernel raises EBD_DEV_TIMEOUT in *dev_status
+ * (device int32, required; bits are OR-ed in) and returns, and the CUDA
+ * context stays usable.  Lets a caller confirm that a stalled pipeline
+ * reports a status instead of hanging the GPU.  Asynchronous on `stream`;
+ * EBD_ERR_INVALID for a null dev_status.
+ */
+ebd_status ebd_check_stalled_wait(int32_t* dev_status, void* stream);
+
+/*
  * Philox4x32-10 words used by the Poisson draw (Section 3.3: independent
  * Bernoulli(pi_i) retention on the tail).  For every unit (b, kvh) and token
  * i < N writes x0[b,kvh,i] (device uint32 [B,Hkv,N]) = output word i % 4 of

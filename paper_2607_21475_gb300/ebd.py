@@ -29,7 +29,8 @@ __all__ = [
     "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
     "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
     "ebd_certified_decode_static", "ebd_certificate_update", "ebd_append", "ebd_reevict",
-    "ebd_gather_queries", "ebd_variance_contributions", "ebd_block_scores", "design_for",
+    "ebd_gather_queries", "ebd_variance_contributions", "ebd_block_scores",
+    "ebd_check_stalled_wait", "design_for",
     "CompactCache",
     "alloc_compact", "ABI_FUNCTIONS",
 ]
@@ -47,6 +48,7 @@ ABI_FUNCTIONS = (
     "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
     "ebd_certified_decode_static", "ebd_certificate_update", "ebd_append", "ebd_reevict",
     "ebd_gather_queries", "ebd_variance_contributions", "ebd_block_scores",
+    "ebd_check_stalled_wait",
 )
 
 
@@ -127,6 +129,7 @@ def lib():
                                                           c_void_p, c_void_p]),
             "ebd_block_scores": (ctypes.c_int, [i32, i32, i32, c_void_p, c_void_p, c_void_p, i32,
                                                 i32, i32, c_void_p, c_void_p]),
+            "ebd_check_stalled_wait": (ctypes.c_int, [c_void_p, c_void_p]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -192,6 +195,14 @@ def ebd_status_string(code: int) -> str:
 
 def ebd_abi_version() -> int:
     return int(lib().ebd_abi_version())
+
+
+def ebd_check_stalled_wait(dev_status: torch.Tensor, stream=None) -> torch.Tensor:
+    """Run the bounded-wait failure path: ~2 s later EBD_DEV_TIMEOUT is OR-ed
+    into dev_status (int32 CUDA tensor [1]) and the context stays usable."""
+    _check("ebd_check_stalled_wait", lib().ebd_check_stalled_wait(
+        _ptr(dev_status, torch.int32, (1,), "dev_status"), _stream(stream)))
+    return dev_status
 
 
 def ebd_philox_uniforms(seed: int, layer: int, x0: torch.Tensor, stream=None):
