@@ -344,8 +344,6 @@ class DecodeResult:
     b_bound: np.ndarray  # [G]     one-pass upper bound on the range term
     r_exact: np.ndarray  # [G]     radius with b_exact
     r_bound: np.ndarray  # [G]     radius with b_bound
-    var_scale: np.ndarray  # [G]   sum (1-pi) p^2 (||v||^2 + ||y_hat||^2): the uncentred
-    #                               moment a one-pass evaluation of V_hat cancels against
 
 
 def certificate_radius(var, b, y_norm, delta: float, eps0: float):
@@ -381,9 +379,9 @@ def hajek_decode(q, K_c, V_c, logw_c, delta: float = 0.1, eps0: float = 1e-9) ->
     if n == 0:
         z = np.zeros(G)
         return DecodeResult(np.zeros((G, d)), np.full(G, -np.inf), z, z.copy(), z.copy(),
-                            z.copy(), z.copy(), z.copy())
+                            z.copy(), z.copy())
     one_minus_pi = -np.expm1(-logw)
-    ys, lses, vs, bes, bbs, scs = [], [], [], [], [], []
+    ys, lses, vs, bes, bbs = [], [], [], [], []
     for h in range(G):
         logits = (K_c @ q[h]) / math.sqrt(d) + logw     # log(a_i / pi_i)
         M = logits.max()
@@ -397,7 +395,6 @@ def hajek_decode(q, K_c, V_c, logw_c, delta: float = 0.1, eps0: float = 1e-9) ->
         b_exact = t.max()
         s = np.sqrt(one_minus_pi) * p
         b_bound = np.max(s * np.linalg.norm(V_c, axis=1)) + np.linalg.norm(y) * np.max(s)
-        scs.append(np.sum(one_minus_pi * p * p * (np.sum(V_c * V_c, axis=1) + y @ y)))
         ys.append(y)
         lses.append(M + math.log(l))
         vs.append(var)
@@ -410,7 +407,7 @@ def hajek_decode(q, K_c, V_c, logw_c, delta: float = 0.1, eps0: float = 1e-9) ->
     yn = np.linalg.norm(y, axis=1)
     return DecodeResult(y, np.array(lses), var, b_exact, b_bound,
                         certificate_radius(var, b_exact, yn, delta, eps0),
-                        certificate_radius(var, b_bound, yn, delta, eps0), np.array(scs))
+                        certificate_radius(var, b_bound, yn, delta, eps0))
 
 
 # ---------------------------------------------------------------------------

@@ -7,12 +7,13 @@
 //   l  = sum w_i                    w_i = exp(q.k_i/sqrt(d) + log(1/pi_i) - M)
 //   o  = sum w_i v_i                (Hajek numerator, Eq. 3)
 //   U  = sum u_i,  u_i = (1 - pi_i) w_i^2   (Theorem 2 weights)
-//   A1 = sum u_i v_i,  A2 = sum u_i ||v_i||^2
+//   A1 = sum u_i v_i,  A2 = sum u_i ||v_i - c||^2  (c: the unit's centring row)
 //   cmax = max sqrt(u_i) ||v_i||,  umax = max sqrt(u_i)   (range-term bound)
 // A maximum increase by D rescales the w-terms by e^-D and the u-terms by
 // e^-2D.  The reduce kernel merges the splits the same way and finishes
 //   y_hat = o / l,   lse = M + log l  (= log N_hat),
-//   V_hat = (A2 - 2 y_hat.A1 + ||y_hat||^2 U) / l^2 = sum u_i ||v_i - y_hat||^2 / l^2,
+//   V_hat = (A2 - 2 (y_hat - c).(A1 - U c) + ||y_hat - c||^2 U) / l^2
+//         = sum u_i ||v_i - y_hat||^2 / l^2,
 //   b_t   = (cmax + ||y_hat|| umax) / l   (bound; >= the definition),
 //   r_t   = (sqrt(2 V_hat ln(1/delta)) + b_t ln(1/delta)) / (||y_hat|| + eps0).
 // The exact range term, max_i sqrt(u_i) ||v_i - y_hat|| / l, needs y_hat and is
@@ -49,6 +50,13 @@ __global__ void __launch_bounds__(kGenThreads) decode_generic_kernel(DecodeArgs 
   const T* Kc = (const T*)a.Kc + (size_t)unit * a.cap * D;
   const T* Vc = (const T*)a.Vc + (size_t)unit * a.cap * D;
   const float* lw = a.logw + (size_t)unit * a.cap;
+  // the unit's centring row (zeros for an empty unit): A2 is taken about it
+  float c[E];
+  {
+    const int cr = centre_row(max(n, 0));
+#pragma unroll
+    for (int j = 0; j < E; ++j) c[j] = cr < 0 ? 0.f : to_f32(Vc[(size_t)cr * D + lane + 32 * j]);
+  }
 
   float q[GM][E], o[GM][E], a1[GM][E];
   float M[GM], l[GM], U[GM], A2[GM], cmax[GM], umax[GM];
@@ -73,10 +81,15 @@ __global__ void __launch_bounds__(kGenThreads) decode_generic_kernel(DecodeArgs 
     const float lwt = lw[t];
     const float omp = -expm1f(-lwt);  // 1 - pi
     const float sq = sqrtf(omp);
-    float vn2 = 0.f;
+    float vn2 = 0.f, vc2 = 0.f;
 #pragma unroll
-    for (int j = 0; j < E; ++j) vn2 = fmaf(v[j], v[j], vn2);
+    for (int j = 0; j < E; ++j) {
+      vn2 = fmaf(v[j], v[j], vn2);
+      const float dv = v[j] - c[j];
+      vc2 = fmaf(dv, dv, vc2);
+    }
     vn2 = warp_sum(vn2);
+    vc2 = warp_sum(vc2);
     const float vn = sqrtf(vn2);
 #pragma unroll
     for (int g = 0; g < GM; ++g) {
@@ -104,7 +117,7 @@ __global__ void __launch_bounds__(kGenThreads) decode_generic_kernel(DecodeArgs 
       const float su = sq * w;
       l[g] += w;
       U[g] += u;
-      A2[g] = fmaf(u, vn2, A2[g]);
+      A2[g] = fmaf(u, vc2, A2[g]);
       cmax[g] = fmaxf(cmax[g], su * vn);
       umax[g] = fmaxf(umax[g], su);
 #pragma unroll
@@ -164,7 +177,7 @@ __global__ void __launch_bounds__(kGenThreads) decode_generic_kernel(DecodeArgs 
 // u*splits .. u*splits + splits - 1.
 constexpr int kReduceWarps = 4;
 
-template <int D>
+template <typename T, int D>
 __global__ void __launch_bounds__(kReduceWarps * 32) decode_reduce_kernel(ReduceArgs a,
                                                                           int n_heads) {
   constexpr int REC = rec_floats(D);
@@ -243,19 +256,13 @@ __global__ void __launch_bounds__(kReduceWarps * 32) decode_reduce_kernel(Reduce
   A2 = warp_sum(A2);
   cmax = warp_max(cmax);
   umax = warp_max(umax);
-  float yy = 0.f, ya = 0.f;
+  float c[PER], yv[PER], ynorm, var;
+  load_centre<T, D, PER>(static_cast<const T*>(a.Vc), unit, a.cap,
+                         min(max(a.n_kept[unit], 0), a.cap), lane, c);
+  finish_head<PER>(o, a1, c, l, U, A2, yv, ynorm, var);
 #pragma unroll
-  for (int e = 0; e < PER; ++e) {
-    const float yv = o[e] / l;
-    a.y[(size_t)hq * D + PER * lane + e] = yv;
-    yy = fmaf(yv, yv, yy);
-    ya = fmaf(yv, a1[e], ya);
-  }
-  yy = warp_sum(yy);
-  ya = warp_sum(ya);
+  for (int e = 0; e < PER; ++e) a.y[(size_t)hq * D + PER * lane + e] = yv[e];
   if (lane == 0) {
-    const float ynorm = sqrtf(yy);
-    const float var = fmaxf(0.f, (A2 - 2.f * ya + yy * U) / (l * l));
     a.lse[hq] = Mx + logf(l);
     a.var[hq] = var;
     if (a.exact) {
@@ -472,6 +479,9 @@ extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32
 
   ReduceArgs r;
   r.part = (const float*)workspace;
+  r.Vc = V_c;
+  r.n_kept = n_kept;
+  r.cap = capacity;
   r.splits = plan.splits;
   r.group = group;
   r.y = y;
@@ -490,10 +500,14 @@ extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32
     st = dispatch_generic(false, dtype, head_dim, a, (int)units, s);
     if (st == EBD_OK) {
       const int rblocks = (n_heads + kReduceWarps - 1) / kReduceWarps;
-      if (head_dim == 128)
-        decode_reduce_kernel<128><<<rblocks, kReduceWarps * 32, 0, s>>>(r, n_heads);
-      else
-        decode_reduce_kernel<64><<<rblocks, kReduceWarps * 32, 0, s>>>(r, n_heads);
+      const dim3 rg(rblocks), rb(kReduceWarps * 32);
+      if (dtype == EBD_F32) {
+        if (head_dim == 128) decode_reduce_kernel<float, 128><<<rg, rb, 0, s>>>(r, n_heads);
+        else decode_reduce_kernel<float, 64><<<rg, rb, 0, s>>>(r, n_heads);
+      } else {
+        if (head_dim == 128) decode_reduce_kernel<__nv_bfloat16, 128><<<rg, rb, 0, s>>>(r, n_heads);
+        else decode_reduce_kernel<__nv_bfloat16, 64><<<rg, rb, 0, s>>>(r, n_heads);
+      }
       st = launch_status();
     }
   }

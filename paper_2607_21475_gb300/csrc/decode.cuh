@@ -6,8 +6,56 @@
 #include <stdint.h>
 
 #include "../../include/ebd.h"
+#include "common.cuh"
 
 namespace ebd {
+
+// Centring row of a unit with n retained rows: the middle one, or -1 (c = 0)
+// for an empty unit.  Every partial record of a unit takes its second moment
+// A2 = sum u ||v - c||^2 about the same row c = V_c[centre_row(n)], and the
+// combine finishes
+//   V_hat l^2 = sum u ||v - y||^2 = A2 - 2 (y - c).(A1 - U c) + ||y - c||^2 U,
+// so no term carries the values' common mean (with A2 about the origin, a mean
+// of 16 on every channel makes each term ~256 times V_hat l^2 and float32
+// rounding of the sums shows in V_hat).  Any retained row serves: c only has
+// to lie within the spread of the values.
+__host__ __device__ constexpr int centre_row(int n) { return n > 0 ? (n - 1) / 2 : -1; }
+
+// Columns PER * lane .. + PER - 1 of the centring row of a unit (n retained
+// rows, cap rows per unit in Vc), as floats; zeros for an empty unit.
+template <typename T, int D, int PER>
+__device__ __forceinline__ void load_centre(const T* Vc, long long unit, int cap, int n, int lane,
+                                            float (&c)[PER]) {
+  const int cr = centre_row(n);
+  const T* row = Vc + ((size_t)unit * cap + (cr < 0 ? 0 : cr)) * D + PER * lane;
+#pragma unroll
+  for (int e = 0; e < PER; ++e) c[e] = cr < 0 ? 0.f : to_f32(row[e]);
+}
+
+// Finish one query head from its combined sums (Eq. 3, Theorem 2): y_hat =
+// o / l on this lane's PER columns, ||y_hat|| and
+//   V_hat = (A2 - 2 (y - c).(A1 - U c) + ||y - c||^2 U) / l^2
+// with A2 taken about the centring row c (every lane gets the warp's sums).
+template <int PER>
+__device__ __forceinline__ void finish_head(const float (&o)[PER], const float (&a1)[PER],
+                                            const float (&c)[PER], float l, float U, float A2,
+                                            float (&yv)[PER], float& ynorm, float& var) {
+  float yy = 0.f, ycyc = 0.f, yca = 0.f;
+#pragma unroll
+  for (int e = 0; e < PER; ++e) {
+    yv[e] = o[e] / l;
+    yy = fmaf(yv[e], yv[e], yy);
+    const float yc = yv[e] - c[e];
+    const float a1c = fmaf(-U, c[e], a1[e]);
+    ycyc = fmaf(yc, yc, ycyc);
+    yca = fmaf(yc, a1c, yca);
+  }
+  yy = warp_sum(yy);
+  ycyc = warp_sum(ycyc);
+  yca = warp_sum(yca);
+  ynorm = sqrtf(yy);
+  var = fmaxf(0.f, (A2 - 2.f * yca + ycyc * U) / (l * l));
+}
 
 // One partial record per (unit, split slot, query head of the group), floats:
 //   [M, l, U, A2, cmax, umax, pad, pad, o[0..D), A1[0..D)]
@@ -41,6 +89,9 @@ struct DecodeArgs {
 
 struct ReduceArgs {
   const float* part;         // CUDA-core path: [units, splits, G, rec_floats(D)]
+  const void* Vc;            // [units, cap, D]: the centring rows (CUDA-core path)
+  const int32_t* n_kept;     // [units]
+  int cap;
   int splits;                // records per unit
   int group;
   float* y;

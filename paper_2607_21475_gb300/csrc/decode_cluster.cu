@@ -13,7 +13,8 @@
 // shared memory; after one cluster barrier CTA 0 combines them and writes
 // y_hat, log N_hat, V_hat, b_t and r_t (Eq. 3, Theorem 2, Eq. 4).  One launch,
 // no workspace, no merge kernel.  Combination rule: w-terms (l, o, cmax,
-// umax) scale by e^(M_part - M), u-terms (U, A2, A1) by its square.
+// umax) scale by e^(M_part - M), u-terms (U, A2, A1) by its square; every
+// part takes A2 about the unit's centring row (decode.cuh).
 #include <cuda_runtime.h>
 #include <math.h>
 
@@ -111,7 +112,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
   const size_t row_base = (size_t)unit * a.cap;
 
   TileAcc<D> st;
-  tile_acc_begin<D>(st, a.Q, unit, G, lane);
+  tile_acc_begin<D>(st, a.Q, a.Vc, unit, G, a.cap, n_u, lane);
   int issued = 0;
   auto issue_next = [&]() {
     const int t = tb + issued;
@@ -179,19 +180,12 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
     }
     return;
   }
-  float yy = 0.f, ya = 0.f;
+  float c[PER], yv[PER], ynorm, var;
+  load_centre<__nv_bfloat16, D, PER>(a.Vc, unit, a.cap, n_u, lane, c);
+  finish_head<PER>(h.o, h.a1, c, h.l, h.U, h.A2, yv, ynorm, var);
 #pragma unroll
-  for (int e = 0; e < PER; ++e) {
-    const float yv = h.o[e] / h.l;
-    a.y[hq * D + PER * lane + e] = yv;
-    yy = fmaf(yv, yv, yy);
-    ya = fmaf(yv, h.a1[e], ya);
-  }
-  yy = warp_sum(yy);
-  ya = warp_sum(ya);
+  for (int e = 0; e < PER; ++e) a.y[hq * D + PER * lane + e] = yv[e];
   if (lane == 0) {
-    const float ynorm = sqrtf(yy);
-    const float var = fmaxf(0.f, (h.A2 - 2.f * ya + yy * h.U) / (h.l * h.l));
     a.lse[hq] = h.M + logf(h.l);
     a.var[hq] = var;
     if (a.exact) {

@@ -2,8 +2,9 @@
 //
 // Same quantities as the CUDA-core path (Eq. 3, Theorem 2, Eq. 4): per query
 // head an online softmax over logits q.k/sqrt(d) + log(1/pi) carrying
-// l = sum w, o = sum w v, U = sum u, A1 = sum u v, A2 = sum u ||v||^2 and the
-// range-bound maxima, with u = (1 - pi) w^2.
+// l = sum w, o = sum w v, U = sum u, A1 = sum u v, A2 = sum u ||v - c||^2
+// (c: the unit's centring row, decode.cuh) and the range-bound maxima, with
+// u = (1 - pi) w^2.
 //
 // Two kernels.  The decode kernel is a persistent grid (one CTA per SM) of 8
 // warps.  Every CTA first builds the prefix of active 16-token tiles per unit
@@ -74,6 +75,9 @@ struct FastArgs {
 struct MergeArgs {
   const int32_t* tile_off;   // [units + 1]
   const float* part;         // records of the decode kernel
+  const __nv_bfloat16* Vc;   // [units, cap, D]: the centring rows
+  const int32_t* n_kept;     // [units]
+  int cap;
   long long warps;           // warps of the decode grid
   int units;
   int group;
@@ -252,7 +256,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     seg_start = toff[u];
     seg_end = toff[u + 1];
     n_u = min(__ldg(a.n_kept + u), a.cap);
-    tile_acc_begin<D>(st, a.Q, u, G, lane);
+    tile_acc_begin<D>(st, a.Q, a.Vc, u, G, a.cap, n_u, lane);
   };
   auto flush_segment = [&]() {
     tile_acc_store<D>(st, a.part + (size_t)(u + gw) * G * REC, G, lane);
@@ -430,23 +434,15 @@ __global__ void __launch_bounds__(MW * 32) decode_merge_kernel(MergeArgs a) {
       a1[e] = fmaf(f2, sh_a[w][PER * lane + e], a1[e]);
     }
   }
-  float yy = 0.f, ya = 0.f;
-  float yv[PER];
-#pragma unroll
-  for (int e = 0; e < PER; ++e) {
-    yv[e] = o[e] / l;
-    yy = fmaf(yv[e], yv[e], yy);
-    ya = fmaf(yv[e], a1[e], ya);
-  }
+  float c[PER], yv[PER], ynorm, var;
+  load_centre<__nv_bfloat16, D, PER>(a.Vc, u, a.cap, min(max(__ldg(a.n_kept + u), 0), a.cap),
+                                     lane, c);
+  finish_head<PER>(o, a1, c, l, U, A2, yv, ynorm, var);
   if constexpr (PER == 4)
     *reinterpret_cast<float4*>(a.y + hq * D + 4 * lane) = make_float4(yv[0], yv[1], yv[2], yv[3]);
   else
     *reinterpret_cast<float2*>(a.y + hq * D + 2 * lane) = make_float2(yv[0], yv[1]);
-  yy = warp_sum(yy);
-  ya = warp_sum(ya);
   if (lane == 0) {
-    const float ynorm = sqrtf(yy);
-    const float var = fmaxf(0.f, (A2 - 2.f * ya + yy * U) / (l * l));
     a.lse[hq] = Mx + logf(l);
     a.var[hq] = var;
     if (a.exact) {
@@ -533,6 +529,9 @@ static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, con
   MergeArgs m;
   m.tile_off = tile_off;
   m.part = recs;
+  m.Vc = f.Vc;
+  m.n_kept = a.n_kept;
+  m.cap = a.cap;
   m.warps = (long long)plan.ctas * kMmaConsumers;
   m.units = units;
   m.group = a.group;

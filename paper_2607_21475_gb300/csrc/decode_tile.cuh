@@ -8,9 +8,13 @@
 //   w = 2^(S log2e/sqrt(d) + log2e log(1/pi) - M), u = (1 - pi) w^2
 //   P[16 x 16]  = [w (rows 0..7); u (rows 8..15)] as bf16 hi + bf16 lo parts
 //   acc[16 x d] += P_hi . V_tile + P_lo . V_tile   (rows 0..7: o, rows 8..15: A1)
-// plus l = sum w, U = sum u, A2 = sum u ||v||^2 and the range-bound maxima
-// cmax = max sqrt(u) ||v||, umax = max sqrt(u).  The hi/lo split keeps ~16
-// mantissa bits of the weights on bf16 tensor cores; ||v||^2 per token comes
+// plus l = sum w, U = sum u, A2 = sum u ||v - c||^2 and the range-bound
+// maxima cmax = max sqrt(u) ||v||, umax = max sqrt(u).  c is the unit's
+// centring row (centre_row in decode.cuh), so that the second moment does not
+// carry the values' common mean: the combine forms
+// V_hat l^2 = A2 - 2 (y - c).(A1 - U c) + ||y - c||^2 U, every term of the
+// size of the spread of v around y.  The hi/lo split keeps ~16 mantissa bits
+// of the weights on bf16 tensor cores; ||v||^2 and ||v - c||^2 per token come
 // from the same V fragments.  The running maximum M is updated lazily:
 // accumulators are rescaled only when a row's maximum grows by more than 2^8,
 // so weights stay below 2^8 and u below 2^16.
@@ -60,14 +64,30 @@ struct TileAcc {
   float acc[D / 8][4];
   float M2, l, U, A2, cmax, umax;  // M2: running maximum in log2 units
   uint32_t qa[D / 16][2];
+  // -c as bf16 pairs: channel 16 jp + lane/4 (low half), 16 jp + 8 + lane/4
+  // (high half) -- the channels of this lane's V fragments
+  uint32_t cneg[D / 16];
 };
 
-// Start a unit: its G query rows as mma A fragments (rows >= G are zero), and
-// empty sums.
+// Start a unit: its G query rows as mma A fragments (rows >= G are zero), its
+// centring row (Vc: the compact V cache, cap rows per unit; n_u: the unit's
+// retained rows), and empty sums.
 template <int D>
-__device__ __forceinline__ void tile_acc_begin(TileAcc<D>& t, const __nv_bfloat16* Q, int u,
-                                               int G, int lane) {
+__device__ __forceinline__ void tile_acc_begin(TileAcc<D>& t, const __nv_bfloat16* Q,
+                                               const __nv_bfloat16* Vc, int u, int G, int cap,
+                                               int n_u, int lane) {
   const int g = lane >> 2, q = lane & 3;
+  {
+    const int cr = centre_row(n_u);
+    const unsigned short* crow =
+        reinterpret_cast<const unsigned short*>(Vc + ((size_t)u * cap + (cr < 0 ? 0 : cr)) * D);
+#pragma unroll
+    for (int jp = 0; jp < D / 16; ++jp) {
+      const uint32_t lo = cr < 0 ? 0u : __ldg(crow + 16 * jp + g);
+      const uint32_t hi = cr < 0 ? 0u : __ldg(crow + 16 * jp + 8 + g);
+      t.cneg[jp] = (lo | (hi << 16)) ^ 0x80008000u;  // both halves negated
+    }
+  }
   const uint32_t* qrow =
       reinterpret_cast<const uint32_t*>(Q + ((size_t)u * G + (g < G ? g : 0)) * D);
 #pragma unroll
@@ -191,6 +211,7 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
   const uint32_t m01 = (tk[0] < n_valid ? 0x0000ffffu : 0u) | (tk[1] < n_valid ? 0xffff0000u : 0u);
   const uint32_t m23 = (tk[2] < n_valid ? 0x0000ffffu : 0u) | (tk[3] < n_valid ? 0xffff0000u : 0u);
   float2 vn01 = make_float2(0.f, 0.f), vn23 = make_float2(0.f, 0.f);
+  float2 vc01 = make_float2(0.f, 0.f), vc23 = make_float2(0.f, 0.f);
   {
     const int tok = ((lane >> 3) & 1) * 8 + (lane & 7);
     const int chunk_sel = lane >> 4;
@@ -211,6 +232,15 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
       const float2 f3 = make_float2(bf16_lo(v3), bf16_hi(v3));
       vn01 = __ffma2_rn(f0, f0, __ffma2_rn(f2, f2, vn01));
       vn23 = __ffma2_rn(f1, f1, __ffma2_rn(f3, f3, vn23));
+      // v - c: exact for bf16 v and c of similar magnitude (masked rows give
+      // -c, finite, and carry u = 0)
+      const float cl = bf16_lo(t.cneg[jp]), ch = bf16_hi(t.cneg[jp]);
+      const float2 e0 = __fadd2_rn(f0, make_float2(cl, cl));
+      const float2 e1 = __fadd2_rn(f1, make_float2(cl, cl));
+      const float2 e2 = __fadd2_rn(f2, make_float2(ch, ch));
+      const float2 e3 = __fadd2_rn(f3, make_float2(ch, ch));
+      vc01 = __ffma2_rn(e0, e0, __ffma2_rn(e2, e2, vc01));
+      vc23 = __ffma2_rn(e1, e1, __ffma2_rn(e3, e3, vc23));
       mma_bf16_16816(t.acc[2 * jp], h0, h1, h2, h3, v0, v1);
       mma_bf16_16816(t.acc[2 * jp], r0, r1, r2, r3, v0, v1);
       mma_bf16_16816(t.acc[2 * jp + 1], h0, h1, h2, h3, v2, v3);
@@ -220,19 +250,22 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
   // every lane's reads of this stage are done before it is refilled
   __syncwarp();
   float vn[4] = {vn01.x, vn01.y, vn23.x, vn23.y};
+  float vc[4] = {vc01.x, vc01.y, vc23.x, vc23.y};
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    vn[i] += __shfl_xor_sync(0xffffffffu, vn[i], 4);
-    vn[i] += __shfl_xor_sync(0xffffffffu, vn[i], 8);
-    vn[i] += __shfl_xor_sync(0xffffffffu, vn[i], 16);
-    t.A2 = fmaf(ut[i], vn[i], t.A2);
+#pragma unroll
+    for (int o = 4; o <= 16; o <<= 1) {
+      vn[i] += __shfl_xor_sync(0xffffffffu, vn[i], o);
+      vc[i] += __shfl_xor_sync(0xffffffffu, vc[i], o);
+    }
+    t.A2 = fmaf(ut[i], vc[i], t.A2);
     t.cmax = fmaxf(t.cmax, suv[i] * sqrtf(vn[i]));
   }
 }
 
 // Write the warp's state as partial records: head g = lane / 4 (g < G) at
-// rec + g * rec_floats(D): [M (natural log), l, U, A2, cmax, umax, -, -,
-// o[D], A1[D]].  The scalar sums are first completed over the four lanes of
+// rec + g * rec_floats(D): [M (natural log), l, U, A2 (about the unit's
+// centring row), cmax, umax, -, -, o[D], A1[D]].  The scalar sums are first completed over the four lanes of
 // a head.
 template <int D>
 __device__ __forceinline__ void tile_acc_store(TileAcc<D>& t, float* rec_base, int G, int lane) {

@@ -426,10 +426,19 @@ DECODE_CASES = [
 ]
 
 
-def _synthetic_cache(B, H, cap, d, dtype, pattern, seed):
+def _synthetic_cache(B, H, cap, d, dtype, pattern, seed, vmean=0.3, outliers=0):
+    """Compact cache with V ~ N(vmean, 1) on every channel; `outliers` channels
+    per unit (drawn by seed) scaled by 8, mean included, as the outlier
+    channels of the 7B-shaped workload."""
     g = torch.Generator().manual_seed(seed)
     Kc = torch.randn((B, H, cap, d), generator=g).to(dtype)
-    Vc = (torch.randn((B, H, cap, d), generator=g) + 0.3).to(dtype)
+    Vf = torch.randn((B, H, cap, d), generator=g) + vmean
+    if outliers:
+        for b in range(B):
+            for h in range(H):
+                ch = torch.randperm(d, generator=g)[:outliers]
+                Vf[b, h, :, ch] *= 8.0
+    Vc = Vf.to(dtype)
     pi = torch.rand((B, H, cap), generator=g) * 0.999 + 1e-3
     pi[torch.rand((B, H, cap), generator=g) < 0.3] = 1.0  # certainty-set rows
     logw = (-torch.log(pi.double())).float()
@@ -460,6 +469,49 @@ def test_decode_matches_oracle_on_synthetic_cache(E, B, H, G, d, cap, dtype, pat
             sl = slice(h * G, (h + 1) * G)
             compare_decode_heads(dec, out[0][b, sl], out[1][b, sl], out[2][b, sl], out[3][b, sl],
                                  out[4][b, sl], exact)
+
+
+# Values sharing a large mean on every channel: V_hat (Theorem 2) is the
+# spread of the retained values about y_hat, a small fraction of their second
+# moment about the origin (1/257 of it at a mean of 16 with unit spread).
+# One case per decode path: clusters of CTAs, one CTA per unit in waves,
+# split-K with many records per unit, split-K with more units than SMs, the
+# CUDA-core kernels for float32 and for a capacity that is not a multiple of
+# 16; the Qwen-7B-shaped outlier channels (x 8) carry the mean too.
+MEAN_CASES = [
+    # B, H, G, d, cap, dtype, pattern, mean, outlier channels
+    (16, 4, 7, 128, 1600, torch.bfloat16, "edges", 16.0, 0),   # clusters of 2
+    (1, 4, 7, 128, 1600, torch.bfloat16, "random", 4.0, 4),    # clusters of 8
+    (32, 8, 4, 128, 256, torch.bfloat16, "edges", 16.0, 0),    # one CTA per unit, 2 waves
+    (1, 1, 8, 128, 32768, torch.bfloat16, "full", 16.0, 0),    # split-K, one unit
+    (20, 10, 4, 128, 256, torch.bfloat16, "edges", 4.0, 4),    # split-K, 200 units
+    (2, 2, 8, 64, 512, torch.bfloat16, "edges", 16.0, 0),      # split-K, head_dim 64
+    (2, 2, 8, 64, 320, torch.float32, "edges", 16.0, 0),       # CUDA cores, float32
+    (2, 3, 5, 128, 1000, torch.bfloat16, "random", 16.0, 4),   # CUDA cores, bf16
+]
+
+
+@pytest.mark.parametrize("exact", [False, True])
+@pytest.mark.parametrize("B,H,G,d,cap,dtype,pattern,mean,outliers", MEAN_CASES)
+def test_decode_certificate_with_large_common_mean(E, B, H, G, d, cap, dtype, pattern, mean,
+                                                   outliers, exact):
+    Kc, Vc, logw, n = _synthetic_cache(B, H, cap, d, dtype, pattern, seed=B * 31 + G + int(mean),
+                                       vmean=mean, outliers=outliers)
+    g = torch.Generator().manual_seed(17)
+    Q = torch.randn((B, H * G, d), generator=g).to(dtype)
+    out = _decode(E, Q.to(DEV), Kc.to(DEV), Vc.to(DEV), logw.to(DEV), n.to(DEV), exact)
+    Qd, Kd, Vd, ld = Q.double().numpy(), Kc.double().numpy(), Vc.double().numpy(), logw.double().numpy()
+    checked = 0
+    for b in range(B):
+        for h in range(H):
+            k = min(int(n[b, h]), cap)
+            dec = O.hajek_decode(Qd[b, h * G:(h + 1) * G], Kd[b, h, :k], Vd[b, h, :k], ld[b, h, :k])
+            sl = slice(h * G, (h + 1) * G)
+            compare_decode_heads(dec, out[0][b, sl], out[1][b, sl], out[2][b, sl], out[3][b, sl],
+                                 out[4][b, sl], exact)
+            yn2 = np.sum(dec.y * dec.y, axis=1)
+            checked += int(np.sum(dec.var > 1e-9 * yn2))
+    assert checked > 0  # the relative bar was exercised, not only the floor
 
 
 def _decode_outputs(E, args, B, Hq, d):
