@@ -31,8 +31,10 @@ the repository's design notes):
   single precision on both sides because that is the precision the device
   path decides it in.
 * The range term b_t of Eq. (4) is produced in two forms: ``exact`` (the
-  definition, needs y_hat inside the max) and ``bound`` (triangle inequality,
-  computable in one pass; always >= exact).
+  definition, needs y_hat inside the max) and ``bound`` (triangle inequality
+  about a reference row c, computable in one pass; always >= exact).  c is
+  the middle retained row, V_c[(n - 1) // 2]: like b_t itself the bound is
+  then unchanged when every value moves by the same vector.
 
 Every function here is pinned by the ``-m "not gpu"`` tests against closed
 forms, library routines, brute-force enumeration and Monte Carlo; none is
@@ -365,8 +367,12 @@ def hajek_decode(q, K_c, V_c, logw_c, delta: float = 0.1, eps0: float = 1e-9) ->
       With w_i = a_i/pi_i this is sum (1-pi_i) w_i^2 ||v_i - y_hat||^2 / N_hat^2;
       tokens with pi_i = 1 (the certainty set) contribute 0 through (1 - pi_i).
     * Eq. (4): b_t = max_{S cap T} sqrt((1-pi_i)/pi_i^2) a_i ||v_i - y_hat|| / N_hat
-      (``b_exact``), and the one-pass bound
-      (max sqrt(1-pi) w ||v|| + ||y_hat|| max sqrt(1-pi) w) / N_hat (``b_bound``).
+      (``b_exact``), and the one-pass bound about the reference row
+      c = V_c[(n - 1) // 2] (``b_bound``):
+      (max sqrt(1-pi) w ||v - c|| + ||y_hat - c|| max sqrt(1-pi) w) / N_hat,
+      which is >= b_exact because ||v_i - y_hat|| <= ||v_i - c|| + ||c - y_hat||.
+      Both forms are unchanged by a common shift of all values (Eq. 4's b_t
+      depends on the values only through v_i - y_hat).
 
     An empty retained set gives y = 0, lse = -inf and a zero certificate.
     """
@@ -381,6 +387,7 @@ def hajek_decode(q, K_c, V_c, logw_c, delta: float = 0.1, eps0: float = 1e-9) ->
         return DecodeResult(np.zeros((G, d)), np.full(G, -np.inf), z, z.copy(), z.copy(),
                             z.copy(), z.copy())
     one_minus_pi = -np.expm1(-logw)
+    c = V_c[(n - 1) // 2]                               # reference row of the bound
     ys, lses, vs, bes, bbs = [], [], [], [], []
     for h in range(G):
         logits = (K_c @ q[h]) / math.sqrt(d) + logw     # log(a_i / pi_i)
@@ -394,7 +401,7 @@ def hajek_decode(q, K_c, V_c, logw_c, delta: float = 0.1, eps0: float = 1e-9) ->
         var = np.sum(one_minus_pi * p * p * dist * dist)
         b_exact = t.max()
         s = np.sqrt(one_minus_pi) * p
-        b_bound = np.max(s * np.linalg.norm(V_c, axis=1)) + np.linalg.norm(y) * np.max(s)
+        b_bound = np.max(s * np.linalg.norm(V_c - c, axis=1)) + np.linalg.norm(y - c) * np.max(s)
         ys.append(y)
         lses.append(M + math.log(l))
         vs.append(var)

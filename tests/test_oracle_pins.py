@@ -397,6 +397,70 @@ def test_range_term_relations():
     assert abs(r2.b_exact[0] ** 2 / r2.var[0] - 1) < 1e-6
 
 
+def _three_row_design(v0, c, v2):
+    """Three retained rows with zero logits: rows 0 and 1 certain (pi = 1),
+    row 2 a tail row with pi = 1/2.  Then w = (1/2, 1/2, 1) e^0 after the
+    max shift (log(1/pi_2) = ln 2), N_hat share p = (1/4, 1/4, 1/2),
+    y_hat = v0/4 + c/4 + v2/2, and row 1 = (3 - 1) // 2 is the reference row
+    c of the one-pass bound."""
+    V = np.array([v0, c, v2], dtype=np.float64)
+    K = np.zeros((3, V.shape[1]))
+    logw = np.array([0.0, 0.0, math.log(2.0)])
+    return hajek_decode(np.zeros((1, V.shape[1])), K, V, logw)
+
+
+def test_range_bound_tight_when_reference_row_lies_between():
+    """Eq. (4) by hand.  v0 = c - 4 e1, v2 = c + e1: y_hat = c - e1/2 lies on
+    the line through c and v2, beyond c, so ||v2 - y|| = ||v2 - c|| + ||c - y||
+    and the one-pass bound equals the definition:
+    sqrt(1 - 1/2) * (1/2) * 3/2 = 3 sqrt(2) / 8.  V_hat = (1/2)(1/4)(9/4) = 9/32.
+    The same holds after a shift of every value (c = (10, -3))."""
+    for c in ([0.0, 0.0], [10.0, -3.0]):
+        c = np.array(c)
+        e1 = np.array([1.0, 0.0])
+        r = _three_row_design(c - 4 * e1, c, c + e1)
+        np.testing.assert_allclose(r.y[0], c - 0.5 * e1, rtol=0, atol=1e-12)
+        assert abs(r.var[0] - 9 / 32) < 1e-12
+        assert abs(r.b_exact[0] - 3 * math.sqrt(2) / 8) < 1e-12
+        assert abs(r.b_bound[0] - 3 * math.sqrt(2) / 8) < 1e-12
+
+
+def test_range_bound_strict_value_by_hand():
+    """v0 = c + 4 e2, v2 = c + e1: y_hat = c + (1/2, 1).
+    b_exact = (sqrt(2)/4) ||(1/2, -1)|| = (sqrt(2)/4)(sqrt(5)/2);
+    b_bound = (sqrt(2)/4) (||v2 - c|| + ||y - c||) = (sqrt(2)/4)(1 + sqrt(5)/2).
+    Shifted by c = (10, 0) the bound keeps that value; a bound about the
+    origin would give (sqrt(2)/4)(11 + ||(10.5, 1)||), and one without the
+    ||y - c|| term (sqrt(2)/4)."""
+    for c in ([0.0, 0.0], [10.0, 0.0]):
+        c = np.array(c)
+        r = _three_row_design(c + np.array([0.0, 4.0]), c, c + np.array([1.0, 0.0]))
+        s2 = math.sqrt(2) / 4
+        assert abs(r.b_exact[0] - s2 * math.sqrt(5) / 2) < 1e-12
+        assert abs(r.b_bound[0] - s2 * (1 + math.sqrt(5) / 2)) < 1e-12
+        assert abs(r.var[0] - 0.5 * 0.25 * 1.25) < 1e-12
+
+
+def test_radius_constants_by_hand():
+    """Eq. (4): r = (sqrt(2 V log(1/delta)) + b log(1/delta)) / (||y|| + eps0),
+    on literal inputs that single out each constant: a missing factor 2 under
+    the root, log(2/delta) in place of log(1/delta), or eps0 left out of the
+    denominator each change one of these values."""
+    e = math.exp(-1.0)
+    assert abs(certificate_radius(0.5, 0.0, 1.0, e, 0.0) - 1.0) < 1e-15
+    assert abs(certificate_radius(0.0, 1.0, 2.0, e, 0.0) - 0.5) < 1e-15
+    assert abs(certificate_radius(2.0, 0.0, 1.0, e ** 2, 0.0) - math.sqrt(8.0)) < 1e-14
+    L = math.log(10.0)
+    assert abs(certificate_radius(2.0, 3.0, 4.0, 0.1, 1.0)
+               - (2 * math.sqrt(L) + 3 * L) / 5) < 1e-14
+    assert abs(certificate_radius(0.0, 1.0, 0.0, e, 1e-9) - 1e9) < 1e-3
+    # through hajek_decode: the tight three-row design at delta = 0.1
+    r = _three_row_design([-4.0, 0.0], [0.0, 0.0], [1.0, 0.0])
+    b = 3 * math.sqrt(2) / 8
+    expect = (math.sqrt(2 * (9 / 32) * L) + b * L) / (0.5 + 1e-9)
+    assert abs(r.r_exact[0] - expect) < 1e-12 and abs(r.r_bound[0] - expect) < 1e-12
+
+
 def test_radius_scale_invariance_and_zero():
     rng = np.random.default_rng(16)
     q = rng.normal(size=(2, 8))
@@ -409,6 +473,11 @@ def test_radius_scale_invariance_and_zero():
     np.testing.assert_allclose(r2.b_exact, 7 * r1.b_exact, rtol=1e-12)
     np.testing.assert_allclose(r2.r_exact, r1.r_exact, rtol=1e-12)
     np.testing.assert_allclose(r2.r_bound, r1.r_bound, rtol=1e-12)
+    # a common shift of every value leaves V_hat and both range terms unchanged
+    r4 = hajek_decode(q, K, V + np.linspace(-30, 30, 8), logw, eps0=0.0)
+    np.testing.assert_allclose(r4.var, r1.var, rtol=1e-9)
+    np.testing.assert_allclose(r4.b_exact, r1.b_exact, rtol=1e-9)
+    np.testing.assert_allclose(r4.b_bound, r1.b_bound, rtol=1e-9)
     # smaller delta widens the radius
     r3 = hajek_decode(q, K, V, logw, delta=0.01)
     assert np.all(r3.r_exact > r1.r_exact)
