@@ -8,13 +8,13 @@
 //   o  = sum w_i v_i                (Hajek numerator, Eq. 3)
 //   U  = sum u_i,  u_i = (1 - pi_i) w_i^2   (Theorem 2 weights)
 //   A1 = sum u_i v_i,  A2 = sum u_i ||v_i - c||^2  (c: the unit's centring row)
-//   cmax = max sqrt(u_i) ||v_i||,  umax = max sqrt(u_i)   (range-term bound)
+//   cmax = max sqrt(u_i) ||v_i - c||,  umax = max sqrt(u_i)   (range-term bound)
 // A maximum increase by D rescales the w-terms by e^-D and the u-terms by
 // e^-2D.  The reduce kernel merges the splits the same way and finishes
 //   y_hat = o / l,   lse = M + log l  (= log N_hat),
 //   V_hat = (A2 - 2 (y_hat - c).(A1 - U c) + ||y_hat - c||^2 U) / l^2
 //         = sum u_i ||v_i - y_hat||^2 / l^2,
-//   b_t   = (cmax + ||y_hat|| umax) / l   (bound; >= the definition),
+//   b_t   = (cmax + ||y_hat - c|| umax) / l   (bound; >= the definition),
 //   r_t   = (sqrt(2 V_hat ln(1/delta)) + b_t ln(1/delta)) / (||y_hat|| + eps0).
 // The exact range term, max_i sqrt(u_i) ||v_i - y_hat|| / l, needs y_hat and is
 // a second pass over the tail rows (EBD_RANGE_EXACT).
@@ -81,16 +81,14 @@ __global__ void __launch_bounds__(kGenThreads) decode_generic_kernel(DecodeArgs 
     const float lwt = lw[t];
     const float omp = -expm1f(-lwt);  // 1 - pi
     const float sq = sqrtf(omp);
-    float vn2 = 0.f, vc2 = 0.f;
+    float vc2 = 0.f;
 #pragma unroll
     for (int j = 0; j < E; ++j) {
-      vn2 = fmaf(v[j], v[j], vn2);
       const float dv = v[j] - c[j];
       vc2 = fmaf(dv, dv, vc2);
     }
-    vn2 = warp_sum(vn2);
     vc2 = warp_sum(vc2);
-    const float vn = sqrtf(vn2);
+    const float vn = sqrtf(vc2);  // ||v - c||
 #pragma unroll
     for (int g = 0; g < GM; ++g) {
       if (g >= G) break;
@@ -256,10 +254,10 @@ __global__ void __launch_bounds__(kReduceWarps * 32) decode_reduce_kernel(Reduce
   A2 = warp_sum(A2);
   cmax = warp_max(cmax);
   umax = warp_max(umax);
-  float c[PER], yv[PER], ynorm, var;
+  float c[PER], yv[PER], ynorm, ycnorm, var;
   load_centre<T, D, PER>(static_cast<const T*>(a.Vc), unit, a.cap,
                          min(max(a.n_kept[unit], 0), a.cap), lane, c);
-  finish_head<PER>(o, a1, c, l, U, A2, yv, ynorm, var);
+  finish_head<PER>(o, a1, c, l, U, A2, yv, ynorm, ycnorm, var);
 #pragma unroll
   for (int e = 0; e < PER; ++e) a.y[(size_t)hq * D + PER * lane + e] = yv[e];
   if (lane == 0) {
@@ -268,7 +266,7 @@ __global__ void __launch_bounds__(kReduceWarps * 32) decode_reduce_kernel(Reduce
     if (a.exact) {
       a.b_t[hq] = 0.f;  // filled by the exact range pass
     } else {
-      const float bt = (cmax + ynorm * umax) / l;
+      const float bt = (cmax + ycnorm * umax) / l;
       a.b_t[hq] = bt;
       a.radius[hq] = (sqrtf(2.f * var * a.log_inv_delta) + bt * a.log_inv_delta) / (ynorm + a.eps0);
     }

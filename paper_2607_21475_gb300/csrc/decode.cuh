@@ -18,7 +18,8 @@ namespace ebd {
 // so no term carries the values' common mean (with A2 about the origin, a mean
 // of 16 on every channel makes each term ~256 times V_hat l^2 and float32
 // rounding of the sums shows in V_hat).  Any retained row serves: c only has
-// to lie within the spread of the values.
+// to lie within the spread of the values.  The one-pass range bound of Eq. 4
+// is taken about the same row: (max sqrt(u) ||v - c|| + ||y - c|| max sqrt(u)) / l.
 __host__ __device__ constexpr int centre_row(int n) { return n > 0 ? (n - 1) / 2 : -1; }
 
 // Columns PER * lane .. + PER - 1 of the centring row of a unit (n retained
@@ -33,13 +34,14 @@ __device__ __forceinline__ void load_centre(const T* Vc, long long unit, int cap
 }
 
 // Finish one query head from its combined sums (Eq. 3, Theorem 2): y_hat =
-// o / l on this lane's PER columns, ||y_hat|| and
+// o / l on this lane's PER columns, ||y_hat||, ||y_hat - c|| and
 //   V_hat = (A2 - 2 (y - c).(A1 - U c) + ||y - c||^2 U) / l^2
 // with A2 taken about the centring row c (every lane gets the warp's sums).
 template <int PER>
 __device__ __forceinline__ void finish_head(const float (&o)[PER], const float (&a1)[PER],
                                             const float (&c)[PER], float l, float U, float A2,
-                                            float (&yv)[PER], float& ynorm, float& var) {
+                                            float (&yv)[PER], float& ynorm, float& ycnorm,
+                                            float& var) {
   float yy = 0.f, ycyc = 0.f, yca = 0.f;
 #pragma unroll
   for (int e = 0; e < PER; ++e) {
@@ -54,6 +56,7 @@ __device__ __forceinline__ void finish_head(const float (&o)[PER], const float (
   ycyc = warp_sum(ycyc);
   yca = warp_sum(yca);
   ynorm = sqrtf(yy);
+  ycnorm = sqrtf(ycyc);
   var = fmaxf(0.f, (A2 - 2.f * yca + ycyc * U) / (l * l));
 }
 

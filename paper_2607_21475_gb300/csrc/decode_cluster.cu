@@ -84,7 +84,7 @@ struct HeadSum {
   }
 };
 
-template <int D, int S>
+template <int D, int S, bool PACK>
 __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterArgs a) {
   using L = MmaTileLayout<D>;
   constexpr int REC = rec_floats(D);
@@ -112,7 +112,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
   const size_t row_base = (size_t)unit * a.cap;
 
   TileAcc<D> st;
-  tile_acc_begin<D>(st, a.Q, a.Vc, unit, G, a.cap, n_u, lane);
+  tile_acc_begin<D, PACK>(st, a.Q, a.Vc, unit, G, a.cap, n_u, lane);
   int issued = 0;
   auto issue_next = [&]() {
     const int t = tb + issued;
@@ -132,14 +132,14 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
     const int s = warp * S + j % S;
     cp_async_wait<S - 1>();  // this lane's copies of tile j are done
     __syncwarp();            // and every lane's
-    tile_consume<D>(st, smem_u32(smem + (size_t)s * L::kStageBytes), lw_s + s * kMmaTile,
+    tile_consume<D, PACK>(st, smem_u32(smem + (size_t)s * L::kStageBytes), lw_s + s * kMmaTile,
                     min(kMmaTile, n_u - t * kMmaTile), lane, kscale);
   }
   cp_async_wait<0>();
   __syncthreads();  // the ring is free: the warps' records go over it
 
   float* wrec = reinterpret_cast<float*>(smem);  // [warps][G][REC]
-  tile_acc_store<D>(st, wrec + (size_t)warp * G * REC, G, lane);
+  tile_acc_store<D, PACK>(st, wrec + (size_t)warp * G * REC, G, lane);
   __syncthreads();
   if (warp < G) {  // this CTA's part of query head `warp`, sent to CTA 0
     HeadSum<D> h;
@@ -180,9 +180,9 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
     }
     return;
   }
-  float c[PER], yv[PER], ynorm, var;
+  float c[PER], yv[PER], ynorm, ycnorm, var;
   load_centre<__nv_bfloat16, D, PER>(a.Vc, unit, a.cap, n_u, lane, c);
-  finish_head<PER>(h.o, h.a1, c, h.l, h.U, h.A2, yv, ynorm, var);
+  finish_head<PER>(h.o, h.a1, c, h.l, h.U, h.A2, yv, ynorm, ycnorm, var);
 #pragma unroll
   for (int e = 0; e < PER; ++e) a.y[hq * D + PER * lane + e] = yv[e];
   if (lane == 0) {
@@ -191,7 +191,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
     if (a.exact) {
       a.b_t[hq] = 0.f;  // filled by the exact range pass
     } else {
-      const float bt = (h.cm + ynorm * h.um) / h.l;
+      const float bt = (h.cm + ycnorm * h.um) / h.l;
       a.b_t[hq] = bt;
       a.radius[hq] = (sqrtf(2.f * var * a.log_inv_delta) + bt * a.log_inv_delta) / (ynorm + a.eps0);
     }
@@ -201,7 +201,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
 // ---------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------
-template <int D, int S>
+template <int D, int S, bool PACK>
 static ebd_status launch_cluster_t(const DecodeArgs& d, const ReduceArgs& r, int units, int C,
                                    cudaStream_t s) {
   using L = MmaTileLayout<D>;
@@ -225,7 +225,7 @@ static ebd_status launch_cluster_t(const DecodeArgs& d, const ReduceArgs& r, int
   a.eps0 = r.eps0;
   a.exact = r.exact;
   const size_t smem = (size_t)a.lead_off + (size_t)C * d.group * rec_floats(D) * 4 + 1024;
-  if (cudaFuncSetAttribute(decode_cluster_kernel<D, S>,
+  if (cudaFuncSetAttribute(decode_cluster_kernel<D, S, PACK>,
                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return EBD_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
@@ -242,7 +242,7 @@ static ebd_status launch_cluster_t(const DecodeArgs& d, const ReduceArgs& r, int
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cuda_status(cudaLaunchKernelEx(&cfg, decode_cluster_kernel<D, S>, a));
+  return cuda_status(cudaLaunchKernelEx(&cfg, decode_cluster_kernel<D, S, PACK>, a));
 }
 
 // Shared memory of a cluster CTA with S ring stages.
@@ -288,12 +288,21 @@ ebd_status launch_cluster_decode(int head_dim, const DecodeArgs& d, const Reduce
   if (C == 0) return EBD_ERR_UNSUPPORTED;
   const size_t max_smem = 227 * 1024;
   const bool three = cluster_smem(head_dim, 3, C, d.group) <= max_smem;
-  if (head_dim == 128)
-    return three ? launch_cluster_t<128, 3>(d, r, units, C, s)
-                 : launch_cluster_t<128, 2>(d, r, units, C, s);
-  if (head_dim == 64)
-    return three ? launch_cluster_t<64, 3>(d, r, units, C, s)
-                 : launch_cluster_t<64, 2>(d, r, units, C, s);
+  const bool pack = d.group <= 4;
+  if (head_dim == 128) {
+    if (pack)
+      return three ? launch_cluster_t<128, 3, true>(d, r, units, C, s)
+                   : launch_cluster_t<128, 2, true>(d, r, units, C, s);
+    return three ? launch_cluster_t<128, 3, false>(d, r, units, C, s)
+                 : launch_cluster_t<128, 2, false>(d, r, units, C, s);
+  }
+  if (head_dim == 64) {
+    if (pack)
+      return three ? launch_cluster_t<64, 3, true>(d, r, units, C, s)
+                   : launch_cluster_t<64, 2, true>(d, r, units, C, s);
+    return three ? launch_cluster_t<64, 3, false>(d, r, units, C, s)
+                 : launch_cluster_t<64, 2, false>(d, r, units, C, s);
+  }
   return EBD_ERR_UNSUPPORTED;
 }
 

@@ -188,7 +188,7 @@ __device__ void block_tile_prefix(const int32_t* __restrict__ n_kept, int units,
   if (tid == 0) toff[units] = carry;
 }
 
-template <int D>
+template <int D, bool PACK>
 __global__ void __launch_bounds__(kMmaThreads, 1)
     decode_mma_kernel(FastArgs a) {
   using L = MmaLayout<D>;
@@ -256,10 +256,10 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     seg_start = toff[u];
     seg_end = toff[u + 1];
     n_u = min(__ldg(a.n_kept + u), a.cap);
-    tile_acc_begin<D>(st, a.Q, a.Vc, u, G, a.cap, n_u, lane);
+    tile_acc_begin<D, PACK>(st, a.Q, a.Vc, u, G, a.cap, n_u, lane);
   };
   auto flush_segment = [&]() {
-    tile_acc_store<D>(st, a.part + (size_t)(u + gw) * G * REC, G, lane);
+    tile_acc_store<D, PACK>(st, a.part + (size_t)(u + gw) * G * REC, G, lane);
   };
 
   // prologue: the first stages of the ring
@@ -279,7 +279,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     const int s = warp * kMmaStagesPerWarp + j % kMmaStagesPerWarp;
     cp_async_wait<kMmaStagesPerWarp - 1>();  // this lane's copies of tile j are done
     __syncwarp();                             // and every lane's
-    tile_consume<D>(st, smem_u32(smem + (size_t)s * L::kStageBytes), lw_s + s * kMmaTile,
+    tile_consume<D, PACK>(st, smem_u32(smem + (size_t)s * L::kStageBytes), lw_s + s * kMmaTile,
                     n_valid, lane, kscale);
   }
   flush_segment();
@@ -434,10 +434,10 @@ __global__ void __launch_bounds__(MW * 32) decode_merge_kernel(MergeArgs a) {
       a1[e] = fmaf(f2, sh_a[w][PER * lane + e], a1[e]);
     }
   }
-  float c[PER], yv[PER], ynorm, var;
+  float c[PER], yv[PER], ynorm, ycnorm, var;
   load_centre<__nv_bfloat16, D, PER>(a.Vc, u, a.cap, min(max(__ldg(a.n_kept + u), 0), a.cap),
                                      lane, c);
-  finish_head<PER>(o, a1, c, l, U, A2, yv, ynorm, var);
+  finish_head<PER>(o, a1, c, l, U, A2, yv, ynorm, ycnorm, var);
   if constexpr (PER == 4)
     *reinterpret_cast<float4*>(a.y + hq * D + 4 * lane) = make_float4(yv[0], yv[1], yv[2], yv[3]);
   else
@@ -448,7 +448,7 @@ __global__ void __launch_bounds__(MW * 32) decode_merge_kernel(MergeArgs a) {
     if (a.exact) {
       a.b_t[hq] = 0.f;  // filled by the exact range pass
     } else {
-      const float bt = (cm + ynorm * um) / l;
+      const float bt = (cm + ycnorm * um) / l;
       a.b_t[hq] = bt;
       a.radius[hq] = (sqrtf(2.f * var * a.log_inv_delta) + bt * a.log_inv_delta) / (ynorm + a.eps0);
     }
@@ -506,8 +506,10 @@ static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, con
   f.cap = a.cap;
   f.group = a.group;
   const int smem = MmaLayout<D>::kBytes;
-  if (cudaFuncSetAttribute(decode_mma_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           smem) != cudaSuccess)
+  const bool pack = a.group <= 4;
+  auto kern = pack ? decode_mma_kernel<D, true> : decode_mma_kernel<D, false>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+      cudaSuccess)
     return EBD_ERR_CUDA;
   {
     // programmatic dependent of whatever precedes it in the stream: its launch
@@ -522,7 +524,7 @@ static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, con
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    const ebd_status st = cuda_status(cudaLaunchKernelEx(&cfg, decode_mma_kernel<D>, f));
+    const ebd_status st = cuda_status(cudaLaunchKernelEx(&cfg, kern, f));
     if (st != EBD_OK) return st;
   }
 

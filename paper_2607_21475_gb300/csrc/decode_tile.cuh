@@ -9,15 +9,23 @@
 //   P[16 x 16]  = [w (rows 0..7); u (rows 8..15)] as bf16 hi + bf16 lo parts
 //   acc[16 x d] += P_hi . V_tile + P_lo . V_tile   (rows 0..7: o, rows 8..15: A1)
 // plus l = sum w, U = sum u, A2 = sum u ||v - c||^2 and the range-bound
-// maxima cmax = max sqrt(u) ||v||, umax = max sqrt(u).  c is the unit's
+// maxima cmax = max sqrt(u) ||v - c||, umax = max sqrt(u).  c is the unit's
 // centring row (centre_row in decode.cuh), so that the second moment does not
 // carry the values' common mean: the combine forms
 // V_hat l^2 = A2 - 2 (y - c).(A1 - U c) + ||y - c||^2 U, every term of the
-// size of the spread of v around y.  The hi/lo split keeps ~16 mantissa bits
-// of the weights on bf16 tensor cores; ||v||^2 and ||v - c||^2 per token come
-// from the same V fragments.  The running maximum M is updated lazily:
+// size of the spread of v around y, and the one-pass range bound
+// (cmax + ||y - c|| umax) / l.  The hi/lo split keeps ~16 mantissa bits of the
+// weights on bf16 tensor cores; ||v - c||^2 per token comes from the same V
+// fragments.  The running maximum M is updated lazily:
 // accumulators are rescaled only when a row's maximum grows by more than 2^8,
 // so weights stay below 2^8 and u below 2^16.
+//
+// Groups of at most four query heads (PACK) use the MMA rows the heads leave
+// free: query rows 4..7 repeat rows 0..3, so lanes 16..31 compute the same
+// weights bit for bit, and the [w; u] V product takes the hi parts of head g
+// in rows g and g + 8 and the lo parts in rows g + 4 and g + 12 -- one MMA per
+// 8 columns instead of two.  o and A1 are then the sums of rows g and g + 4
+// (resp. g + 8 and g + 12), added when the state is stored.
 //
 // A tile stage holds K and V as 64-column (128-byte) halves of 16 rows in the
 // 128-byte swizzle pattern (chunk ch of row r at r * 128 + ((ch ^ (r & 7)) << 4))
@@ -69,25 +77,28 @@ struct TileAcc {
   uint32_t cneg[D / 16];
 };
 
-// Start a unit: its G query rows as mma A fragments (rows >= G are zero), its
-// centring row (Vc: the compact V cache, cap rows per unit; n_u: the unit's
-// retained rows), and empty sums.
-template <int D>
+// Start a unit: its G query rows as mma A fragments (rows >= G are zero; with
+// PACK, rows 4..7 repeat rows 0..3), its centring row (Vc: the compact V
+// cache, cap rows per unit; n_u: the unit's retained rows), and empty sums.
+template <int D, bool PACK>
 __device__ __forceinline__ void tile_acc_begin(TileAcc<D>& t, const __nv_bfloat16* Q,
                                                const __nv_bfloat16* Vc, int u, int G, int cap,
                                                int n_u, int lane) {
-  const int g = lane >> 2, q = lane & 3;
+  const int q = lane & 3;
   {
+    // channels of this lane's V fragments: 16 jp + lane/4 and 16 jp + 8 + lane/4
+    const int col = lane >> 2;
     const int cr = centre_row(n_u);
     const unsigned short* crow =
         reinterpret_cast<const unsigned short*>(Vc + ((size_t)u * cap + (cr < 0 ? 0 : cr)) * D);
 #pragma unroll
     for (int jp = 0; jp < D / 16; ++jp) {
-      const uint32_t lo = cr < 0 ? 0u : __ldg(crow + 16 * jp + g);
-      const uint32_t hi = cr < 0 ? 0u : __ldg(crow + 16 * jp + 8 + g);
+      const uint32_t lo = cr < 0 ? 0u : __ldg(crow + 16 * jp + col);
+      const uint32_t hi = cr < 0 ? 0u : __ldg(crow + 16 * jp + 8 + col);
       t.cneg[jp] = (lo | (hi << 16)) ^ 0x80008000u;  // both halves negated
     }
   }
+  const int g = PACK ? (lane >> 2) & 3 : lane >> 2;  // query row of this lane's A fragments
   const uint32_t* qrow =
       reinterpret_cast<const uint32_t*>(Q + ((size_t)u * G + (g < G ? g : 0)) * D);
 #pragma unroll
@@ -126,7 +137,7 @@ __device__ __forceinline__ void tile_copy(unsigned char* st, float* lw_dst,
 
 // Fold one tile (stage at shared address kbase, its log(1/pi) at lw; tokens
 // >= n_valid are outside the unit) into the warp's state.
-template <int D>
+template <int D, bool PACK>
 __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, const float* lw,
                                              int n_valid, int lane, float kscale) {
   using L = MmaTileLayout<D>;
@@ -198,19 +209,23 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
   const uint32_t r2 = pack_bf16(wv[2] - bf16_lo(h2), wv[3] - bf16_hi(h2));
   const uint32_t r3 = pack_bf16(uv[2] - bf16_lo(h3), uv[3] - bf16_hi(h3));
   // The scalar sums use exactly the weights the tensor cores multiply with
-  // (hi + lo), so that V_hat = (A2 - 2 y.A1 + |y|^2 U) / l^2 cancels
-  // consistently when y_hat sits close to the retained values.
+  // (hi + lo), so that V_hat = (A2 - 2 (y - c).(A1 - U c) + |y - c|^2 U) / l^2
+  // stays consistent when few tail rows carry it.
   const float wt[4] = {bf16_lo(h0) + bf16_lo(r0), bf16_hi(h0) + bf16_hi(r0),
                        bf16_lo(h2) + bf16_lo(r2), bf16_hi(h2) + bf16_hi(r2)};
   const float ut[4] = {bf16_lo(h1) + bf16_lo(r1), bf16_hi(h1) + bf16_hi(r1),
                        bf16_lo(h3) + bf16_lo(r3), bf16_hi(h3) + bf16_hi(r3)};
   t.l += (wt[0] + wt[1]) + (wt[2] + wt[3]);
   t.U += (ut[0] + ut[1]) + (ut[2] + ut[3]);
+  // PACK: lanes 0..15 feed the hi parts (rows g, g + 8), lanes 16..31 the lo
+  // parts of the same head (rows g + 4, g + 12)
+  const bool upper = PACK && lane >= 16;
+  const uint32_t p0 = upper ? r0 : h0, p1 = upper ? r1 : h1;
+  const uint32_t p2 = upper ? r2 : h2, p3 = upper ? r3 : h3;
 
   // ---- acc += P V, ||v||^2 -------------------------------------------------
   const uint32_t m01 = (tk[0] < n_valid ? 0x0000ffffu : 0u) | (tk[1] < n_valid ? 0xffff0000u : 0u);
   const uint32_t m23 = (tk[2] < n_valid ? 0x0000ffffu : 0u) | (tk[3] < n_valid ? 0xffff0000u : 0u);
-  float2 vn01 = make_float2(0.f, 0.f), vn23 = make_float2(0.f, 0.f);
   float2 vc01 = make_float2(0.f, 0.f), vc23 = make_float2(0.f, 0.f);
   {
     const int tok = ((lane >> 3) & 1) * 8 + (lane & 7);
@@ -230,8 +245,6 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
       const float2 f1 = make_float2(bf16_lo(v1), bf16_hi(v1));
       const float2 f2 = make_float2(bf16_lo(v2), bf16_hi(v2));
       const float2 f3 = make_float2(bf16_lo(v3), bf16_hi(v3));
-      vn01 = __ffma2_rn(f0, f0, __ffma2_rn(f2, f2, vn01));
-      vn23 = __ffma2_rn(f1, f1, __ffma2_rn(f3, f3, vn23));
       // v - c: exact for bf16 v and c of similar magnitude (masked rows give
       // -c, finite, and carry u = 0)
       const float cl = bf16_lo(t.cneg[jp]), ch = bf16_hi(t.cneg[jp]);
@@ -241,25 +254,27 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
       const float2 e3 = __fadd2_rn(f3, make_float2(ch, ch));
       vc01 = __ffma2_rn(e0, e0, __ffma2_rn(e2, e2, vc01));
       vc23 = __ffma2_rn(e1, e1, __ffma2_rn(e3, e3, vc23));
-      mma_bf16_16816(t.acc[2 * jp], h0, h1, h2, h3, v0, v1);
-      mma_bf16_16816(t.acc[2 * jp], r0, r1, r2, r3, v0, v1);
-      mma_bf16_16816(t.acc[2 * jp + 1], h0, h1, h2, h3, v2, v3);
-      mma_bf16_16816(t.acc[2 * jp + 1], r0, r1, r2, r3, v2, v3);
+      if constexpr (PACK) {
+        mma_bf16_16816(t.acc[2 * jp], p0, p1, p2, p3, v0, v1);
+        mma_bf16_16816(t.acc[2 * jp + 1], p0, p1, p2, p3, v2, v3);
+      } else {
+        mma_bf16_16816(t.acc[2 * jp], h0, h1, h2, h3, v0, v1);
+        mma_bf16_16816(t.acc[2 * jp], r0, r1, r2, r3, v0, v1);
+        mma_bf16_16816(t.acc[2 * jp + 1], h0, h1, h2, h3, v2, v3);
+        mma_bf16_16816(t.acc[2 * jp + 1], r0, r1, r2, r3, v2, v3);
+      }
     }
   }
   // every lane's reads of this stage are done before it is refilled
   __syncwarp();
-  float vn[4] = {vn01.x, vn01.y, vn23.x, vn23.y};
   float vc[4] = {vc01.x, vc01.y, vc23.x, vc23.y};
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-#pragma unroll
-    for (int o = 4; o <= 16; o <<= 1) {
-      vn[i] += __shfl_xor_sync(0xffffffffu, vn[i], o);
-      vc[i] += __shfl_xor_sync(0xffffffffu, vc[i], o);
-    }
+    vc[i] += __shfl_xor_sync(0xffffffffu, vc[i], 4);
+    vc[i] += __shfl_xor_sync(0xffffffffu, vc[i], 8);
+    vc[i] += __shfl_xor_sync(0xffffffffu, vc[i], 16);
     t.A2 = fmaf(ut[i], vc[i], t.A2);
-    t.cmax = fmaxf(t.cmax, suv[i] * sqrtf(vn[i]));
+    t.cmax = fmaxf(t.cmax, suv[i] * sqrtf(vc[i]));
   }
 }
 
@@ -267,10 +282,16 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
 // rec + g * rec_floats(D): [M (natural log), l, U, A2 (about the unit's
 // centring row), cmax, umax, -, -, o[D], A1[D]].  The scalar sums are first completed over the four lanes of
 // a head.
-template <int D>
+template <int D, bool PACK>
 __device__ __forceinline__ void tile_acc_store(TileAcc<D>& t, float* rec_base, int G, int lane) {
   constexpr int REC = rec_floats(D);
   const int g = lane >> 2, q = lane & 3;
+  if constexpr (PACK) {  // add the lo rows (lanes 16..31) to the hi rows
+#pragma unroll
+    for (int j = 0; j < D / 8; ++j)
+#pragma unroll
+      for (int k = 0; k < 4; ++k) t.acc[j][k] += __shfl_xor_sync(0xffffffffu, t.acc[j][k], 16);
+  }
 #pragma unroll
   for (int o = 1; o <= 2; o <<= 1) {
     t.l += __shfl_xor_sync(0xffffffffu, t.l, o);

@@ -423,6 +423,9 @@ DECODE_CASES = [
     (20, 10, 4, 128, 256, torch.bfloat16, "edges"),   # 200 units: a 66%-full last wave
     (20, 10, 4, 128, 96, torch.bfloat16, "edges"),    # 200 units of 6 tiles
     (4, 40, 4, 128, 8256, torch.bfloat16, "random"),  # 160 units of 516 tiles
+    # groups of 1 and 3 heads: the hi/lo weight parts share one MMA (rows g, g + 4)
+    (2, 4, 1, 128, 512, torch.bfloat16, "edges"),
+    (6, 8, 3, 64, 256, torch.bfloat16, "random"),
 ]
 
 
