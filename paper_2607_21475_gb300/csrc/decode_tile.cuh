@@ -36,6 +36,8 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 #include "decode.cuh"
 #include "ptx.cuh"
@@ -145,8 +147,11 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
   const uint32_t vbase = kbase + L::kHalves * L::kBoxBytes;
 
   // ---- S = Q K^T ---------------------------------------------------------
+  // even and odd k-steps accumulate separately: two dependent MMA chains of
+  // D/32 per 8 tokens instead of one of D/16
   float sc0[4] = {0.f, 0.f, 0.f, 0.f}, sc1[4] = {0.f, 0.f, 0.f, 0.f};
   {
+    float sd0[4] = {0.f, 0.f, 0.f, 0.f}, sd1[4] = {0.f, 0.f, 0.f, 0.f};
     const int tok = ((lane >> 4) << 3) + (lane & 7);
     const int half_sel = (lane >> 3) & 1;
 #pragma unroll
@@ -156,8 +161,13 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
           kbase + (chunk >> 3) * L::kBoxBytes + tok * 128 + (((chunk & 7) ^ (tok & 7)) << 4);
       uint32_t b0, b1, b2, b3;
       ldsm_x4(addr, b0, b1, b2, b3);
-      mma_bf16_16816(sc0, t.qa[kk][0], 0u, t.qa[kk][1], 0u, b0, b1);
-      mma_bf16_16816(sc1, t.qa[kk][0], 0u, t.qa[kk][1], 0u, b2, b3);
+      mma_bf16_16816(kk & 1 ? sd0 : sc0, t.qa[kk][0], 0u, t.qa[kk][1], 0u, b0, b1);
+      mma_bf16_16816(kk & 1 ? sd1 : sc1, t.qa[kk][0], 0u, t.qa[kk][1], 0u, b2, b3);
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      sc0[i] += sd0[i];
+      sc1[i] += sd1[i];
     }
   }
 
@@ -192,14 +202,22 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
     t.umax *= f;
     t.M2 = mx;
   }
+  // 1 - pi and its square root depend on the token only: lane L computes
+  // them for token L % 16 (0 past the unit) and the lanes that use them read
+  // them with shuffles
+  float omp_t, som_t;
+  {
+    const int tt = lane & (kMmaTile - 1);
+    omp_t = tt < n_valid ? one_minus_exp_neg(lw[tt]) : 0.f;
+    som_t = sqrtf(omp_t);
+  }
   float wv[4], uv[4], suv[4];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const bool val = tk[i] < n_valid;
     wv[i] = exp2f(x[i] - t.M2);
-    const float omp = val ? one_minus_exp_neg(lwv[i]) : 0.f;  // 1 - pi
+    const float omp = __shfl_sync(0xffffffffu, omp_t, tk[i]);  // 1 - pi
     uv[i] = omp * wv[i] * wv[i];
-    suv[i] = sqrtf(omp) * wv[i];
+    suv[i] = __shfl_sync(0xffffffffu, som_t, tk[i]) * wv[i];
     t.umax = fmaxf(t.umax, suv[i]);
   }
   const uint32_t h0 = pack_bf16(wv[0], wv[1]), h1 = pack_bf16(uv[0], uv[1]);
@@ -223,11 +241,16 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
   const uint32_t p0 = upper ? r0 : h0, p1 = upper ? r1 : h1;
   const uint32_t p2 = upper ? r2 : h2, p3 = upper ? r3 : h3;
 
-  // ---- acc += P V, ||v||^2 -------------------------------------------------
-  const uint32_t m01 = (tk[0] < n_valid ? 0x0000ffffu : 0u) | (tk[1] < n_valid ? 0xffff0000u : 0u);
-  const uint32_t m23 = (tk[2] < n_valid ? 0x0000ffffu : 0u) | (tk[3] < n_valid ? 0xffff0000u : 0u);
+  // ---- acc += P V, ||v - c||^2 ----------------------------------------------
+  // Rows past the unit (the last tile only) are zeroed before use: the buffer
+  // may hold anything there, and 0 * NaN would reach the sums.
   float2 vc01 = make_float2(0.f, 0.f), vc23 = make_float2(0.f, 0.f);
-  {
+  auto pv_pass = [&](auto masked) {
+    constexpr bool kMasked = decltype(masked)::value;
+    const uint32_t m01 =
+        (tk[0] < n_valid ? 0x0000ffffu : 0u) | (tk[1] < n_valid ? 0xffff0000u : 0u);
+    const uint32_t m23 =
+        (tk[2] < n_valid ? 0x0000ffffu : 0u) | (tk[3] < n_valid ? 0xffff0000u : 0u);
     const int tok = ((lane >> 3) & 1) * 8 + (lane & 7);
     const int chunk_sel = lane >> 4;
 #pragma unroll
@@ -237,10 +260,12 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
           vbase + (chunk >> 3) * L::kBoxBytes + tok * 128 + (((chunk & 7) ^ (tok & 7)) << 4);
       uint32_t v0, v1, v2, v3;
       ldsm_x4_trans(addr, v0, v1, v2, v3);
-      v0 &= m01;
-      v2 &= m01;
-      v1 &= m23;
-      v3 &= m23;
+      if constexpr (kMasked) {
+        v0 &= m01;
+        v2 &= m01;
+        v1 &= m23;
+        v3 &= m23;
+      }
       const float2 f0 = make_float2(bf16_lo(v0), bf16_hi(v0));
       const float2 f1 = make_float2(bf16_lo(v1), bf16_hi(v1));
       const float2 f2 = make_float2(bf16_lo(v2), bf16_hi(v2));
@@ -264,7 +289,9 @@ __device__ __forceinline__ void tile_consume(TileAcc<D>& t, uint32_t kbase, cons
         mma_bf16_16816(t.acc[2 * jp + 1], r0, r1, r2, r3, v2, v3);
       }
     }
-  }
+  };
+  if (n_valid >= kMmaTile) pv_pass(std::false_type{});
+  else pv_pass(std::true_type{});
   // every lane's reads of this stage are done before it is refilled
   __syncwarp();
   float vc[4] = {vc01.x, vc01.y, vc23.x, vc23.y};
