@@ -86,6 +86,11 @@ def parse_args():
                    help="instead of the step: time the added rows (append/re-eviction cadence, "
                         "certificate aggregation, systematic select, observation queries, "
                         "variance contributions), one JSON line each")
+    p.add_argument("--coverage", action="store_true",
+                   help="instead of the step: coverage of the realised error by the "
+                        "certificate over many Philox seeds, one JSON line per workload "
+                        "(the Qwen-7B shape, the 16k shape at 10/25/50%%, the 32k dialogue)")
+    p.add_argument("--coverage-seeds", type=int, default=200)
     return p.parse_args()
 
 
@@ -490,14 +495,24 @@ def e2e_run(path: Path, steps: int, in_place: bool, n_kept_layers=None):
 
 
 # --------------------------------------------------------------------------- oracle
-def oracle_sample(w: Workload, inputs, seconds: float, max_units=None):
+def oracle_sample(w: Workload, inputs, seconds: float, max_units=None, cc=None,
+                  dev_scores=None):
     """Run the float64 oracle on units of layer 0 until `seconds` of CPU time.
-    Returns (units, evict_s, decode_s, decode_bytes)."""
+    Returns (units, evict_s, decode_s, decode_bytes, parity).  With `cc` (the
+    device's compact cache of layer 0) each sampled unit's kept set is also
+    compared with the oracle's (untimed): parity counts the tail draws with
+    |u - pi| < 1e-5 (where float32 and float64 pi may decide differently),
+    the units whose kept sets differ, and the differing tokens outside that
+    band (0 when the path is right).  For attention-scored workloads the
+    comparison evicts on the device's float32 scores (`dev_scores`)."""
     from oracle import ebd_oracle as O
     B, H, G, d = w.batch, w.n_kv_heads, w.group, w.head_dim
     units = 0
     t_ev = t_dec = 0.0
     dbytes = 0
+    par = {"units": 0, "near_ties": 0, "units_differing": 0, "tokens_differing_outside_band": 0}
+    if cc is not None:
+        n_dev = cc.n_kept.cpu()
     total_units = B * H if max_units is None else min(max_units, B * H)
     for u in range(total_units):
         b, h = divmod(u, H)
@@ -522,9 +537,24 @@ def oracle_sample(w: Workload, inputs, seconds: float, max_units=None):
         n = min(r.n_kept, w.capacity)
         dbytes += n * (2 * d * w.elem_bytes + 4) + G * d * w.elem_bytes + G * (d + 4) * 4
         units += 1
+        if cc is not None:
+            rr = r
+            if dev_scores is not None:
+                rr = O.evict_unit(K, V, dev_scores[b, h].cpu().numpy(), n_sink=w.n_sink,
+                                  n_recent=w.n_recent, k_head=w.k_head,
+                                  budget_tokens=w.budget_tokens, eps=w.eps, seed=w.philox_seed,
+                                  layer=0, b=b, kvh=h, capacity=w.capacity)
+            near = ~rr.certain & (np.abs(rr.u - rr.pi) < 1e-5)
+            ng = int(n_dev[b, h])
+            got = set(cc.idx_c[b, h, :min(ng, w.capacity)].cpu().numpy().tolist())
+            diff = got ^ set(rr.idx.tolist())
+            par["units"] += 1
+            par["near_ties"] += int(near.sum())
+            par["units_differing"] += int(bool(diff) or ng != rr.n_kept)
+            par["tokens_differing_outside_band"] += sum(1 for i in diff if not near[i])
         if t_ev + t_dec >= seconds:
             break
-    return units, t_ev, t_dec, dbytes
+    return units, t_ev, t_dec, dbytes, par
 
 
 def _to_f64(a):
@@ -631,7 +661,7 @@ def run_reference(args, world, rank):
     units = 0
     for i in range(args.warmup + args.steps):
         t = time.perf_counter()
-        u, t_ev, t_dec, db = oracle_sample(w, inputs, per_step)
+        u, t_ev, t_dec, db, _ = oracle_sample(w, inputs, per_step)
         dt = time.perf_counter() - t
         if i >= args.warmup:
             vals.append(db / t_dec / 1e9)
@@ -766,12 +796,17 @@ def run_ours(args, world, rank, local):
                              "Q copied")
 
     cpu = None
+    parity = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        u, t_ev, t_dec, db = oracle_sample(w, path.inputs[0], args.cpu_seconds)
+        u, t_ev, t_dec, db, par = oracle_sample(
+            w, path.inputs[0], args.cpu_seconds, cc=path.cc[0],
+            dev_scores=path.scores[0] if path.scored else None)
         cpu = {"value": db / t_dec / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
                "sample": f"{u} of {w.batch * w.n_kv_heads} (batch row, kv head) units of "
                          f"layer 0: eviction + certified decode ({t_ev + t_dec:.1f} s)",
                "evict_mtok_s": u * w.n_ctx / t_ev / 1e6}
+        parity = dict(par, note="kept sets of the sampled layer-0 units, device against the "
+                                "float64 oracle; tokens may differ only where |u - pi| < 1e-5")
         if not args.no_all_cores:
             try:
                 cpu["all_cores"] = oracle_all_cores(w, path.inputs[0], args.all_core_units)
@@ -789,7 +824,8 @@ def run_ours(args, world, rank, local):
         "decode_pct_of_measured_hbm": 100.0 * value / world / hbm_peak,
         "evict_mtok_s": evict_mtok, "evict_kernels_back_to_back_mtok_s": evict_serial_mtok,
         "phases_ms": ph_ms, "kernels": kern,
-        "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "e2e_copy_all": e2e_copy,
+        "roofline": roof, "cpu_baseline": cpu, "parity_sample": parity, "e2e": e2e,
+        "e2e_copy_all": e2e_copy,
         "gpu_launches": launches,
         "clocks": clk,
     }
@@ -1032,6 +1068,91 @@ def run_sweep(args):
         torch.cuda.empty_cache()
 
 
+# ------------------------------------------------------------------ coverage
+COVERAGE_WORKLOADS = ["qwen7b_6k", "qwen7b_16k_b10", "qwen7b_16k_b25", "qwen7b_16k_b50",
+                      "dialogue_32k"]
+
+
+def coverage_run(w: Workload, seeds, dev, layer: int = 0, delta: float = 0.1,
+                 q_scale: float = 0.0):
+    """Coverage of the realised error by the certificate (Section 3.4, Eq. 4):
+    for each Philox seed, ebd_evict + ebd_certified_decode (both range modes)
+    over the whole layer on the device, then, for every query head,
+    err = ||y_hat - y|| / ||y_hat|| against the full-cache attention y of
+    Eq. 1 from the float64 oracle.  Returns the fraction of (seed, head)
+    cases with err <= r_t for the one-pass bound and for the exact range term,
+    and medians of r_t and err.  q_scale > 0: the peaked-attention variant of
+    the workload (sharpened decode queries, scores accumulated on the device
+    from observation queries that resemble them; workloads.py)."""
+    from oracle import ebd_oracle as O
+    from paper_2607_21475_gb300 import ebd
+    from paper_2607_21475_gb300.workloads import peaked_attention_inputs
+    if q_scale > 0:
+        inp = peaked_attention_inputs(w, layer, dev, q_scale=q_scale)
+    else:
+        inp = make_layer_inputs(w, layer, dev)
+    B, H, G, d, N = w.batch, w.n_kv_heads, w.group, w.head_dim, w.n_ctx
+    Hq = w.n_q_heads
+    if "q_obs" in inp:
+        scores = torch.empty((B, H, N), dtype=torch.float32, device=dev)
+        ebd.ebd_score(inp["q_obs"], inp["K"], scores)
+    else:
+        scores = inp["scores"]
+    y_full = np.empty((B, Hq, d))
+    for b in range(B):
+        for h in range(H):
+            y_full[b, h * G:(h + 1) * G] = O.full_attention(
+                inp["Q"][b, h * G:(h + 1) * G].double().cpu().numpy(),
+                inp["K"][b, h].double().cpu().numpy(), inp["V"][b, h].double().cpu().numpy())
+    cc = ebd.alloc_compact(B, H, w.capacity, d, w.torch_dtype, dev)
+    y = torch.empty((B, Hq, d), dtype=torch.float32, device=dev)
+    lse, var, bt, r_b, r_e = (torch.empty((B, Hq), dtype=torch.float32, device=dev)
+                              for _ in range(5))
+    errs, rbs, res = [], [], []
+    for s in seeds:
+        des = ebd.design_for(batch=B, n_kv_heads=H, group=G, head_dim=d, n_ctx=N, layer=layer,
+                             seed=int(s), n_sink=w.n_sink, n_recent=w.n_recent, k_head=w.k_head,
+                             budget_tokens=w.budget_tokens, bisect_iters=w.bisect_iters,
+                             eps=w.eps)
+        ebd.ebd_evict(des, inp["K"], inp["V"], scores, None, cc)
+        ebd.ebd_certified_decode(inp["Q"], cc.K_c, cc.V_c, cc.logw_c, cc.n_kept, y, lse, var, bt,
+                                 r_e, delta=delta, range_mode=ebd.EBD_RANGE_EXACT)
+        ebd.ebd_certified_decode(inp["Q"], cc.K_c, cc.V_c, cc.logw_c, cc.n_kept, y, lse, var, bt,
+                                 r_b, delta=delta, range_mode=ebd.EBD_RANGE_BOUND)
+        yh = y.double().cpu().numpy()
+        errs.append(np.linalg.norm(yh - y_full, axis=-1) / np.linalg.norm(yh, axis=-1))
+        rbs.append(r_b.double().cpu().numpy())
+        res.append(r_e.double().cpu().numpy())
+    torch.cuda.synchronize()
+    if cc.dev_status.item():
+        raise RuntimeError(f"{w.name}: device status {cc.dev_status.item()}")
+    err, rb, re_ = (np.concatenate([a.ravel() for a in x]) for x in (errs, rbs, res))
+    return {
+        "workload": w.name, "seeds": len(seeds), "cases": int(err.size),
+        "delta": delta, "layer": layer,
+        "inputs": (f"peaked: decode queries x {q_scale}, scores accumulated from observation "
+                   f"queries resembling them" if q_scale > 0 else "as the workload states"),
+        "coverage_bound": float(np.mean(err <= rb)), "coverage_exact": float(np.mean(err <= re_)),
+        "median_radius_bound": float(np.median(rb)), "median_radius_exact": float(np.median(re_)),
+        "median_rel_error": float(np.median(err)), "p99_rel_error": float(np.quantile(err, 0.99)),
+        "note": ("fraction of (seed, query head) cases with ||y_hat - y|| / ||y_hat|| <= r_t, "
+                 "y the full-cache attention of Eq. 1 (float64 oracle), y_hat and r_t from "
+                 "the CUDA path; a reported number, not a pinned one"),
+    }
+
+
+def run_coverage(args):
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    names = [args.workload] if args.workload != "dialogue_32k" or "--workload" in sys.argv[1:] \
+        else COVERAGE_WORKLOADS
+    for name in names:
+        w = WORKLOADS[name]
+        for qs in (0.0, 2.0, 3.0):
+            print(json.dumps(coverage_run(w, range(args.coverage_seeds), dev, q_scale=qs)))
+            torch.cuda.empty_cache()
+
+
 def main():
     args = parse_args()
     world, rank, local = dist_setup(args)
@@ -1043,6 +1164,9 @@ def main():
     elif args.rows:
         if rank == 0:
             run_rows(args)
+    elif args.coverage:
+        if rank == 0:
+            run_coverage(args)
     else:
         run_ours(args, world, rank, local)
     if world > 1 and args.impl == "ours":

@@ -23,7 +23,8 @@ from dataclasses import dataclass, field, replace
 
 import torch
 
-__all__ = ["Workload", "WORKLOADS", "sweep_workloads", "make_layer_inputs", "unit_seed"]
+__all__ = ["Workload", "WORKLOADS", "sweep_workloads", "make_layer_inputs",
+           "peaked_attention_inputs", "unit_seed"]
 
 
 @dataclass(frozen=True)
@@ -180,3 +181,27 @@ def make_layer_inputs(w: Workload, layer: int = 0, device="cpu", batch=None):
             raise ValueError(w.score_kind)
         out["scores"] = s.contiguous()
     return out
+
+
+def peaked_attention_inputs(w: Workload, layer: int = 0, device="cpu", q_scale: float = 3.0,
+                            obs_noise: float = 0.5, n_obs: int = 64):
+    """A workload's K, V with decode queries sharpened and observation queries
+    that resemble them, for measuring the certificate where attention is
+    concentrated (with K, Q ~ N(0, 1) at d = 128 each query spreads its mass
+    over thousands of tokens and the full-cache output is close to 0).
+
+    Q = q_scale * Q0 (Q0 the workload's queries); ``q_obs`` [B,Hkv,n_obs*G,d]:
+    row r of KV head h is q_scale * (Q0[h*G + r // n_obs] + obs_noise * z),
+    z ~ N(0, 1), so scores accumulated from them rank tokens the way the
+    decode queries weight them.  Returns the dict of make_layer_inputs with
+    Q replaced, ``q_obs`` added and ``scores`` removed."""
+    inp = make_layer_inputs(w, layer, device)
+    inp.pop("scores", None)
+    B, Hkv, G, d = w.batch, w.n_kv_heads, w.group, w.head_dim
+    q0 = inp["Q"].float()
+    gz = _gen(device, unit_seed(w, layer, 6))
+    z = torch.randn((B, Hkv, n_obs * G, d), generator=gz, device=device, dtype=torch.float32)
+    base = q0.view(B, Hkv, G, 1, d).expand(B, Hkv, G, n_obs, d).reshape(B, Hkv, G * n_obs, d)
+    inp["q_obs"] = (q_scale * (base + obs_noise * z)).to(w.torch_dtype).contiguous()
+    inp["Q"] = (q_scale * q0).to(w.torch_dtype).contiguous()
+    return inp

@@ -87,3 +87,21 @@ def test_inputs_are_deterministic_per_seed_and_layer():
     for k in ("K", "V", "Q", "scores"):
         assert torch.equal(a[k], b[k])
         assert not torch.equal(a[k], c[k])
+
+
+def test_peaked_attention_inputs_follow_their_recipe():
+    """Sharpened queries: Q = 3 Q0; observation row r of KV head h is
+    3 (Q0[h G + r // 64] + 0.5 z): its mean over the 64 rows of a query head
+    sits within a few standard errors of that head's query."""
+    from paper_2607_21475_gb300.workloads import peaked_attention_inputs
+    w = WORKLOADS["qwen7b_6k"].with_(batch=1)
+    base = make_layer_inputs(w, 2, "cpu")
+    inp = peaked_attention_inputs(w, 2, "cpu", q_scale=3.0, obs_noise=0.5)
+    assert "scores" not in inp and inp["q_obs"].shape == (1, 4, 64 * 7, 128)
+    assert torch.equal(inp["K"], base["K"]) and torch.equal(inp["V"], base["V"])
+    torch.testing.assert_close(inp["Q"].float(), (3 * base["Q"].float()).to(torch.bfloat16).float())
+    qo = inp["q_obs"].float().view(1, 4, 7, 64, 128)
+    dev = (qo.mean(dim=3) - 3 * base["Q"].float().view(1, 4, 7, 128)).abs()
+    assert float(dev.max()) < 6 * 3 * 0.5 / 8 + 0.1  # 6 standard errors of a 64-row mean
+    again = peaked_attention_inputs(w, 2, "cpu", q_scale=3.0, obs_noise=0.5)
+    assert torch.equal(again["q_obs"], inp["q_obs"])
