@@ -54,8 +54,11 @@ typedef enum {
 typedef enum { EBD_F32 = 0, EBD_BF16 = 1 } ebd_dtype;
 
 /* Range term b_t of Eq. (4).  BOUND (default) is the one-pass triangle
- * inequality bound  (max sqrt(1-pi) w ||v|| + ||y_hat|| max sqrt(1-pi) w) / N_hat,
- * never below the definition.  EXACT evaluates the definition
+ * inequality bound about a reference row c, the unit's middle retained row
+ * V_c[(n - 1) / 2]:
+ *   (max sqrt(1-pi) w ||v - c|| + ||y_hat - c|| max sqrt(1-pi) w) / N_hat,
+ * never below the definition and, like it, unchanged when every value moves
+ * by the same vector.  EXACT evaluates the definition
  * max_{S cap T} sqrt(1-pi_i) w_i ||v_i - y_hat|| / N_hat with a second pass over
  * the compact cache once y_hat is known. */
 typedef enum { EBD_RANGE_BOUND = 0, EBD_RANGE_EXACT = 1 } ebd_range_mode;
@@ -220,6 +223,19 @@ ebd_status ebd_gather(const ebd_design* design, ebd_dtype dtype, const void* K, 
                       void* V_c, void* stream);
 
 /*
+ * One workspace size for a whole layer (the boundary of Section 3.1's problem
+ * statement: the design fixed per layer, the retained set of `capacity` rows
+ * per unit): the largest of ebd_evict_workspace_bytes(design, 0) (scores
+ * given), ebd_evict_workspace_bytes(design, 64 * group) (accumulated-attention
+ * scoring from 64 observation positions per query head, the window of
+ * Appendix B) and ebd_decode_workspace_bytes(dtype, B, Hkv, G, d, capacity)
+ * for either dtype.  A buffer of this size serves every call of the layer;
+ * the per-call queries give exact, smaller sizes.  0 for a NULL design or
+ * capacity < 1.  ebd_compute_pi, ebd_select and ebd_gather need none.
+ */
+size_t ebd_workspace_bytes(const ebd_design* design, int32_t capacity);
+
+/*
  * Certified decode step (Eq. 3, Theorem 2, Eq. 4) for every query head.
  *   Q        device [B,Hkv*G,d] (dtype): query heads kvh*G .. kvh*G+G-1 read the
  *            compact cache of KV head kvh
@@ -234,7 +250,9 @@ ebd_status ebd_gather(const ebd_design* design, ebd_dtype dtype, const void* K, 
  *   dev_status device int32, nullable
  * An empty unit (n_kept = 0) gives y = 0, lse = -inf and a zero certificate.
  * Needs workspace of ebd_decode_workspace_bytes(...) bytes for the split-K
- * partial records.  Supports d in {64, 128} and 1 <= G <= 8.
+ * partial records.  Supports d in {64, 128} and 1 <= G <= 16; a group of
+ * more than 8 query heads is decoded in two slices of at most 8 heads, one
+ * pass over the compact cache each (EBD_ERR_UNSUPPORTED beyond 16).
  * Results are reproducible bit for bit: a request always takes the same
  * kernels and the same summation order on a given GPU (the choice depends on
  * the request's shape and the GPU's SM count, so GPUs with another SM count

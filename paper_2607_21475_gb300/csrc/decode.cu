@@ -19,8 +19,10 @@
 // The exact range term, max_i sqrt(u_i) ||v_i - y_hat|| / l, needs y_hat and is
 // a second pass over the tail rows (EBD_RANGE_EXACT).
 //
-// This file holds the CUDA-core path (any supported dtype, head_dim 64/128,
-// G <= 8).  Its record layout and reduce are shared with the tensor-core path.
+// This file holds the CUDA-core path (any supported dtype, head_dim 64/128, at
+// most 8 query heads per pass) and the entry point, which decodes a group of
+// up to 16 heads in slices.  The record layout and reduce are shared with the
+// tensor-core path.
 #include <cuda_runtime.h>
 #include <math.h>
 
@@ -41,12 +43,11 @@ __global__ void __launch_bounds__(kGenThreads) decode_generic_kernel(DecodeArgs 
   const int unit = blockIdx.y, split = blockIdx.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = a.group;
-  const int b = unit / a.n_kv_heads, kvh = unit - b * a.n_kv_heads;
   const int n = min(a.n_kept[unit], a.cap);
   const int t0 = split * a.tokens_per_split;
   const int t1 = min(n, t0 + a.tokens_per_split);
   const float scale = rsqrtf((float)D);
-  const T* Q = (const T*)a.Q + ((size_t)b * a.n_kv_heads * G + (size_t)kvh * G) * D;
+  const T* Q = (const T*)a.Q + (size_t)unit * a.gstride * D;
   const T* Kc = (const T*)a.Kc + (size_t)unit * a.cap * D;
   const T* Vc = (const T*)a.Vc + (size_t)unit * a.cap * D;
   const float* lw = a.logw + (size_t)unit * a.cap;
@@ -181,10 +182,11 @@ __global__ void __launch_bounds__(kReduceWarps * 32) decode_reduce_kernel(Reduce
   constexpr int REC = rec_floats(D);
   constexpr int PER = D / 32;
   const int lane = threadIdx.x & 31;
-  const int hq = blockIdx.x * kReduceWarps + (threadIdx.x >> 5);
-  if (hq >= n_heads) return;
+  const int hs = blockIdx.x * kReduceWarps + (threadIdx.x >> 5);  // head of the slice
+  if (hs >= n_heads) return;
   const int G = a.group;
-  const int unit = hq / G, g = hq - unit * G;
+  const int unit = hs / G, g = hs - unit * G;
+  const int hq = unit * a.gstride + g;  // output row
   const long long first = (long long)unit * a.splits;
   const int count = a.splits;
   const size_t slot = (size_t)G * REC;
@@ -281,18 +283,15 @@ __global__ void __launch_bounds__(kGenThreads) decode_exact_range_kernel(DecodeA
   const int unit = blockIdx.y, split = blockIdx.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = a.group;
-  const int b = unit / a.n_kv_heads, kvh = unit - b * a.n_kv_heads;
   const int n = min(a.n_kept[unit], a.cap);
   const int t0 = split * a.tokens_per_split;
   const int t1 = min(n, t0 + a.tokens_per_split);
   const float scale = rsqrtf((float)D);
-  const size_t hq0 = (size_t)unit * G;
+  const size_t hq0 = (size_t)unit * a.gstride;
   const T* Q = (const T*)a.Q + hq0 * D;
   const T* Kc = (const T*)a.Kc + (size_t)unit * a.cap * D;
   const T* Vc = (const T*)a.Vc + (size_t)unit * a.cap * D;
   const float* lw = a.logw + (size_t)unit * a.cap;
-  (void)b;
-  (void)kvh;
   float q[GM][E], yv[GM][E], lse[GM], best[GM];
 #pragma unroll
   for (int g = 0; g < GM; ++g) {
@@ -414,9 +413,17 @@ static DecodePlan plan_generic(long long units, int group, int head_dim, int cap
   return p;
 }
 
+// Groups of more than kSliceHeads query heads are decoded in slices of at
+// most kSliceHeads heads, one pass over the compact cache each (the
+// tensor-core tile holds 8 query rows and their 8 u rows).
+constexpr int kSliceHeads = 8;
+static int decode_slices(int group) { return (group + kSliceHeads - 1) / kSliceHeads; }
+
 DecodePlan plan_decode(ebd_dtype dtype, int batch, int n_kv_heads, int group, int head_dim,
                        int capacity) {
   const long long units = (long long)batch * n_kv_heads;
+  const int slices = decode_slices(group);
+  group = (group + slices - 1) / slices;  // the largest slice; slices reuse the workspace
   DecodePlan p = plan_generic(units, group, head_dim, capacity);
   if (fast_decode_supported(dtype, group, head_dim, capacity)) {
     const size_t generic_ws = p.ws_bytes;
@@ -437,6 +444,43 @@ extern "C" size_t ebd_decode_workspace_bytes(ebd_dtype dtype, int32_t batch, int
   return plan_decode(dtype, batch, n_kv_heads, group, head_dim, capacity).ws_bytes;
 }
 
+extern "C" size_t ebd_workspace_bytes(const ebd_design* design, int32_t capacity) {
+  if (!design || capacity < 1) return 0;
+  const ebd_design& d = *design;
+  size_t need = ebd_evict_workspace_bytes(design, 0);
+  const size_t scored = ebd_evict_workspace_bytes(design, 64 * d.group);
+  if (scored > need) need = scored;
+  for (ebd_dtype t : {EBD_F32, EBD_BF16}) {
+    const size_t dec =
+        ebd_decode_workspace_bytes(t, d.batch, d.n_kv_heads, d.group, d.head_dim, capacity);
+    if (dec > need) need = dec;
+  }
+  return need;
+}
+
+namespace ebd {
+
+ebd_status check_decode_args(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads, int32_t group,
+                             int32_t head_dim, const void* Q, const void* K_c, const void* V_c,
+                             const float* logw_c, const int32_t* n_kept, int32_t capacity,
+                             float delta, float eps0, ebd_range_mode range_mode, const float* y,
+                             const float* lse, const float* var_hat, const float* b_t,
+                             const float* radius) {
+  if (dtype != EBD_F32 && dtype != EBD_BF16) return EBD_ERR_INVALID;
+  if (batch < 1 || n_kv_heads < 1 || group < 1 || capacity < 1) return EBD_ERR_INVALID;
+  if (!Q || !K_c || !V_c || !logw_c || !n_kept || !y || !lse || !var_hat || !b_t || !radius)
+    return EBD_ERR_INVALID;
+  if (!(delta > 0.f && delta < 1.f) || !(eps0 >= 0.f)) return EBD_ERR_INVALID;
+  if (range_mode != EBD_RANGE_BOUND && range_mode != EBD_RANGE_EXACT) return EBD_ERR_INVALID;
+  if (head_dim != 64 && head_dim != 128) return EBD_ERR_UNSUPPORTED;
+  if (group > 2 * kSliceHeads) return EBD_ERR_UNSUPPORTED;
+  const long long units = (long long)batch * n_kv_heads;
+  if (units * group > 0x7fffffffLL || units > 65535) return EBD_ERR_UNSUPPORTED;
+  return EBD_OK;
+}
+
+}  // namespace ebd
+
 extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads,
                                            int32_t group, int32_t head_dim, const void* Q,
                                            const void* K_c, const void* V_c, const float* logw_c,
@@ -445,34 +489,27 @@ extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32
                                            float* lse, float* var_hat, float* b_t, float* radius,
                                            int32_t* dev_status, void* workspace, size_t ws_bytes,
                                            void* stream) {
-  if (dtype != EBD_F32 && dtype != EBD_BF16) return EBD_ERR_INVALID;
-  if (batch < 1 || n_kv_heads < 1 || group < 1 || capacity < 1) return EBD_ERR_INVALID;
-  if (!Q || !K_c || !V_c || !logw_c || !n_kept || !y || !lse || !var_hat || !b_t || !radius)
-    return EBD_ERR_INVALID;
-  if (!(delta > 0.f && delta < 1.f) || !(eps0 >= 0.f)) return EBD_ERR_INVALID;
-  if (range_mode != EBD_RANGE_BOUND && range_mode != EBD_RANGE_EXACT) return EBD_ERR_INVALID;
-  if (head_dim != 64 && head_dim != 128) return EBD_ERR_UNSUPPORTED;
-  if (group > 8) return EBD_ERR_UNSUPPORTED;
+  const ebd_status arg = check_decode_args(dtype, batch, n_kv_heads, group, head_dim, Q, K_c,
+                                           V_c, logw_c, n_kept, capacity, delta, eps0,
+                                           range_mode, y, lse, var_hat, b_t, radius);
+  if (arg != EBD_OK) return arg;
   const long long units = (long long)batch * n_kv_heads;
-  if (units * group > 0x7fffffffLL || units > 65535) return EBD_ERR_UNSUPPORTED;
   const DecodePlan plan = plan_decode(dtype, batch, n_kv_heads, group, head_dim, capacity);
   if (!workspace || ws_bytes < plan.ws_bytes) return EBD_ERR_CAPACITY;
   cudaStream_t s = (cudaStream_t)stream;
+  const size_t esize = dtype == EBD_F32 ? 4 : 2;
 
   DecodeArgs a;
-  a.Q = Q;
   a.Kc = K_c;
   a.Vc = V_c;
   a.logw = logw_c;
   a.n_kept = n_kept;
   a.cap = capacity;
   a.n_kv_heads = n_kv_heads;
-  a.group = group;
+  a.gstride = group;
   a.splits = plan.splits;
   a.tokens_per_split = plan.tokens_per_split;
   a.part = (float*)workspace;
-  a.y = y;
-  a.lse = lse;
   a.dev_status = dev_status;
 
   ReduceArgs r;
@@ -481,42 +518,58 @@ extern "C" ebd_status ebd_certified_decode(ebd_dtype dtype, int32_t batch, int32
   r.n_kept = n_kept;
   r.cap = capacity;
   r.splits = plan.splits;
-  r.group = group;
+  r.gstride = group;
+  r.log_inv_delta = logf(1.f / delta);
+  r.eps0 = eps0;
+  r.exact = range_mode == EBD_RANGE_EXACT;
+
+  // one pass per slice of at most kSliceHeads query heads (one slice for G <= 8);
+  // the slices run in stream order and reuse the workspace
+  const int slices = decode_slices(group);
+  for (int sl = 0; sl < slices; ++sl) {
+    const int h0 = sl * group / slices, h1 = (sl + 1) * group / slices;
+    a.group = r.group = h1 - h0;
+    a.Q = static_cast<const char*>(Q) + (size_t)h0 * head_dim * esize;
+    a.y = r.y = y + (size_t)h0 * head_dim;
+    a.lse = r.lse = lse + h0;
+    r.var = var_hat + h0;
+    a.b_t = r.b_t = b_t + h0;
+    r.radius = radius + h0;
+    const int n_heads = (int)(units * a.group);
+    ebd_status st;
+    if (plan.fast && fast_decode_usable(a, r, (int)units)) {
+      st = launch_fast_decode(dtype, head_dim, plan, a, r, (int)units, workspace, s);
+    } else {
+      st = dispatch_generic(false, dtype, head_dim, a, (int)units, s);
+      if (st == EBD_OK) {
+        const int rblocks = (n_heads + kReduceWarps - 1) / kReduceWarps;
+        const dim3 rg(rblocks), rb(kReduceWarps * 32);
+        if (dtype == EBD_F32) {
+          if (head_dim == 128) decode_reduce_kernel<float, 128><<<rg, rb, 0, s>>>(r, n_heads);
+          else decode_reduce_kernel<float, 64><<<rg, rb, 0, s>>>(r, n_heads);
+        } else {
+          if (head_dim == 128) decode_reduce_kernel<__nv_bfloat16, 128><<<rg, rb, 0, s>>>(r, n_heads);
+          else decode_reduce_kernel<__nv_bfloat16, 64><<<rg, rb, 0, s>>>(r, n_heads);
+        }
+        st = launch_status();
+      }
+    }
+    if (st != EBD_OK) return st;
+    // exact range term: second pass over the slice's tail rows
+    if (r.exact) {
+      st = dispatch_generic(true, dtype, head_dim, a, (int)units, s);
+      if (st != EBD_OK) return st;
+    }
+  }
+  if (!r.exact) return EBD_OK;
+  // the radius of every query head from its V_hat and exact range term
+  r.group = r.gstride = group;
   r.y = y;
   r.lse = lse;
   r.var = var_hat;
   r.b_t = b_t;
   r.radius = radius;
-  r.log_inv_delta = logf(1.f / delta);
-  r.eps0 = eps0;
-  r.exact = range_mode == EBD_RANGE_EXACT;
   const int n_heads = (int)(units * group);
-  ebd_status st;
-  if (plan.fast && fast_decode_usable(a, r, (int)units)) {
-    st = launch_fast_decode(dtype, head_dim, plan, a, r, (int)units, workspace, s);
-  } else {
-    st = dispatch_generic(false, dtype, head_dim, a, (int)units, s);
-    if (st == EBD_OK) {
-      const int rblocks = (n_heads + kReduceWarps - 1) / kReduceWarps;
-      const dim3 rg(rblocks), rb(kReduceWarps * 32);
-      if (dtype == EBD_F32) {
-        if (head_dim == 128) decode_reduce_kernel<float, 128><<<rg, rb, 0, s>>>(r, n_heads);
-        else decode_reduce_kernel<float, 64><<<rg, rb, 0, s>>>(r, n_heads);
-      } else {
-        if (head_dim == 128) decode_reduce_kernel<__nv_bfloat16, 128><<<rg, rb, 0, s>>>(r, n_heads);
-        else decode_reduce_kernel<__nv_bfloat16, 64><<<rg, rb, 0, s>>>(r, n_heads);
-      }
-      st = launch_status();
-    }
-  }
-  if (st != EBD_OK) return st;
-  if (!r.exact) return EBD_OK;
-  // exact range term: second pass over the tail rows, then the radius
-  a.splits = plan.splits;
-  a.tokens_per_split = plan.tokens_per_split;
-  a.b_t = b_t;
-  st = dispatch_generic(true, dtype, head_dim, a, (int)units, s);
-  if (st != EBD_OK) return st;
   const int warps = 4;
   if (head_dim == 128)
     decode_radius_kernel<128><<<(n_heads + warps - 1) / warps, warps * 32, 0, s>>>(r, n_heads);

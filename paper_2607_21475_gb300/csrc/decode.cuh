@@ -72,6 +72,11 @@ __host__ __device__ constexpr bool rec_is_squared(int e, int D) {
   return e == kRecU || e == kRecA2 || e >= kRecHead + D;
 }
 
+// Groups of more than 8 query heads are decoded in slices of at most 8 heads
+// (one pass over the compact cache each): `group` is the slice's head count,
+// `gstride` the group size of the Q / output layout (query head g of unit u
+// of the slice at row u * gstride + g of the slice's Q and output pointers,
+// which the host offsets to the slice's first head).
 struct DecodeArgs {
   const void* Q;          // [B, Hkv*G, D]
   const void* Kc;         // [units, cap, D]
@@ -81,6 +86,7 @@ struct DecodeArgs {
   int cap;
   int n_kv_heads;
   int group;
+  int gstride;
   int splits;             // split slots per unit in `part`
   int tokens_per_split;   // CUDA-core path: token range of one split
   float* part;            // [units, splits, G, rec_floats(D)]
@@ -97,6 +103,7 @@ struct ReduceArgs {
   int cap;
   int splits;                // records per unit
   int group;
+  int gstride;
   float* y;
   float* lse;
   float* var;
@@ -117,6 +124,15 @@ struct DecodePlan {
 
 DecodePlan plan_decode(ebd_dtype dtype, int batch, int n_kv_heads, int group, int head_dim,
                        int capacity);
+
+// Argument checks of ebd_certified_decode (everything but the workspace), so
+// that its variants answer a bad request with the same status.
+ebd_status check_decode_args(ebd_dtype dtype, int32_t batch, int32_t n_kv_heads, int32_t group,
+                             int32_t head_dim, const void* Q, const void* K_c, const void* V_c,
+                             const float* logw_c, const int32_t* n_kept, int32_t capacity,
+                             float delta, float eps0, ebd_range_mode range_mode, const float* y,
+                             const float* lse, const float* var_hat, const float* b_t,
+                             const float* radius);
 
 // Tensor-core path (decode_mma.cu): decode kernel, then a merge kernel
 // launched as its programmatic dependent (plus a prefix kernel above 4096

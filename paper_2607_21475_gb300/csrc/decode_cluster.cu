@@ -33,7 +33,8 @@ struct ClusterArgs {
   const float* logw;        // [units, cap]
   const int32_t* n_kept;    // [units]
   int cap;
-  int group;
+  int group;                // query heads of this slice (decode.cuh)
+  int gstride;              // query heads per unit in the Q / output layout
   int csize;                // CTAs per cluster (per unit)
   int lw_off;               // shared-memory layout, bytes: log(1/pi) stages
   int lead_off;             // CTA records gathered in CTA 0: [csize][G][rec_floats(D)]
@@ -112,7 +113,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
   const size_t row_base = (size_t)unit * a.cap;
 
   TileAcc<D> st;
-  tile_acc_begin<D, PACK>(st, a.Q, a.Vc, unit, G, a.cap, n_u, lane);
+  tile_acc_begin<D, PACK>(st, a.Q, a.Vc, unit, G, a.gstride, a.cap, n_u, lane);
   int issued = 0;
   auto issue_next = [&]() {
     const int t = tb + issued;
@@ -168,7 +169,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
 
   HeadSum<D> h;
   h.combine<8>(lead + (size_t)warp * REC, C, (size_t)G * REC, lane);
-  const long long hq = (long long)unit * G + warp;
+  const long long hq = (long long)unit * a.gstride + warp;
   if (h.M == -INFINITY) {  // no retained row: y = 0, lse = -inf, zero certificate
 #pragma unroll
     for (int e = 0; e < PER; ++e) a.y[hq * D + PER * lane + e] = 0.f;
@@ -213,6 +214,7 @@ static ebd_status launch_cluster_t(const DecodeArgs& d, const ReduceArgs& r, int
   a.n_kept = d.n_kept;
   a.cap = d.cap;
   a.group = d.group;
+  a.gstride = d.gstride;
   a.csize = C;
   a.lw_off = kMmaConsumers * S * L::kStageBytes;
   a.lead_off = (int)align_up((size_t)a.lw_off + (size_t)kMmaConsumers * S * kMmaTile * 4, 16);

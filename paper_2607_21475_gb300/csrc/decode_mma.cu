@@ -69,7 +69,8 @@ struct FastArgs {
   int32_t* dev_status;
   int units;
   int cap;
-  int group;
+  int group;                 // query heads of this slice (decode.cuh)
+  int gstride;               // query heads per unit in the Q layout
 };
 
 struct MergeArgs {
@@ -80,7 +81,8 @@ struct MergeArgs {
   int cap;
   long long warps;           // warps of the decode grid
   int units;
-  int group;
+  int group;                 // query heads of this slice
+  int gstride;               // query heads per unit in the output layout
   float* y;                  // [units * G, D]
   float* lse;                // [units * G]
   float* var;
@@ -256,7 +258,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     seg_start = toff[u];
     seg_end = toff[u + 1];
     n_u = min(__ldg(a.n_kept + u), a.cap);
-    tile_acc_begin<D, PACK>(st, a.Q, a.Vc, u, G, a.cap, n_u, lane);
+    tile_acc_begin<D, PACK>(st, a.Q, a.Vc, u, G, a.gstride, a.cap, n_u, lane);
   };
   auto flush_segment = [&]() {
     tile_acc_store<D, PACK>(st, a.part + (size_t)(u + gw) * G * REC, G, lane);
@@ -306,8 +308,8 @@ __global__ void __launch_bounds__(MW * 32) decode_merge_kernel(MergeArgs a) {
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = a.group;
-  const long long hq = blockIdx.x;
-  const int u = (int)(hq / G), g = (int)(hq - (long long)u * G);
+  const int u = (int)(blockIdx.x / G), g = (int)(blockIdx.x - u * G);
+  const long long hq = (long long)u * a.gstride + g;  // output row
   const long long t0 = a.tile_off[u], t1 = a.tile_off[u + 1];
   if (t1 == t0) {  // no retained row: y = 0, lse = -inf, zero certificate
     if (warp == 0) {
@@ -505,6 +507,7 @@ static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, con
   f.units = units;
   f.cap = a.cap;
   f.group = a.group;
+  f.gstride = a.gstride;
   const int smem = MmaLayout<D>::kBytes;
   const bool pack = a.group <= 4;
   auto kern = pack ? decode_mma_kernel<D, true> : decode_mma_kernel<D, false>;
@@ -537,6 +540,7 @@ static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, con
   m.warps = (long long)plan.ctas * kMmaConsumers;
   m.units = units;
   m.group = a.group;
+  m.gstride = a.gstride;
   m.y = r.y;
   m.lse = r.lse;
   m.var = r.var;

@@ -79,13 +79,14 @@ struct TileAcc {
   uint32_t cneg[D / 16];
 };
 
-// Start a unit: its G query rows as mma A fragments (rows >= G are zero; with
-// PACK, rows 4..7 repeat rows 0..3), its centring row (Vc: the compact V
-// cache, cap rows per unit; n_u: the unit's retained rows), and empty sums.
+// Start a unit: its G query rows (row u * qstride + g of Q) as mma A fragments
+// (rows >= G are zero; with PACK, rows 4..7 repeat rows 0..3), its centring
+// row (Vc: the compact V cache, cap rows per unit; n_u: the unit's retained
+// rows), and empty sums.
 template <int D, bool PACK>
 __device__ __forceinline__ void tile_acc_begin(TileAcc<D>& t, const __nv_bfloat16* Q,
-                                               const __nv_bfloat16* Vc, int u, int G, int cap,
-                                               int n_u, int lane) {
+                                               const __nv_bfloat16* Vc, int u, int G, int qstride,
+                                               int cap, int n_u, int lane) {
   const int q = lane & 3;
   {
     // channels of this lane's V fragments: 16 jp + lane/4 and 16 jp + 8 + lane/4
@@ -102,7 +103,7 @@ __device__ __forceinline__ void tile_acc_begin(TileAcc<D>& t, const __nv_bfloat1
   }
   const int g = PACK ? (lane >> 2) & 3 : lane >> 2;  // query row of this lane's A fragments
   const uint32_t* qrow =
-      reinterpret_cast<const uint32_t*>(Q + ((size_t)u * G + (g < G ? g : 0)) * D);
+      reinterpret_cast<const uint32_t*>(Q + ((size_t)u * qstride + (g < G ? g : 0)) * D);
 #pragma unroll
   for (int kk = 0; kk < D / 16; ++kk) {
     t.qa[kk][0] = g < G ? __ldg(qrow + 8 * kk + q) : 0u;

@@ -1457,7 +1457,7 @@ extern "C" const char* ebd_status_string(ebd_status s) {
   return "EBD_ERR_UNKNOWN";
 }
 
-extern "C" int32_t ebd_abi_version(void) { return 2; }
+extern "C" int32_t ebd_abi_version(void) { return 3; }
 
 extern "C" ebd_status ebd_philox_uniforms(uint64_t seed, int32_t layer, int32_t batch,
                                           int32_t n_kv_heads, int32_t n_ctx, uint32_t* x0,

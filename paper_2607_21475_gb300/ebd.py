@@ -27,7 +27,7 @@ __all__ = [
     "EBD_SAMPLING_SYSTEMATIC", "lib", "lib_path",
     "ebd_status_string", "ebd_abi_version", "ebd_philox_uniforms", "ebd_score_workspace_bytes",
     "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
-    "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
+    "ebd_gather", "ebd_decode_workspace_bytes", "ebd_workspace_bytes", "ebd_certified_decode",
     "ebd_certified_decode_static", "ebd_certificate_update", "ebd_append", "ebd_reevict",
     "ebd_gather_queries", "ebd_variance_contributions", "ebd_block_scores",
     "ebd_check_stalled_wait", "design_for",
@@ -45,7 +45,7 @@ EBD_SAMPLING_POISSON, EBD_SAMPLING_SYSTEMATIC = 0, 1
 ABI_FUNCTIONS = (
     "ebd_status_string", "ebd_abi_version", "ebd_philox_uniforms", "ebd_score_workspace_bytes",
     "ebd_score", "ebd_compute_pi", "ebd_evict_workspace_bytes", "ebd_evict", "ebd_select",
-    "ebd_gather", "ebd_decode_workspace_bytes", "ebd_certified_decode",
+    "ebd_gather", "ebd_decode_workspace_bytes", "ebd_workspace_bytes", "ebd_certified_decode",
     "ebd_certified_decode_static", "ebd_certificate_update", "ebd_append", "ebd_reevict",
     "ebd_gather_queries", "ebd_variance_contributions", "ebd_block_scores",
     "ebd_check_stalled_wait",
@@ -104,6 +104,7 @@ def lib():
             "ebd_gather": (ctypes.c_int, [P, ctypes.c_int, c_void_p, c_void_p, c_void_p, c_void_p,
                                           i32, c_void_p, c_void_p, c_void_p]),
             "ebd_decode_workspace_bytes": (sz, [ctypes.c_int, i32, i32, i32, i32, i32]),
+            "ebd_workspace_bytes": (sz, [P, i32]),
             "ebd_certified_decode": (ctypes.c_int, [ctypes.c_int, i32, i32, i32, i32, c_void_p,
                                                     c_void_p, c_void_p, c_void_p, c_void_p, i32,
                                                     f32, f32, ctypes.c_int, c_void_p, c_void_p,
@@ -248,6 +249,11 @@ def ebd_compute_pi(design: EbdDesign, scores: torch.Tensor, pi: torch.Tensor,
 
 def ebd_evict_workspace_bytes(design: EbdDesign, n_obs: int) -> int:
     return int(lib().ebd_evict_workspace_bytes(ctypes.byref(design), int(n_obs)))
+
+
+def ebd_workspace_bytes(design: EbdDesign, capacity: int) -> int:
+    """One workspace size serving every call of a layer with this design."""
+    return int(lib().ebd_workspace_bytes(ctypes.byref(design), int(capacity)))
 
 
 @dataclass

@@ -69,7 +69,7 @@ def test_status_strings_and_version(E):
     L = E.lib()
     for code in range(6):
         assert L.ebd_status_string(code).startswith(b"EBD_")
-    assert E.ebd_abi_version() == 2
+    assert E.ebd_abi_version() == 3
 
 
 def test_bad_arguments_are_rejected_synchronously(E):
@@ -105,14 +105,15 @@ def test_bad_arguments_are_rejected_synchronously(E):
     a4 = list(args)
     a4[0] = byref(d_odd)
     assert L.ebd_evict(*a4) == 4
-    # decode: head_dim outside {64,128}, group > 8, delta outside (0,1), null outputs
+    # decode: head_dim outside {64,128}, group > 16, delta outside (0,1), null outputs
+    # (each refused before anything is enqueued)
     dec = [0, 1, 1, 1, 64, fake, fake, fake, fake, fake, 64, ctypes.c_float(0.1),
            ctypes.c_float(1e-9), 0, fake, fake, fake, fake, fake, null, fake, 1 << 20, null]
     x = list(dec)
     x[4] = 96
     assert L.ebd_certified_decode(*x) == 4
     x = list(dec)
-    x[3] = 9
+    x[3] = 17
     assert L.ebd_certified_decode(*x) == 4
     x = list(dec)
     x[11] = ctypes.c_float(1.0)
@@ -133,3 +134,22 @@ def test_workspace_queries(E):
     assert E.ebd_evict_workspace_bytes(d, 0) == 0
     assert E.ebd_evict_workspace_bytes(d, 448) >= 8 * 4 * (6144 + 448) * 4
     assert E.ebd_score_workspace_bytes(8, 4, 448) >= 8 * 4 * 448 * 4
+
+
+def test_one_workspace_size_serves_every_call_of_a_layer(E):
+    """ebd_workspace_bytes(design, capacity) is the largest per-call need:
+    eviction with given scores, with scoring from 64 observation positions
+    per query head, and the decode in either dtype -- including a group of
+    16 query heads, decoded in slices of 8."""
+    for G, N, cap in ((7, 6144, 1728), (4, 32768, 3520), (16, 8192, 1024)):
+        d = E.design_for(batch=8, n_kv_heads=4, group=G, head_dim=128, n_ctx=N,
+                         k_head=cap // 8, budget_tokens=cap // 2)
+        need = E.ebd_workspace_bytes(d, cap)
+        parts = [E.ebd_evict_workspace_bytes(d, 0), E.ebd_evict_workspace_bytes(d, 64 * G)]
+        parts += [E.ebd_decode_workspace_bytes(t, 8, 4, G, 128, cap)
+                  for t in (E.EBD_F32, E.EBD_BF16)]
+        assert need == max(parts) > 0
+    assert E.lib().ebd_workspace_bytes(None, 64) == 0
+    # a group of 16 heads needs the workspace of one slice of 8
+    assert (E.ebd_decode_workspace_bytes(E.EBD_BF16, 8, 4, 16, 128, 1024)
+            == E.ebd_decode_workspace_bytes(E.EBD_BF16, 8, 4, 8, 128, 1024))

@@ -426,6 +426,13 @@ DECODE_CASES = [
     # groups of 1 and 3 heads: the hi/lo weight parts share one MMA (rows g, g + 4)
     (2, 4, 1, 128, 512, torch.bfloat16, "edges"),
     (6, 8, 3, 64, 256, torch.bfloat16, "random"),
+    # groups of 9..16 heads: two slices of <= 8 heads, one pass each
+    (2, 4, 12, 128, 512, torch.bfloat16, "edges"),    # split-K, slices of 6
+    (16, 4, 12, 128, 1600, torch.bfloat16, "random"), # one CTA per unit, slices of 6
+    (3, 2, 16, 64, 320, torch.bfloat16, "random"),    # split-K, slices of 8, head_dim 64
+    (40, 8, 16, 128, 256, torch.bfloat16, "edges"),   # 320 units, slices of 8
+    (2, 2, 12, 64, 200, torch.float32, "edges"),      # CUDA cores
+    (2, 3, 9, 128, 1000, torch.bfloat16, "random"),   # CUDA cores, slices of 4 + 5
 ]
 
 
@@ -650,10 +657,12 @@ def test_evict_then_decode_tiny_end_to_end(E):
     E.ebd_evict(des, inp["K"].to(DEV), inp["V"].to(DEV), inp["scores"].to(DEV), None, cc)
     out = _decode(E, inp["Q"].to(DEV), cc.K_c, cc.V_c, cc.logw_c, cc.n_kept)
     npi = {k: v.double().numpy() for k, v in inp.items()}
+    decoded = ties = 0
     for b in range(B):
         for h in range(H):
             ref = oracle_unit(w, npi, b, h, 0, scores=inp["scores"][b, h].numpy())
             n = int(cc.n_kept[b, h])
+            ties += int(np.sum(~ref.certain & (np.abs(ref.u - ref.pi) < TIE_BAND)))
             same = n == ref.n_kept and np.array_equal(cc.idx_c[b, h, :n].cpu().numpy(), ref.idx)
             if not same:
                 continue  # a near tie moved one token; covered by test_evict_matches_oracle
@@ -661,6 +670,9 @@ def test_evict_then_decode_tiny_end_to_end(E):
             sl = slice(h * G, (h + 1) * G)
             compare_decode_heads(dec, out[0][b, sl], out[1][b, sl], out[2][b, sl], out[3][b, sl],
                                  out[4][b, sl], False)
+            decoded += 1
+    # every unit without a draw in the tie band is decoded and checked
+    assert decoded >= 1 and decoded >= B * H - ties
 
 
 # ------------------------------------------------------------------ scoring
