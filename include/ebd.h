@@ -80,7 +80,7 @@ typedef enum { EBD_RANGE_BOUND = 0, EBD_RANGE_EXACT = 1 } ebd_range_mode;
  * (C_{i-1} - u, C_i - u].  Its inclusion probability is pi_i and the tail
  * sample has floor or ceil of sum pi tokens; joint inclusion probabilities do
  * not factor, so the certificate's variance form is then an approximation.
- * Supported for N <= 32768. */
+ * Supported at every context length (1 <= N <= 2^20). */
 typedef enum { EBD_SAMPLING_POISSON = 0, EBD_SAMPLING_SYSTEMATIC = 1 } ebd_sampling;
 
 /* Design of one layer's eviction (Section 3.3 and Appendix B of the paper). */

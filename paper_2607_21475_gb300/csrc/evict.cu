@@ -152,22 +152,24 @@ __device__ __forceinline__ void load4(const float* s, int i0, int N, bool vec4, 
 }
 
 // Exclusive prefix over the block, in thread order, of `cnt`, and the block
-// total; two barriers (sh.tot is free again when it returns).
-__device__ __forceinline__ int big_scan(int cnt, int& total, BigScratch& sh) {
+// total; two barriers (sh.tot is free again when it returns).  T = unsigned
+// sums modulo 2^32 (the systematic walk).
+template <typename T>
+__device__ __forceinline__ T big_scan(T cnt, T& total, BigScratch& sh) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  int incl = cnt;
+  T incl = cnt;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    const int n = __shfl_up_sync(0xffffffffu, incl, o);
+    const T n = __shfl_up_sync(0xffffffffu, incl, o);
     if (lane >= o) incl += n;
   }
-  if (lane == 31) sh.tot[warp] = incl;
+  if (lane == 31) sh.tot[warp] = (int)incl;
   __syncthreads();
-  int before = 0, tot = 0;
+  T before = 0, tot = 0;
 #pragma unroll 8
   for (int w = 0; w < kSelWarps; ++w) {
-    const int c = sh.tot[w];
-    before += w < warp ? c : 0;
+    const T c = (T)sh.tot[w];
+    before += w < warp ? c : (T)0;
     tot += c;
   }
   __syncthreads();
@@ -463,7 +465,15 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
 
   // ---- E3 + E4a: draws, stable compaction of (index, log 1/pi) -------------
   const bool compact = a.n_kept != nullptr;
+  const bool systematic = compact && a.systematic;
   int kept = 0;
+  // Systematic design (as in the shared-memory kernel): the tail in token
+  // order, pi in units of 2^-32 (rounded to the nearest unit; pi = 1 adds 0
+  // and is always kept), one uniform u per unit at counter word 0 = 2^32 - 1;
+  // a tail token is kept when the running fraction of C - u carries out.
+  // `frac`: that fraction before the current step (sums modulo 2^32).
+  uint32_t frac = 0u;
+  if (systematic) frac = 0u - ((draw_block(a.seed, a.layer, b, kvh, -1).x >> 8) << 8);
 #pragma unroll 1
   for (int base = 0; base < N; base += kBigStep * kBigUnroll) {
     float v[kBigUnroll][4];
@@ -475,10 +485,10 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
       const int i0 = base + q * kBigStep + 4 * tid;
       const uint32_t c4 = i0 < N ? cert4(i0) : 0xFu;
       uint4 w = make_uint4(0u, 0u, 0u, 0u);
-      if (compact && i0 < N) w = draw_block(a.seed, a.layer, b, kvh, i0 >> 2);
+      if (compact && !systematic && i0 < N) w = draw_block(a.seed, a.layer, b, kvh, i0 >> 2);
       const uint32_t wr[4] = {w.x, w.y, w.z, w.w};
       float pis[4];
-      uint32_t keep4 = 0u;
+      uint32_t keep4 = 0u, tail4 = 0u, units4[4] = {0u, 0u, 0u, 0u}, tsum = 0u;
 #pragma unroll
       for (int r = 0; r < 4; ++r) {
         const int i = i0 + r;
@@ -489,11 +499,33 @@ __global__ void __launch_bounds__(kSelThreads, 1) evict_select_kernel(SelectArgs
         pis[r] = pi;
         if (a.pi_out) a.pi_out[(size_t)unit * Nrow + i] = pi;
         if (a.mask_out) a.mask_out[(size_t)unit * Nrow + i] = ct ? 1 : 0;
-        if (compact && (ct || word_to_uniform(wr[r]) < pi)) keep4 |= 1u << r;
+        if (systematic) {
+          if (ct) {
+            keep4 |= 1u << r;
+          } else {
+            tail4 |= 1u << r;
+            units4[r] = pi >= 1.f ? 0u : __float2uint_rn(pi * 4294967296.f);
+            tsum += units4[r];
+          }
+        } else if (compact && (ct || word_to_uniform(wr[r]) < pi)) {
+          keep4 |= 1u << r;
+        }
+      }
+      if (systematic) {
+        uint32_t stotal;
+        uint32_t run = frac + big_scan<uint32_t>(tsum, stotal, sh);
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          if (!((tail4 >> r) & 1u)) continue;
+          const uint32_t before = run;
+          run += units4[r];
+          if (pis[r] >= 1.f || run < before) keep4 |= 1u << r;  // a carry: an integer crossed
+        }
+        frac += stotal;
       }
       if (compact) {
         int total;
-        int p = kept + big_scan(__popc(keep4), total, sh);
+        int p = kept + big_scan<int>(__popc(keep4), total, sh);
 #pragma unroll
         for (int r = 0; r < 4; ++r) {
           if (!((keep4 >> r) & 1u)) continue;
@@ -1393,7 +1425,6 @@ ebd_status launch_select_range(const ebd_design* d, const float* scores, const i
     evict_select_smem_kernel<<<units, kRegThreads, smem, stream>>>(a, groups);
     return launch_status();
   }
-  if (a.systematic && idx_c) return EBD_ERR_UNSUPPORTED;
   // certainty bits (padded to 16 bytes), then the per-warp first-digit histograms
   const int words_pad = ((d->n_ctx + 31) / 32 + 3) & ~3;
   const size_t smem = (size_t)words_pad * 4 + (size_t)kSelWarps * 256 * 4;

@@ -809,7 +809,11 @@ def test_append_then_reevict_then_decode_matches_oracle(E):
 @pytest.mark.parametrize("B,H,N,budget,dist", [(2, 3, 1000, 100, "lognormal"),
                                                (1, 4, 20000, 2000, "pareto"),
                                                (2, 2, 32768, 3277, "lognormal"),
-                                               (1, 2, 70001, 7000, "lognormal")])
+                                               (1, 2, 70001, 7000, "lognormal"),
+                                               (1, 2, 131072, 13107, "pareto"),
+                                               # beyond 8 x 32768 tokens: the select whose
+                                               # scores stay in global memory
+                                               (1, 1, 300000, 30000, "lognormal")])
 def test_systematic_select_matches_oracle(E, B, H, N, budget, dist):
     g = torch.Generator().manual_seed(N + budget)
     if dist == "lognormal":
