@@ -271,8 +271,9 @@ def source_sha(relpath):
 
 
 def traffic_for(kernel, workload):
-    """DRAM bytes per launch from a committed ncu capture, if its kernel source
-    is unchanged since the capture (else null)."""
+    """DRAM bytes per launch from a committed ncu capture, if its kernel's
+    sources (one file, or a list whose hashes are joined by '+') are unchanged
+    since the capture (else null)."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
@@ -281,7 +282,8 @@ def traffic_for(kernel, workload):
         return None
     for e in entries:
         if e.get("kernel") == kernel and e.get("workload") == workload:
-            if e.get("source_sha") == source_sha(e["source"]):
+            src = e["source"] if isinstance(e["source"], list) else [e["source"]]
+            if e.get("source_sha") == "+".join(source_sha(f) for f in src):
                 return float(e["dram_bytes_per_launch"])
     return None
 
@@ -492,6 +494,24 @@ def e2e_run(path: Path, steps: int, in_place: bool, n_kept_layers=None):
     t1.record()
     torch.cuda.synchronize()
     return t0.elapsed_time(t1) / steps, h2d, d2h
+
+
+def host_link_peak(dev, nbytes: int = 512 << 20, reps: int = 5):
+    """Measured host -> device rate of this box's link: a page-locked buffer
+    copied to the device (best of `reps`, CUDA events), in GB/s -- the
+    denominator of the end-to-end line's link fraction."""
+    src = torch.empty(nbytes, dtype=torch.uint8).pin_memory()
+    dst = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    best = float("inf")
+    for _ in range(reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        dst.copy_(src, non_blocking=True)
+        b.record()
+        torch.cuda.synchronize()
+        best = min(best, a.elapsed_time(b))
+    del src, dst
+    return nbytes / (best * 1e-3) / 1e9
 
 
 # --------------------------------------------------------------------------- oracle
@@ -786,6 +806,14 @@ def run_ours(args, world, rank, local):
         e2e_copy["inputs"] = ("K, V, Q and the " + ("observation queries" if path.scored else
                               "scores") + " copied to the device each step")
         e2e = e2e_line(True)
+        link = host_link_peak(dev)
+        for line_ in (e2e, e2e_copy):
+            moved = (line_["h2d_bytes_per_step"] + line_["d2h_bytes_per_step"]) / (
+                line_["ms_per_step"] * 1e-3) / 1e9
+            line_["host_link"] = {"achieved_gbs": moved, "h2d_peak_gbs": link,
+                                  "frac": moved / link,
+                                  "peak_source": "page-locked 512 MiB host->device copy, "
+                                                 "best of 5, measured in this run"}
         if path.scored:
             e2e["inputs"] = ("K, Q and the observation queries copied (scoring reads every key); "
                              "V read in place from page-locked host memory (the gather reads "
