@@ -18,6 +18,7 @@
 #include <cuda_runtime.h>
 
 #include "common.cuh"
+#include "decode.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -112,14 +113,20 @@ __global__ void __launch_bounds__(kCtbThreads)
 // and the query heads as its N (padded to 8), both products share one
 // fragment layout: S^T = K Q^T (Q fragments in registers) and V Y^T (y_hat as
 // bf16 hi + lo, about 16 bits), so each lane holds, for tokens g and g + 8
-// (g = lane / 4) and heads 2q, 2q + 1 (q = lane % 4): the logit, v . y_hat,
-// and ||v||^2 from the same V fragments.  The contribution is
-// (1 - pi) p^2 (||v||^2 - 2 v . y_hat + ||y_hat||^2), p = 2^(x log2e - lse log2e).
+// (g = lane / 4) and heads 2q, 2q + 1 (q = lane % 4): the logit,
+// v . (y_hat - c) and ||v - c||^2 from the same V fragments, c the unit's
+// centring row (decode.cuh).  The contribution is
+// (1 - pi) p^2 (||v - c||^2 - 2 (v - c).(y_hat - c) + ||y_hat - c||^2),
+// p = 2^(x log2e - lse log2e): every term of the size of the values' spread,
+// none of their common mean.  With a head column to spare (SPARE: G < 8) the
+// product's column G carries c, so that ||v - c||^2 = ||v||^2 - 2 v.c + ||c||^2
+// per token (exact products, a float32 cancellation of one token's terms);
+// with G = 8 the V fragments are centred element by element.
 constexpr int kCtmWarps = 8;
 constexpr int kCtmTilesPerWarp = 16;
 constexpr int kCtmStages = 3;
 
-template <int D>
+template <int D, bool SPARE>
 __global__ void __launch_bounds__(kCtmWarps * 32)
     contrib_mma_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ Kc,
                        const __nv_bfloat16* __restrict__ Vc, const float* __restrict__ logw,
@@ -146,10 +153,24 @@ __global__ void __launch_bounds__(kCtmWarps * 32)
   const int t_end = min(ntiles, t_begin + kCtmTilesPerWarp);
   const size_t hq0 = (size_t)unit * G;
 
-  // B fragments (k = d index, n = head): Q and y_hat (hi, lo) of head g
+  // the unit's centring row c (bf16, exact as a V row; zeros for an empty
+  // unit): pairs at channels 16 kk + 2q (.x) and 16 kk + 8 + 2q (.y), the
+  // channels of this lane's V fragments
+  const int cr = centre_row(n);
+  const __nv_bfloat16* crow = Vc + ((size_t)unit * cap + (cr < 0 ? 0 : cr)) * D;
+  uint32_t cp[D / 16][2];  // -c, both bf16 halves negated
+#pragma unroll
+  for (int kk = 0; kk < D / 16; ++kk) {
+    const uint32_t* c32 = reinterpret_cast<const uint32_t*>(crow + 16 * kk);
+    cp[kk][0] = (cr < 0 ? 0u : c32[q]) ^ 0x80008000u;
+    cp[kk][1] = (cr < 0 ? 0u : c32[4 + q]) ^ 0x80008000u;
+  }
+  // B fragments (k = d index, n = head): Q and y_hat - c (hi, lo) of head g;
+  // with SPARE, column G carries c itself (bf16, exact: lo part 0)
   uint32_t qb[D / 16][2], yh[D / 16][2], yl[D / 16][2];
   {
     const bool hv = g < G;
+    const bool cv = SPARE && g == G;
     const __nv_bfloat16* qrow = Q + (hq0 + (hv ? g : 0)) * D;
     const float* yrow = y + (hq0 + (hv ? g : 0)) * D;
 #pragma unroll
@@ -159,28 +180,44 @@ __global__ void __launch_bounds__(kCtmWarps * 32)
       qb[kk][1] = hv ? q32[4 + q] : 0u;
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
-        const float y0 = hv ? yrow[16 * kk + 8 * h + 2 * q] : 0.f;
-        const float y1 = hv ? yrow[16 * kk + 8 * h + 2 * q + 1] : 0.f;
+        const float y0 = hv ? yrow[16 * kk + 8 * h + 2 * q] + bf16_lo(cp[kk][h]) : 0.f;
+        const float y1 = hv ? yrow[16 * kk + 8 * h + 2 * q + 1] + bf16_hi(cp[kk][h]) : 0.f;
         const uint32_t hi = pack_bf16(y0, y1);
-        yh[kk][h] = hi;
-        yl[kk][h] = pack_bf16(y0 - bf16_lo(hi), y1 - bf16_hi(hi));
+        yh[kk][h] = cv ? cp[kk][h] ^ 0x80008000u : hi;
+        yl[kk][h] = cv ? 0u : pack_bf16(y0 - bf16_lo(hi), y1 - bf16_hi(hi));
       }
     }
   }
-  // per-head constants for the heads this lane's C fragments hold (2q, 2q + 1)
-  float l2[2], yy[2] = {0.f, 0.f};
+  // per-head constants for the heads this lane's C fragments hold (2q, 2q + 1):
+  // ||y_hat - c||^2 and c . (y_hat - c), by warp reductions
+  float l2[2], yy[2] = {0.f, 0.f}, cy[2] = {0.f, 0.f}, cc = 0.f;
 #pragma unroll
   for (int c = 0; c < 2; ++c) {
     const int h = 2 * q + c;
     l2[c] = h < G ? lse[hq0 + h] * kLog2e : 0.f;
   }
-  for (int h = 0; h < G; ++h) {  // ||y_hat_h||^2 by a warp reduction
+  for (int h = 0; h < G; ++h) {
+    float s2 = 0.f, sc = 0.f;
+#pragma unroll
+    for (int e = lane; e < D; e += 32) {
+      const float ce = cr < 0 ? 0.f : __bfloat162float(crow[e]);
+      const float yc = y[(hq0 + h) * D + e] - ce;
+      s2 = fmaf(yc, yc, s2);
+      sc = fmaf(ce, yc, sc);
+    }
+    s2 = warp_sum(s2);
+    sc = warp_sum(sc);
+    if (h == 2 * q) { yy[0] = s2; cy[0] = sc; }
+    if (h == 2 * q + 1) { yy[1] = s2; cy[1] = sc; }
+  }
+  if constexpr (SPARE) {  // ||c||^2
     float s2 = 0.f;
 #pragma unroll
-    for (int e = lane; e < D; e += 32) s2 = fmaf(y[(hq0 + h) * D + e], y[(hq0 + h) * D + e], s2);
-    s2 = warp_sum(s2);
-    if (h == 2 * q) yy[0] = s2;
-    if (h == 2 * q + 1) yy[1] = s2;
+    for (int e = lane; e < D; e += 32) {
+      const float ce = cr < 0 ? 0.f : __bfloat162float(crow[e]);
+      s2 = fmaf(ce, ce, s2);
+    }
+    cc = warp_sum(s2);
   }
   const float kscale = kLog2e * rsqrtf((float)D);
 
@@ -215,7 +252,7 @@ __global__ void __launch_bounds__(kCtmWarps * 32)
       const uint32_t kbase = smem_u32(sm[warp][slot]);
       const uint32_t vbase = kbase + kHalves * kBox;
       float st[4] = {0.f, 0.f, 0.f, 0.f}, vy[4] = {0.f, 0.f, 0.f, 0.f};
-      float vn0 = 0.f, vn1 = 0.f;  // ||v||^2 partials of tokens g and g + 8
+      float2 vn0 = make_float2(0.f, 0.f), vn1 = make_float2(0.f, 0.f);  // ||v - c||^2 of tokens g, g + 8
       const int tok = (lane & 7) + ((lane >> 3) & 1) * 8;
       const int csel = lane >> 4;
 #pragma unroll
@@ -229,16 +266,35 @@ __global__ void __launch_bounds__(kCtmWarps * 32)
         ldsm_x4(vbase + off, v0, v1, v2, v3);
         mma_bf16_16816(vy, v0, v1, v2, v3, yh[kk][0], yh[kk][1]);
         mma_bf16_16816(vy, v0, v1, v2, v3, yl[kk][0], yl[kk][1]);
-        // v0, v2: token g; v1, v3: token g + 8 (two bf16 each)
-        vn0 = fmaf(bf16_lo(v0), bf16_lo(v0), fmaf(bf16_hi(v0), bf16_hi(v0), vn0));
-        vn0 = fmaf(bf16_lo(v2), bf16_lo(v2), fmaf(bf16_hi(v2), bf16_hi(v2), vn0));
-        vn1 = fmaf(bf16_lo(v1), bf16_lo(v1), fmaf(bf16_hi(v1), bf16_hi(v1), vn1));
-        vn1 = fmaf(bf16_lo(v3), bf16_lo(v3), fmaf(bf16_hi(v3), bf16_hi(v3), vn1));
+        // v0, v2 token g, v1, v3 token g + 8 (two bf16 each; channels
+        // 16 kk + 2q (v0, v1) and 16 kk + 8 + 2q (v2, v3)): ||v||^2 (SPARE)
+        // or ||v - c||^2
+        float2 e0 = make_float2(bf16_lo(v0), bf16_hi(v0)), e2 = make_float2(bf16_lo(v2), bf16_hi(v2));
+        float2 e1 = make_float2(bf16_lo(v1), bf16_hi(v1)), e3 = make_float2(bf16_lo(v3), bf16_hi(v3));
+        if constexpr (!SPARE) {
+          const float2 ca = make_float2(bf16_lo(cp[kk][0]), bf16_hi(cp[kk][0]));
+          const float2 cb = make_float2(bf16_lo(cp[kk][1]), bf16_hi(cp[kk][1]));
+          e0 = __fadd2_rn(e0, ca);
+          e2 = __fadd2_rn(e2, cb);
+          e1 = __fadd2_rn(e1, ca);
+          e3 = __fadd2_rn(e3, cb);
+        }
+        vn0 = __ffma2_rn(e0, e0, __ffma2_rn(e2, e2, vn0));
+        vn1 = __ffma2_rn(e1, e1, __ffma2_rn(e3, e3, vn1));
       }
-      vn0 += __shfl_xor_sync(0xffffffffu, vn0, 1);
-      vn0 += __shfl_xor_sync(0xffffffffu, vn0, 2);
-      vn1 += __shfl_xor_sync(0xffffffffu, vn1, 1);
-      vn1 += __shfl_xor_sync(0xffffffffu, vn1, 2);
+      float vs0 = vn0.x + vn0.y, vs1 = vn1.x + vn1.y;
+      vs0 += __shfl_xor_sync(0xffffffffu, vs0, 1);
+      vs0 += __shfl_xor_sync(0xffffffffu, vs0, 2);
+      vs1 += __shfl_xor_sync(0xffffffffu, vs1, 1);
+      vs1 += __shfl_xor_sync(0xffffffffu, vs1, 2);
+      if constexpr (SPARE) {
+        // v.c of tokens g and g + 8 sits in column G: lane 4 g + G / 2
+        const int src = 4 * g + (G >> 1);
+        const float vc0 = __shfl_sync(0xffffffffu, (G & 1) ? vy[1] : vy[0], src);
+        const float vc1 = __shfl_sync(0xffffffffu, (G & 1) ? vy[3] : vy[2], src);
+        vs0 = vs0 - 2.f * vc0 + cc;  // ||v - c||^2
+        vs1 = vs1 - 2.f * vc1 + cc;
+      }
       // C fragment: st[0], st[1] = (token g, heads 2q, 2q+1); st[2], st[3] = (token g + 8, ...)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
@@ -247,8 +303,9 @@ __global__ void __launch_bounds__(kCtmWarps * 32)
         if (r >= nv || h >= G) continue;
         const float lw = slw[warp][slot][r];
         const float p = exp2f(fmaf(st[e], kscale, fmaf(lw, kLog2e, -l2[e & 1])));
-        const float vv = (e >> 1) ? vn1 : vn0;
-        const float dist = fmaxf(0.f, vv - 2.f * vy[e] + yy[e & 1]);
+        const float vv = (e >> 1) ? vs1 : vs0;  // ||v - c||^2
+        // (v - c).(y_hat - c) = v.(y_hat - c) - c.(y_hat - c)
+        const float dist = fmaxf(0.f, vv - 2.f * (vy[e] - cy[e & 1]) + yy[e & 1]);
         const float omp = lw > 0.f ? one_minus_exp_neg(lw) : 0.f;
         contrib[(hq0 + h) * cap + tok0 + r] = omp * p * p * dist;
       }
@@ -365,7 +422,9 @@ extern "C" ebd_status ebd_variance_contributions(ebd_dtype dtype, int32_t batch,
     const int per_cta = kCtmWarps * kCtmTilesPerWarp;
     const dim3 grid((ntiles + per_cta - 1) / per_cta, u);
     const int smem = kCtmWarps * kCtmStages * (2 * (head_dim / 64) * 16 * 128 + 16 * 4) + 1024;
-    auto kern = head_dim == 64 ? contrib_mma_kernel<64> : contrib_mma_kernel<128>;
+    const bool spare = group < 8;
+    auto kern = head_dim == 64 ? (spare ? contrib_mma_kernel<64, true> : contrib_mma_kernel<64, false>)
+                               : (spare ? contrib_mma_kernel<128, true> : contrib_mma_kernel<128, false>);
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
         cudaSuccess)
       return EBD_ERR_CUDA;

@@ -891,8 +891,12 @@ def test_snapkv_window_scores_match_oracle(E):
                                                (2, 2, 8, 64, 512, torch.bfloat16),
                                                (1, 3, 4, 128, 1000, torch.bfloat16),
                                                (1, 2, 4, 64, 300, torch.float32)])
-def test_variance_contributions_and_block_scores_match_oracle(E, B, H, G, d, cap, dtype):
-    Kc, Vc, logw, n = _synthetic_cache(B, H, cap, d, dtype, "random", seed=77)
+@pytest.mark.parametrize("vmean", [0.3, 16.0])
+def test_variance_contributions_and_block_scores_match_oracle(E, B, H, G, d, cap, dtype, vmean):
+    """Per-token terms of Theorem 2's V_hat and 64-token block scores; a common
+    mean of 16 on every value channel checks that each term is formed about a
+    retained row rather than from ||v||^2 - 2 v.y + ||y||^2."""
+    Kc, Vc, logw, n = _synthetic_cache(B, H, cap, d, dtype, "random", seed=77, vmean=vmean)
     idx = torch.sort(torch.randperm(cap * 4, generator=torch.Generator().manual_seed(5))[:cap])[0]
     idx_c = idx.int().view(1, 1, cap).expand(B, H, cap).contiguous()
     Q = torch.randn((B, H * G, d), generator=torch.Generator().manual_seed(8)).to(dtype)
