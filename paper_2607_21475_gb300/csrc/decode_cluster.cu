@@ -10,7 +10,8 @@
 // The partial states then meet without leaving the chip: the eight warps' in
 // shared memory (over the ring), where warp g combines query head g; the
 // cluster's CTAs' in the shared memory of CTA 0, written through distributed
-// shared memory; after one cluster barrier CTA 0 combines them and writes
+// shared memory; after one cluster barrier (which the other CTAs arrive at
+// and leave) CTA 0 combines them and writes
 // y_hat, log N_hat, V_hat, b_t and r_t (Eq. 3, Theorem 2, Eq. 4).  One launch,
 // no workspace, no merge kernel.  Combination rule: w-terms (l, o, cmax,
 // umax) scale by e^(M_part - M), u-terms (U, A2, A1) by its square; every
@@ -38,6 +39,7 @@ struct ClusterArgs {
   int csize;                // CTAs per cluster (per unit)
   int lw_off;               // shared-memory layout, bytes: log(1/pi) stages
   int lead_off;             // CTA records gathered in CTA 0: [csize][G][rec_floats(D)]
+  int cen_off;              // the unit's centring row (D bf16), staged for the finish
   float* y;
   float* lse;
   float* var;
@@ -85,6 +87,44 @@ struct HeadSum {
   }
 };
 
+// L2 prefetch of the first kPrefetchTiles tiles of a warp's range (K, V and
+// log(1/pi) rows; the ranges as in the kernel below), its n_kept value read
+// now; warp 0 also asks for the unit's query rows (G rows of D bf16 at q_rows)
+// and its centring row.  A few tiles per warp keep the prefetched bytes of all
+// resident CTAs far below the L2's size (152 x 8 x 32 KB).  The log(1/pi)
+// range is trimmed to whole 16-byte blocks.
+constexpr int kPrefetchTiles = 4;
+template <int D>
+__device__ __forceinline__ void prefetch_first_tiles(const __nv_bfloat16* Kc,
+                                                     const __nv_bfloat16* Vc, const float* logw,
+                                                     const __nv_bfloat16* q_rows, int G,
+                                                     const int32_t* n_kept_u, size_t row_base,
+                                                     int cap, uint32_t rank, int C, int warp,
+                                                     int lane) {
+  if (lane > 4) return;
+  const int n = min(max(ld_cg_s32(n_kept_u), 0), cap);
+  if (warp == 0 && lane >= 3) {
+    if (lane == 3) bulk_prefetch_l2(q_rows, (uint32_t)G * D * 2);
+    else if (n > 0) bulk_prefetch_l2(Vc + (row_base + centre_row(n)) * D, D * 2);
+    return;
+  }
+  if (lane > 2) return;
+  const int T = (n + kMmaTile - 1) / kMmaTile;
+  const int c0 = (int)((long long)rank * T / C), c1 = (int)((long long)(rank + 1) * T / C);
+  const int tb = c0 + (int)((long long)warp * (c1 - c0) / kMmaConsumers);
+  const int te = c0 + (int)((long long)(warp + 1) * (c1 - c0) / kMmaConsumers);
+  const int r0 = tb * kMmaTile, r1 = min(min(te, tb + kPrefetchTiles) * kMmaTile, n);
+  if (r1 <= r0) return;
+  if (lane < 2) {
+    const __nv_bfloat16* src = (lane == 0 ? Kc : Vc) + (row_base + r0) * D;
+    bulk_prefetch_l2(src, (uint32_t)(r1 - r0) * D * 2);
+  } else {
+    const uintptr_t b = (reinterpret_cast<uintptr_t>(logw + row_base + r0) + 15) & ~uintptr_t(15);
+    const uintptr_t e = reinterpret_cast<uintptr_t>(logw + row_base + r1) & ~uintptr_t(15);
+    if (e > b) bulk_prefetch_l2(reinterpret_cast<const void*>(b), (uint32_t)(e - b));
+  }
+}
+
 template <int D, int S, bool PACK>
 __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterArgs a) {
   using L = MmaTileLayout<D>;
@@ -95,25 +135,34 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
       (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);  // swizzle atoms
   float* lw_s = reinterpret_cast<float*>(smem + a.lw_off);
   float* lead = reinterpret_cast<float*>(smem + a.lead_off);
+  const __nv_bfloat16* cen_s = reinterpret_cast<const __nv_bfloat16*>(smem + a.cen_off);
 
-  // launched as a programmatic dependent: wait for the predecessor's outputs
-  // before the first read; let a following dependent launch early
-  grid_dependency_wait();
-  grid_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int C = a.csize, G = a.group;
   const uint32_t rank = cluster_rank();
   const int unit = blockIdx.x / C;
+  const size_t row_base = (size_t)unit * a.cap;
+  // launched as a programmatic dependent, this CTA may start while the
+  // predecessor runs: every warp asks L2 for the first tiles of its range,
+  // the range taken from a possibly stale n_kept (a hint; L2 prefetches never
+  // change what a load returns), so that the stream overlaps the
+  // predecessor's tail.  Every value it uses is read after the wait; then a
+  // following dependent may launch early.
+  prefetch_first_tiles<D>(a.Kc, a.Vc, a.logw, a.Q + (size_t)unit * a.gstride * D, G,
+                          a.n_kept + unit, row_base, a.cap, rank, C, warp, lane);
+  grid_dependency_wait();
+  grid_launch_dependents();
   const int n_u = min(max(__ldg(a.n_kept + unit), 0), a.cap);
   const int T = (n_u + kMmaTile - 1) / kMmaTile;
   const int c0 = (int)((long long)rank * T / C), c1 = (int)((long long)(rank + 1) * T / C);
   const int tb = c0 + (int)((long long)warp * (c1 - c0) / kMmaConsumers);
   const int te = c0 + (int)((long long)(warp + 1) * (c1 - c0) / kMmaConsumers);
   const float kscale = kLog2e * rsqrtf((float)D);
-  const size_t row_base = (size_t)unit * a.cap;
 
-  TileAcc<D> st;
-  tile_acc_begin<D, PACK>(st, a.Q, a.Vc, unit, G, a.gstride, a.cap, n_u, lane);
+  // CTA 0 stages the centring row for the finish with the first copies
+  const int cr = centre_row(n_u);
+  if (rank == 0 && warp == 0 && cr >= 0 && lane < D / 8)
+    cp_async16(smem + a.cen_off + 16 * lane, a.Vc + (row_base + cr) * D + 8 * lane);
   int issued = 0;
   auto issue_next = [&]() {
     const int t = tb + issued;
@@ -125,8 +174,12 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
     cp_async_commit();
     ++issued;
   };
+  // the first stages of the ring go out before the query and centring loads,
+  // whose latency they then hide
 #pragma unroll
   for (int p = 0; p < S - 1; ++p) issue_next();
+  TileAcc<D> st;
+  tile_acc_begin<D, PACK>(st, a.Q, a.Vc, unit, G, a.gstride, a.cap, n_u, lane);
   int j = 0;
   for (int t = tb; t < te; ++t, ++j) {
     issue_next();  // tile j + S - 1 into the stage tile j - 1 left
@@ -164,8 +217,11 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
       }
     }
   }
-  cluster_barrier();
+  // every thread arrives; only CTA 0's head warps wait for the records, the
+  // other CTAs leave at once and free their SMs for what follows
+  cluster_arrive_release();
   if (rank != 0 || warp >= G) return;
+  cluster_wait_acquire();
 
   HeadSum<D> h;
   h.combine<8>(lead + (size_t)warp * REC, C, (size_t)G * REC, lane);
@@ -182,7 +238,8 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
     return;
   }
   float c[PER], yv[PER], ynorm, ycnorm, var;
-  load_centre<__nv_bfloat16, D, PER>(a.Vc, unit, a.cap, n_u, lane, c);
+#pragma unroll
+  for (int e = 0; e < PER; ++e) c[e] = cr < 0 ? 0.f : __bfloat162float(cen_s[PER * lane + e]);
   finish_head<PER>(h.o, h.a1, c, h.l, h.U, h.A2, yv, ynorm, ycnorm, var);
 #pragma unroll
   for (int e = 0; e < PER; ++e) a.y[hq * D + PER * lane + e] = yv[e];
@@ -218,6 +275,7 @@ static ebd_status launch_cluster_t(const DecodeArgs& d, const ReduceArgs& r, int
   a.csize = C;
   a.lw_off = kMmaConsumers * S * L::kStageBytes;
   a.lead_off = (int)align_up((size_t)a.lw_off + (size_t)kMmaConsumers * S * kMmaTile * 4, 16);
+  a.cen_off = (int)align_up((size_t)a.lead_off + (size_t)C * d.group * rec_floats(D) * 4, 16);
   a.y = r.y;
   a.lse = r.lse;
   a.var = r.var;
@@ -226,7 +284,7 @@ static ebd_status launch_cluster_t(const DecodeArgs& d, const ReduceArgs& r, int
   a.log_inv_delta = r.log_inv_delta;
   a.eps0 = r.eps0;
   a.exact = r.exact;
-  const size_t smem = (size_t)a.lead_off + (size_t)C * d.group * rec_floats(D) * 4 + 1024;
+  const size_t smem = (size_t)a.cen_off + (size_t)D * 2 + 1024;
   if (cudaFuncSetAttribute(decode_cluster_kernel<D, S, PACK>,
                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return EBD_ERR_CUDA;
@@ -251,7 +309,7 @@ static ebd_status launch_cluster_t(const DecodeArgs& d, const ReduceArgs& r, int
 static size_t cluster_smem(int D, int S, int C, int G) {
   const size_t stage = (size_t)2 * (D / 64) * kMmaTile * 128;
   const size_t lw = align_up((size_t)kMmaConsumers * S * stage + kMmaConsumers * S * kMmaTile * 4, 16);
-  return lw + (size_t)C * G * rec_floats(D) * 4 + 1024;
+  return align_up(lw + (size_t)C * G * rec_floats(D) * 4, 16) + (size_t)D * 2 + 1024;
 }
 
 int cluster_decode_size(int units, int cap) {

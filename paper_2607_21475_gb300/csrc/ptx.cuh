@@ -88,6 +88,20 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
       : "memory");
 }
 
+// Bulk prefetch of global memory into L2 (16-byte aligned address, size % 16
+// == 0).  A hint: it changes no value any load returns, since L2 is where the
+// device's reads and writes meet, so it may run before a dependency wait.
+__device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
+// A 32-bit load that bypasses L1 (no line of it stays there for later loads).
+__device__ __forceinline__ int ld_cg_s32(const int32_t* p) {
+  int v;
+  asm volatile("ld.global.cg.s32 %0, [%1];" : "=r"(v) : "l"(p));
+  return v;
+}
+
 // 16-byte asynchronous copy global -> shared (L2 only), completion tracked per
 // thread by commit/wait groups.
 __device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc) {
@@ -177,6 +191,15 @@ __device__ __forceinline__ void cluster_barrier() {
   asm volatile(
       "barrier.cluster.arrive.release.aligned;\n\t"
       "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// The two halves of it: every thread of the cluster arrives once (its writes
+// before the arrival ordered before it); a thread that waits sees the writes
+// of every thread that arrived.  A thread may arrive and exit without waiting.
+__device__ __forceinline__ void cluster_arrive_release() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_acquire() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 }  // namespace ebd
