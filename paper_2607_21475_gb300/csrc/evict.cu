@@ -801,7 +801,9 @@ __device__ __forceinline__ void choose_digit(const unsigned* whist, RegScratch& 
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(kRegThreads, 1) evict_select_smem_kernel(SelectArgs a, int JG) {
+// 1024 threads of at most 56 registers (57,344 of the SM's 65,536) leave room
+// for one 128-thread gather CTA beside a select CTA in the pipelined eviction.
+__global__ void __maxnreg__(56) evict_select_smem_kernel(SelectArgs a, int JG) {
   extern __shared__ float4 s4[];  // [JG][1024]: scores of thread t, group g at s4[g*1024 + t]
   // followed by the per-warp radix histograms [kRegWarps][kHistStride]
   unsigned* whist = reinterpret_cast<unsigned*>(s4 + JG * kRegThreads);

@@ -682,6 +682,7 @@ def test_evict_then_decode_tiny_end_to_end(E):
     (1, 1, 33, 129, 128, torch.bfloat16),
     (1, 3, 512, 777, 64, torch.bfloat16),    # tcgen05 path at its 512-row limit, d = 64
     (3, 1, 129, 256, 128, torch.bfloat16),   # two 128-row tiles, one partial; N = one key tile
+    (2, 2, 256, 100, 128, torch.bfloat16),   # two full row tiles; N under half a key tile
     (1, 1, 1, 1, 128, torch.bfloat16),       # single row, single key
     (1, 2, 600, 500, 128, torch.bfloat16),   # above 512 rows: the mma.sync kernels
 ])
