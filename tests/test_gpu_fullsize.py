@@ -11,7 +11,7 @@ import pytest
 import torch
 
 from oracle import ebd_oracle as O
-from tests.parity import compare_decode_heads, compare_evict_unit
+from tests.parity import E0_RTOL, compare_decode_heads, compare_evict_unit
 
 pytestmark = pytest.mark.gpu
 
@@ -142,8 +142,7 @@ def test_fullsize_attention_scored_workload(E):
     for b, h in _sample_units(B, H):
         ref = O.accumulated_attention_scores(inp["q_obs"][b, h].double().cpu().numpy(),
                                              inp["K"][b, h].double().cpu().numpy())
-        np.testing.assert_allclose(scores[b, h].double().cpu().numpy(), ref, rtol=1e-4,
-                                   atol=1e-7 * R)
+        np.testing.assert_allclose(scores[b, h].double().cpu().numpy(), ref, rtol=E0_RTOL, atol=0)
     # the fused path (scores computed inside ebd_evict) keeps exactly what the
     # two-call path keeps on the scores ebd_score produced
     des = _design(E, w, layer)

@@ -8,7 +8,8 @@ import pytest
 import torch
 
 from oracle import ebd_oracle as O
-from tests.parity import TIE_BAND, compare_decode_heads, compare_evict_unit, oracle_unit
+from tests.parity import (E0_RTOL, TIE_BAND, compare_decode_heads, compare_evict_unit,
+                          oracle_unit)
 
 pytestmark = pytest.mark.gpu
 
@@ -697,7 +698,7 @@ def test_score_matches_oracle(E, B, H, R, N, d, dtype):
     for b in range(B):
         for h in range(H):
             ref = O.accumulated_attention_scores(q[b, h].double().numpy(), K[b, h].double().numpy())
-            np.testing.assert_allclose(got[b, h], ref, rtol=1e-4, atol=1e-7 * R)
+            np.testing.assert_allclose(got[b, h], ref, rtol=E0_RTOL, atol=0)
             assert abs(got[b, h].sum() - R) < 1e-3 * R
 
 
@@ -885,7 +886,7 @@ def test_snapkv_window_scores_match_oracle(E):
     for b in range(B):
         for h in range(H):
             ref = O.accumulated_attention_scores(qd[b, h], K[b, h].double().numpy())
-            np.testing.assert_allclose(f64(s)[b, h], ref, rtol=1e-4, atol=1e-7 * G * 64)
+            np.testing.assert_allclose(f64(s)[b, h], ref, rtol=E0_RTOL, atol=0)
 
 
 @pytest.mark.parametrize("B,H,G,d,cap,dtype", [(2, 4, 7, 128, 1600, torch.bfloat16),
