@@ -1,7 +1,8 @@
 // Certified decode on thread-block clusters: one cluster of C = 1, 2, 4 or 8
 // CTAs per (batch row, KV head) unit, C the largest that keeps units * C <=
-// SMs (C = 1: one CTA holds the whole unit and combines it alone; with more
-// units than SMs those CTAs run in waves).
+// SMs and gives every CTA at least 8 tiles at capacity (C = 1: one CTA holds
+// the whole unit and combines it alone; with more units than SMs those CTAs
+// run in waves).
 //
 // CTA r of a unit's cluster takes tiles [r T / C, (r + 1) T / C) of the unit's
 // T active 16-token tiles and splits them into eight contiguous ranges, one
@@ -331,11 +332,14 @@ int cluster_decode_size(int units, int cap) {
   int C = 1;  // one CTA per unit (no partner CTAs) when only one fits per SM
   while (C < 8 && 2 * C * units <= sms) C *= 2;
   // measured: the on-chip combine pays off when every CTA has a few tiles to
-  // stream (at least 8 at capacity) and either the clusters cover most SMs or,
-  // with fewer CTAs, each CTA's share stays within what one SM streams quickly
-  // (at most 160 tiles: on 4 units the single launch beats the split-K pair by
-  // up to 20% there, and loses beyond ~250 tiles); otherwise the split-K
-  // kernels over every SM are faster
+  // stream (at least 8 at capacity; fewer CTAs per unit rather than the
+  // split-K pair when the largest C leaves less: 4k contexts at 5-10% on 4 or
+  // 32 units, 15.5-16.9 -> 10.7-12.3 us) and either the clusters cover most
+  // SMs or, with fewer CTAs, each CTA's share stays within what one SM
+  // streams quickly (at most 160 tiles: on 4 units the single launch beats the
+  // split-K pair by up to 20% there, and loses beyond ~250 tiles); otherwise
+  // the split-K kernels over every SM are faster
+  while (C > 1 && (cap / kMmaTile) / C < 8) C /= 2;
   const int per_cta = (cap / kMmaTile) / C;
   if (per_cta < 8) return 0;
   if (4 * units * C < 3 * sms && per_cta > 160) return 0;
