@@ -551,9 +551,12 @@ static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, con
   m.exact = r.exact;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)((long long)units * a.group));
-  // a few records per head: 2 warps (one wave of CTAs); many: 8 warps
-  const bool wide = (long long)plan.ctas * kMmaConsumers > 12LL * units;
-  cfg.blockDim = dim3((wide ? 8 : 2) * 32);
+  // a few records per head: 2 warps (one wave of CTAs); many: 8 warps;
+  // hundreds (few long units): 16 warps, so that each keeps few rounds of
+  // record loads in flight
+  const long long per_unit = (long long)plan.ctas * kMmaConsumers / units;
+  const int mw = per_unit > 96 ? 16 : per_unit > 12 ? 8 : 2;
+  cfg.blockDim = dim3(mw * 32);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -561,7 +564,8 @@ static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, con
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  if (wide) return cuda_status(cudaLaunchKernelEx(&cfg, decode_merge_kernel<D, 8>, m));
+  if (mw == 16) return cuda_status(cudaLaunchKernelEx(&cfg, decode_merge_kernel<D, 16>, m));
+  if (mw == 8) return cuda_status(cudaLaunchKernelEx(&cfg, decode_merge_kernel<D, 8>, m));
   return cuda_status(cudaLaunchKernelEx(&cfg, decode_merge_kernel<D, 2>, m));
 }
 
