@@ -891,6 +891,8 @@ def test_snapkv_window_scores_match_oracle(E):
 
 @pytest.mark.parametrize("B,H,G,d,cap,dtype", [(2, 4, 7, 128, 1600, torch.bfloat16),
                                                (2, 2, 8, 64, 512, torch.bfloat16),
+                                               (1, 2, 8, 128, 256, torch.bfloat16),
+                                               (1, 2, 3, 64, 320, torch.bfloat16),
                                                (1, 3, 4, 128, 1000, torch.bfloat16),
                                                (1, 2, 4, 64, 300, torch.float32)])
 @pytest.mark.parametrize("vmean", [0.3, 16.0])
