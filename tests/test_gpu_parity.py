@@ -807,6 +807,56 @@ def test_append_then_reevict_then_decode_matches_oracle(E):
     print("near ties", ties)
 
 
+def test_append_and_decode_back_to_back_match_oracle(E):
+    """Append -> certified decode, six times back to back on one stream with no
+    synchronisation: the append lets its successor launch early, so each
+    decode starts (and asks L2 for its rows, from a possibly stale n_kept)
+    while the append that writes its last row, n_kept and log(1/pi) may still
+    run.  Every step's outputs are checked against the oracle on that step's
+    cache (the evicted rows plus the rows appended so far, pi = 1)."""
+    from paper_2607_21475_gb300.workloads import WORKLOADS, make_layer_inputs
+    w = WORKLOADS["qwen7b_16k_b25"].with_(batch=2, n_ctx=6000)
+    layer, steps = 3, 6
+    inp = make_layer_inputs(w, layer, DEV)
+    B, H, G, d, N = w.batch, w.n_kv_heads, w.group, w.head_dim, w.n_ctx
+    # whole 16-row tiles: the tensor-core path (8 units: clusters of 8 CTAs)
+    cap = (w.capacity + steps + 15) // 16 * 16
+    des = _design(E, B, H, G, d, N, layer, w.philox_seed, w.k_head, w.budget_tokens)
+    cc = E.alloc_compact(B, H, cap, d, w.torch_dtype, DEV)
+    E.ebd_evict(des, inp["K"], inp["V"], inp["scores"], None, cc)
+    torch.cuda.synchronize()
+    assert cc.dev_status.item() == 0
+    n0 = cc.n_kept.cpu().numpy().copy()
+    assert n0.max() + steps <= cap
+    K0 = [[cc.K_c[b, h, :n0[b, h]].double().cpu().numpy() for h in range(H)] for b in range(B)]
+    V0 = [[cc.V_c[b, h, :n0[b, h]].double().cpu().numpy() for h in range(H)] for b in range(B)]
+    L0 = [[cc.logw_c[b, h, :n0[b, h]].double().cpu().numpy() for h in range(H)] for b in range(B)]
+    g = torch.Generator().manual_seed(29)
+    k_new = torch.randn((steps, B, H, d), generator=g).to(w.torch_dtype).to(DEV)
+    v_new = (torch.randn((steps, B, H, d), generator=g) + 0.5).to(w.torch_dtype).to(DEV)
+    qs = torch.randn((steps, B, H * G, d), generator=g).to(w.torch_dtype).to(DEV)
+    outs = []
+    for t in range(steps):  # all enqueued, one synchronisation at the end
+        E.ebd_append(cc, k_new[t], v_new[t], torch.full((B,), N + t, dtype=torch.int32, device=DEV))
+        y = torch.full((B, H * G, d), float("nan"), device=DEV)
+        rest = [torch.full((B, H * G), float("nan"), device=DEV) for _ in range(4)]
+        E.ebd_certified_decode(qs[t], cc.K_c, cc.V_c, cc.logw_c, cc.n_kept, y, *rest)
+        outs.append([y] + rest)
+    torch.cuda.synchronize()
+    assert cc.dev_status.item() == 0
+    kn, vn = k_new.double().cpu().numpy(), v_new.double().cpu().numpy()
+    for t in range(steps):
+        got = [o.double().cpu().numpy() for o in outs[t]]
+        for b in range(B):
+            for h in range(H):
+                K = np.concatenate([K0[b][h], kn[:t + 1, b, h]])
+                V = np.concatenate([V0[b][h], vn[:t + 1, b, h]])
+                lw = np.concatenate([L0[b][h], np.zeros(t + 1)])
+                dec = O.hajek_decode(qs[t, b, h * G:(h + 1) * G].double().cpu().numpy(), K, V, lw)
+                sl = slice(h * G, (h + 1) * G)
+                compare_decode_heads(dec, *(x[b, sl] for x in got), False)
+
+
 # ------------------------------------------------------- systematic design
 @pytest.mark.parametrize("B,H,N,budget,dist", [(2, 3, 1000, 100, "lognormal"),
                                                (1, 4, 20000, 2000, "pareto"),
