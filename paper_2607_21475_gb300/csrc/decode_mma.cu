@@ -294,8 +294,12 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
 // own maximum: every lane reads the same record headers and D/32 columns of o
 // and A1.  The MW warp partials are then combined in shared memory by warp 0,
 // which writes the outputs.  Records of unit u: index u + gw for every working
-// decode warp gw whose tile range meets u.
-template <int D, int MW>
+// decode warp gw whose tile range meets u.  With CL > 1 a cluster of CL CTAs
+// takes one query head, CTA r the r-th of CL equal slices of its records;
+// each CTA's combined part goes to CTA 0 through distributed shared memory,
+// every thread arrives at the cluster barrier, and CTA 0 (warp 0) waits,
+// combines the CL parts in rank order and writes the outputs.
+template <int D, int MW, int CL>
 __global__ void __launch_bounds__(MW * 32) decode_merge_kernel(MergeArgs a) {
   constexpr int REC = rec_floats(D);
   constexpr int PER = D / 32;
@@ -303,16 +307,19 @@ __global__ void __launch_bounds__(MW * 32) decode_merge_kernel(MergeArgs a) {
   __shared__ float sh_s[MW][8];  // M, l, U, A2, cmax, umax per warp
   __shared__ __align__(16) float sh_o[MW][D];
   __shared__ __align__(16) float sh_a[MW][D];
+  __shared__ __align__(16) float lead[CL][8 + 2 * D];  // CTA parts, in CTA 0
   grid_dependency_wait();
   grid_launch_dependents();  // a following dependent grid may launch now
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = a.group;
-  const int u = (int)(blockIdx.x / G), g = (int)(blockIdx.x - u * G);
+  const int head = (int)(blockIdx.x / CL);
+  const uint32_t rank = CL > 1 ? cluster_rank() : 0u;
+  const int u = head / G, g = head - u * G;
   const long long hq = (long long)u * a.gstride + g;  // output row
   const long long t0 = a.tile_off[u], t1 = a.tile_off[u + 1];
   if (t1 == t0) {  // no retained row: y = 0, lse = -inf, zero certificate
-    if (warp == 0) {
+    if (warp == 0 && rank == 0) {
 #pragma unroll
       for (int e = 0; e < PER; ++e) a.y[hq * D + PER * lane + e] = 0.f;
       if (lane == 0) {
@@ -329,6 +336,8 @@ __global__ void __launch_bounds__(MW * 32) decode_merge_kernel(MergeArgs a) {
   const long long gf = ((t0 + 1) * W - 1) / Ta;  // first decode warp meeting u
   const long long gl = (t1 * W - 1) / Ta;        // last
   const int count = (int)(gl - gf + 1);
+  // this CTA's slice of the head's records
+  const int kb = (int)((long long)rank * count / CL), ke = (int)((long long)(rank + 1) * count / CL);
   const float* R0 = a.part + ((size_t)(u + gf) * G + g) * REC;
   const size_t slot = (size_t)G * REC;
 
@@ -336,14 +345,14 @@ __global__ void __launch_bounds__(MW * 32) decode_merge_kernel(MergeArgs a) {
   float o[PER], a1[PER];
 #pragma unroll
   for (int e = 0; e < PER; ++e) o[e] = a1[e] = 0.f;
-  for (int k0 = warp; k0 < count; k0 += BATCH * MW) {
+  for (int k0 = kb + warp; k0 < ke; k0 += BATCH * MW) {
     float4 h[BATCH];
     float2 c[BATCH];
     float ov[BATCH][PER], av[BATCH][PER];
 #pragma unroll
     for (int i = 0; i < BATCH; ++i) {
       const int k = k0 + i * MW;
-      if (k < count) {
+      if (k < ke) {
         const float* R = R0 + k * slot;
         h[i] = __ldcg(reinterpret_cast<const float4*>(R));
         c[i] = __ldcg(reinterpret_cast<const float2*>(R + kRecCmax));
@@ -412,29 +421,74 @@ __global__ void __launch_bounds__(MW * 32) decode_merge_kernel(MergeArgs a) {
     sh_a[warp][PER * lane + e] = a1[e];
   }
   __syncthreads();
-  if (warp != 0) return;
 
   float Mx = -INFINITY;
+  if (warp == 0) {
 #pragma unroll
-  for (int w = 0; w < MW; ++w) Mx = fmaxf(Mx, sh_s[w][0]);
-  l = U = A2 = cm = um = 0.f;
+    for (int w = 0; w < MW; ++w) Mx = fmaxf(Mx, sh_s[w][0]);
+    l = U = A2 = cm = um = 0.f;
 #pragma unroll
-  for (int e = 0; e < PER; ++e) o[e] = a1[e] = 0.f;
+    for (int e = 0; e < PER; ++e) o[e] = a1[e] = 0.f;
 #pragma unroll
-  for (int w = 0; w < MW; ++w) {
-    const float Ms = sh_s[w][0];
-    if (Ms == -INFINITY) continue;
-    const float f = expf(Ms - Mx), f2 = f * f;
-    l = fmaf(f, sh_s[w][1], l);
-    U = fmaf(f2, sh_s[w][2], U);
-    A2 = fmaf(f2, sh_s[w][3], A2);
-    cm = fmaxf(cm, f * sh_s[w][4]);
-    um = fmaxf(um, f * sh_s[w][5]);
+    for (int w = 0; w < MW; ++w) {
+      const float Ms = sh_s[w][0];
+      if (Ms == -INFINITY) continue;
+      const float f = expf(Ms - Mx), f2 = f * f;
+      l = fmaf(f, sh_s[w][1], l);
+      U = fmaf(f2, sh_s[w][2], U);
+      A2 = fmaf(f2, sh_s[w][3], A2);
+      cm = fmaxf(cm, f * sh_s[w][4]);
+      um = fmaxf(um, f * sh_s[w][5]);
 #pragma unroll
-    for (int e = 0; e < PER; ++e) {
-      o[e] = fmaf(f, sh_o[w][PER * lane + e], o[e]);
-      a1[e] = fmaf(f2, sh_a[w][PER * lane + e], a1[e]);
+      for (int e = 0; e < PER; ++e) {
+        o[e] = fmaf(f, sh_o[w][PER * lane + e], o[e]);
+        a1[e] = fmaf(f2, sh_a[w][PER * lane + e], a1[e]);
+      }
     }
+  }
+  if constexpr (CL > 1) {
+    if (warp == 0) {  // this CTA's part, to CTA 0
+      const uint32_t dst = cluster_map(smem_u32(&lead[rank][0]), 0);
+      if (lane == 0) {
+        st_cluster4(dst, Mx, l, U, A2);
+        st_cluster4(dst + 16, cm, um, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int e = 0; e < PER; e += 2) {
+        asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(dst + 4 * (8 + PER * lane + e)),
+                     "f"(o[e]), "f"(o[e + 1]) : "memory");
+        asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(dst + 4 * (8 + D + PER * lane + e)),
+                     "f"(a1[e]), "f"(a1[e + 1]) : "memory");
+      }
+    }
+    // every thread arrives; CTA 0's warp 0 alone waits for the parts
+    cluster_arrive_release();
+    if (rank != 0 || warp != 0) return;
+    cluster_wait_acquire();
+    Mx = -INFINITY;
+#pragma unroll
+    for (int r = 0; r < CL; ++r) Mx = fmaxf(Mx, lead[r][0]);
+    l = U = A2 = cm = um = 0.f;
+#pragma unroll
+    for (int e = 0; e < PER; ++e) o[e] = a1[e] = 0.f;
+#pragma unroll
+    for (int r = 0; r < CL; ++r) {
+      const float Ms = lead[r][0];
+      if (Ms == -INFINITY) continue;
+      const float f = expf(Ms - Mx), f2 = f * f;
+      l = fmaf(f, lead[r][1], l);
+      U = fmaf(f2, lead[r][2], U);
+      A2 = fmaf(f2, lead[r][3], A2);
+      cm = fmaxf(cm, f * lead[r][4]);
+      um = fmaxf(um, f * lead[r][5]);
+#pragma unroll
+      for (int e = 0; e < PER; ++e) {
+        o[e] = fmaf(f, lead[r][8 + PER * lane + e], o[e]);
+        a1[e] = fmaf(f2, lead[r][8 + D + PER * lane + e], a1[e]);
+      }
+    }
+  } else {
+    if (warp != 0) return;
   }
   float c[PER], yv[PER], ynorm, ycnorm, var;
   load_centre<__nv_bfloat16, D, PER>(a.Vc, u, a.cap, min(max(__ldg(a.n_kept + u), 0), a.cap),
@@ -550,23 +604,34 @@ static ebd_status launch_fast_t(const DecodePlan& plan, const DecodeArgs& a, con
   m.eps0 = r.eps0;
   m.exact = r.exact;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)((long long)units * a.group));
+  const long long heads = (long long)units * a.group;
+  cfg.gridDim = dim3((unsigned)heads);
   // a few records per head: 2 warps (one wave of CTAs); many: 8 warps;
-  // hundreds (few long units): 16 warps, so that each keeps few rounds of
-  // record loads in flight
+  // hundreds (few long units): clusters of 4 CTAs of 16 warps per head, so
+  // that more SMs share the records and each warp keeps few rounds of record
+  // loads in flight
   const long long per_unit = (long long)plan.ctas * kMmaConsumers / units;
   const int mw = per_unit > 96 ? 16 : per_unit > 12 ? 8 : 2;
   cfg.blockDim = dim3(mw * 32);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  if (mw == 16) return cuda_status(cudaLaunchKernelEx(&cfg, decode_merge_kernel<D, 16>, m));
-  if (mw == 8) return cuda_status(cudaLaunchKernelEx(&cfg, decode_merge_kernel<D, 8>, m));
-  return cuda_status(cudaLaunchKernelEx(&cfg, decode_merge_kernel<D, 2>, m));
+  if (mw == 16) {
+    constexpr int CL = 4;
+    cfg.gridDim = dim3((unsigned)(heads * CL));
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = CL;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.numAttrs = 2;
+    return cuda_status(cudaLaunchKernelEx(&cfg, decode_merge_kernel<D, 16, CL>, m));
+  }
+  if (mw == 8) return cuda_status(cudaLaunchKernelEx(&cfg, decode_merge_kernel<D, 8, 1>, m));
+  return cuda_status(cudaLaunchKernelEx(&cfg, decode_merge_kernel<D, 2, 1>, m));
 }
 
 ebd_status launch_fast_decode(ebd_dtype dtype, int head_dim, const DecodePlan& plan,

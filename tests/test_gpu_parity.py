@@ -411,6 +411,9 @@ DECODE_CASES = [
     (2, 3, 5, 128, 1000, torch.bfloat16, "random"),  # capacity not a multiple of 16: CUDA cores
     (1, 64, 4, 128, 256, torch.bfloat16, "random"),  # more warps than tiles
     (1, 1, 8, 128, 32768, torch.bfloat16, "full"),    # one unit, hundreds of partial records
+    # few long units: split-K, each head's records merged by a cluster of CTAs
+    (2, 2, 4, 128, 24576, torch.bfloat16, "edges"),   # empty and one-row units among them
+    (1, 2, 4, 64, 16384, torch.bfloat16, "random"),   # head_dim 64
     # cluster kernel (units * C covering most SMs, long per-CTA ranges)
     (16, 4, 7, 128, 1600, torch.bfloat16, "edges"),   # 64 units, clusters of 2, empty units
     (8, 8, 8, 64, 1600, torch.bfloat16, "random"),    # head_dim 64, G = 8
