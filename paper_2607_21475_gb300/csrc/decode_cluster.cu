@@ -12,7 +12,8 @@
 // shared memory (over the ring), where warp g combines query head g; the
 // cluster's CTAs' in the shared memory of CTA 0, written through distributed
 // shared memory; after one cluster barrier (which the other CTAs arrive at
-// and leave) CTA 0 combines them and writes
+// and leave) CTA 0 combines them and writes (with one CTA per unit its own
+// combine is the head's state, and it writes at once)
 // y_hat, log N_hat, V_hat, b_t and r_t (Eq. 3, Theorem 2, Eq. 4).  One launch,
 // no workspace, no merge kernel.  Combination rule: w-terms (l, o, cmax,
 // umax) scale by e^(M_part - M), u-terms (U, A2, A1) by its square; every
@@ -196,36 +197,39 @@ __global__ void __launch_bounds__(kMmaThreads, 1) decode_cluster_kernel(ClusterA
   float* wrec = reinterpret_cast<float*>(smem);  // [warps][G][REC]
   tile_acc_store<D, PACK>(st, wrec + (size_t)warp * G * REC, G, lane);
   __syncthreads();
-  if (warp < G) {  // this CTA's part of query head `warp`, sent to CTA 0
-    HeadSum<D> h;
+  HeadSum<D> h;  // this CTA's part of query head `warp`
+  if (warp < G)
     h.combine<kMmaConsumers>(wrec + (size_t)warp * REC, kMmaConsumers, (size_t)G * REC, lane);
-    const uint32_t dst = cluster_map(smem_u32(lead + ((size_t)rank * G + warp) * REC), 0);
-    if (lane == 0) {
-      st_cluster4(dst + 4 * kRecM, h.M, h.l, h.U, h.A2);
-      st_cluster4(dst + 4 * kRecCmax, h.cm, h.um, 0.f, 0.f);
-    }
-    if constexpr (PER == 4) {  // 16-byte stores: lane holds columns 4 lane .. + 3
-      st_cluster4(dst + 4 * (kRecHead + 4 * lane), h.o[0], h.o[1], h.o[2], h.o[3]);
-      st_cluster4(dst + 4 * (kRecHead + D + 4 * lane), h.a1[0], h.a1[1], h.a1[2], h.a1[3]);
-    } else {  // lanes 2k and 2k + 1 hold columns 4k .. 4k + 3: even lanes store both
-      const float o2 = __shfl_down_sync(0xffffffffu, h.o[0], 1);
-      const float o3 = __shfl_down_sync(0xffffffffu, h.o[1], 1);
-      const float b2 = __shfl_down_sync(0xffffffffu, h.a1[0], 1);
-      const float b3 = __shfl_down_sync(0xffffffffu, h.a1[1], 1);
-      if ((lane & 1) == 0) {
-        st_cluster4(dst + 4 * (kRecHead + 2 * lane), h.o[0], h.o[1], o2, o3);
-        st_cluster4(dst + 4 * (kRecHead + D + 2 * lane), h.a1[0], h.a1[1], b2, b3);
+  if (C > 1) {
+    if (warp < G) {  // sent to CTA 0
+      const uint32_t dst = cluster_map(smem_u32(lead + ((size_t)rank * G + warp) * REC), 0);
+      if (lane == 0) {
+        st_cluster4(dst + 4 * kRecM, h.M, h.l, h.U, h.A2);
+        st_cluster4(dst + 4 * kRecCmax, h.cm, h.um, 0.f, 0.f);
+      }
+      if constexpr (PER == 4) {  // 16-byte stores: lane holds columns 4 lane .. + 3
+        st_cluster4(dst + 4 * (kRecHead + 4 * lane), h.o[0], h.o[1], h.o[2], h.o[3]);
+        st_cluster4(dst + 4 * (kRecHead + D + 4 * lane), h.a1[0], h.a1[1], h.a1[2], h.a1[3]);
+      } else {  // lanes 2k and 2k + 1 hold columns 4k .. 4k + 3: even lanes store both
+        const float o2 = __shfl_down_sync(0xffffffffu, h.o[0], 1);
+        const float o3 = __shfl_down_sync(0xffffffffu, h.o[1], 1);
+        const float b2 = __shfl_down_sync(0xffffffffu, h.a1[0], 1);
+        const float b3 = __shfl_down_sync(0xffffffffu, h.a1[1], 1);
+        if ((lane & 1) == 0) {
+          st_cluster4(dst + 4 * (kRecHead + 2 * lane), h.o[0], h.o[1], o2, o3);
+          st_cluster4(dst + 4 * (kRecHead + D + 2 * lane), h.a1[0], h.a1[1], b2, b3);
+        }
       }
     }
+    // every thread arrives; only CTA 0's head warps wait for the records, the
+    // other CTAs leave at once and free their SMs for what follows
+    cluster_arrive_release();
+    if (rank != 0 || warp >= G) return;
+    cluster_wait_acquire();
+    h.combine<8>(lead + (size_t)warp * REC, C, (size_t)G * REC, lane);
+  } else if (warp >= G) {
+    return;  // one CTA per unit: its part is the head's whole state
   }
-  // every thread arrives; only CTA 0's head warps wait for the records, the
-  // other CTAs leave at once and free their SMs for what follows
-  cluster_arrive_release();
-  if (rank != 0 || warp >= G) return;
-  cluster_wait_acquire();
-
-  HeadSum<D> h;
-  h.combine<8>(lead + (size_t)warp * REC, C, (size_t)G * REC, lane);
   const long long hq = (long long)unit * a.gstride + warp;
   if (h.M == -INFINITY) {  // no retained row: y = 0, lse = -inf, zero certificate
 #pragma unroll
