@@ -12,12 +12,15 @@
 // shared memory (over the ring), where warp g combines query head g; the
 // cluster's CTAs' in the shared memory of CTA 0, written through distributed
 // shared memory; after one cluster barrier (which the other CTAs arrive at
-// and leave) CTA 0 combines them and writes (with one CTA per unit its own
-// combine is the head's state, and it writes at once)
-// y_hat, log N_hat, V_hat, b_t and r_t (Eq. 3, Theorem 2, Eq. 4).  One launch,
-// no workspace, no merge kernel.  Combination rule: w-terms (l, o, cmax,
-// umax) scale by e^(M_part - M), u-terms (U, A2, A1) by its square; every
-// part takes A2 about the unit's centring row (decode.cuh).
+// and leave) CTA 0 combines them and writes y_hat, log N_hat, V_hat, b_t and
+// r_t (Eq. 3, Theorem 2, Eq. 4).  With one CTA per unit its own combine is
+// the head's state and it writes at once.  One launch, no workspace, no merge
+// kernel.  Combination rule: w-terms (l, o, cmax, umax) scale by
+// e^(M_part - M), u-terms (U, A2, A1) by its square; every part takes A2
+// about the unit's centring row (decode.cuh).  Launched as a programmatic
+// dependent, each CTA asks L2 for the first tiles of its warps' ranges before
+// its dependency wait, so that a layer's stream starts under the tail of the
+// launch before it.
 #include <cuda_runtime.h>
 #include <math.h>
 
