@@ -20,8 +20,9 @@
 // reloading Q only when the unit changes.
 //
 // Roles: warps 0-15 are the epilogue (warps w, w + 4, w + 8, w + 12 read
-// tensor-memory lanes 32 (w % 4) .. + 31 and take every fourth 32-column chunk
-// of the accumulator); warp 16 allocates tensor memory and one of its lanes
+// tensor-memory lanes 32 (w % 4) .. + 31; in pass 1 warp w takes the 64
+// columns from 64 (w / 4) on, in pass 2 every fourth 32-column chunk of the
+// accumulator); warp 16 allocates tensor memory and one of its lanes
 // issues the TMA copies (128-byte swizzle) and the tcgen05.mma instructions.
 // Hand-offs use mbarriers: TMA -> MMA (transaction counts), MMA -> epilogue
 // and MMA -> smem reuse (tcgen05.commit), epilogue -> MMA (512 arrivals).  The
@@ -212,7 +213,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     __syncwarp();
   } else {
-    // epilogue: thread = query row (tensor-memory lane) x every fourth 32-key chunk
+    // epilogue: thread = query row (tensor-memory lane) x 64 keys of each tile
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const float sc = a.scale2;
     for (int j = 0; j < nk; ++j) {
@@ -223,22 +224,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
       tc_fence_after();
       const int kvalid = a.n_ctx - j * kTcKeys1;  // keys of this tile inside the unit
-      // this warp's two 32-key chunks (grp and grp + 4) loaded together, one
-      // wait, one running-max update and one pass of exponentials over 64 keys
-      const int nv0 = kvalid - grp * 32, nv1 = nv0 - 4 * 32;
-      if (nv0 > 0) {
+      // this warp's 64 keys (columns 64 grp ..) in one load, one wait, one
+      // running-max update and one pass of exponentials
+      const int nv = kvalid - grp * 64;
+      if (nv > 0) {
         uint32_t r[64];
-        tmem_ld32(tmem + lane_base + b * kTcKeys1 + grp * 32,
-                  *reinterpret_cast<uint32_t(*)[32]>(r));
-        tmem_ld32(tmem + lane_base + b * kTcKeys1 + (grp + 4) * 32,
-                  *reinterpret_cast<uint32_t(*)[32]>(r + 32));
+        tmem_ld64(tmem + lane_base + b * kTcKeys1 + grp * 64, r);
         tmem_ld_wait();
-        if (nv0 < 32 || nv1 < 32) {  // the unit's last keys: the rest belongs to the next unit
+        if (nv < 64) {  // the unit's last keys: the rest belongs to the next unit
 #pragma unroll
-          for (int i = 0; i < 64; ++i) {
-            const bool in = i < 32 ? i < nv0 : i - 32 < nv1;
-            if (!in) r[i] = __float_as_uint(-INFINITY);
-          }
+          for (int i = 0; i < 64; ++i)
+            if (i >= nv) r[i] = __float_as_uint(-INFINITY);
         }
         float m4[4] = {__uint_as_float(r[0]), __uint_as_float(r[1]), __uint_as_float(r[2]),
                        __uint_as_float(r[3])};
