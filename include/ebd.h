@@ -20,12 +20,13 @@
  *   by the matching *_workspace_bytes query.
  * - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
  *   stream).  Every call only enqueues work on it and returns: results are
- *   valid once the stream has been synchronised.  The certified decode (and
- *   its merge) and ebd_append are launched as programmatic dependents of
- *   whatever precedes them on the stream: they may start while it runs, but
- *   read and write memory only after it has completed, except for L2
- *   prefetch hints (of the compact-cache rows, queries and n_kept-sized
- *   ranges), which never change what a load returns.
+ *   valid once the stream has been synchronised.  The tensor-core kernels of
+ *   the certified decode (and its merge) are launched as programmatic
+ *   dependents of whatever precedes them on the stream, and ebd_append lets
+ *   what follows it launch early: a decode may start while its predecessor
+ *   runs, but reads and writes memory only after that has completed, except
+ *   for L2 prefetch hints (of its compact-cache rows and queries), which
+ *   never change what a load returns.
  * - Tensors are dense, row-major, with the last dimension contiguous.
  *   B = batch, Hkv = KV heads, G = query heads per KV head (Hq = Hkv * G),
  *   d = head_dim, N = context length, cap = compact-cache capacity per unit.
