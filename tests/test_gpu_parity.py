@@ -498,6 +498,8 @@ MEAN_CASES = [
     (1, 4, 7, 128, 1600, torch.bfloat16, "random", 4.0, 4),    # clusters of 8
     (32, 8, 4, 128, 256, torch.bfloat16, "edges", 16.0, 0),    # one CTA per unit, 2 waves
     (1, 1, 8, 128, 32768, torch.bfloat16, "full", 16.0, 0),    # split-K, one unit
+    (2, 2, 4, 128, 24576, torch.bfloat16, "edges", 4.0, 4),    # few long units: clustered merge
+    (2, 4, 7, 128, 256, torch.bfloat16, "random", 16.0, 0),    # clusters shrunk to 8 tiles per CTA
     (20, 10, 4, 128, 256, torch.bfloat16, "edges", 4.0, 4),    # split-K, 200 units
     (2, 2, 8, 64, 512, torch.bfloat16, "edges", 16.0, 0),      # split-K, head_dim 64
     (2, 2, 8, 64, 320, torch.float32, "edges", 16.0, 0),       # CUDA cores, float32
