@@ -468,11 +468,24 @@ def e2e_run(path: Path, steps: int, in_place: bool, n_kept_layers=None):
         ev_ws = torch.empty(ebd.ebd_evict_workspace_bytes(path.designs[0], w.n_obs * w.group),
                             dtype=torch.uint8, device=dev)
 
+    # the copies run on their own stream, layer after layer, while the
+    # compute stream works on the layers already copied (each layer waits for
+    # its own inputs only); a step's copies start after the previous step's
+    # compute, so no input buffer is overwritten while still read
+    comp = torch.cuda.current_stream()
+    copy_stream = torch.cuda.Stream(device=dev)
+    ready = [torch.cuda.Event() for _ in range(w.n_layers)]
+
     def one():
+        copy_stream.wait_stream(comp)
+        with torch.cuda.stream(copy_stream):
+            for l in range(w.n_layers):
+                for k in copied:
+                    path.inputs[l][k].copy_(host_in[l][k], non_blocking=True)
+                ready[l].record(copy_stream)
         for l in range(w.n_layers):
             inp, hi = path.inputs[l], host_in[l]
-            for k in copied:
-                inp[k].copy_(hi[k], non_blocking=True)
+            comp.wait_event(ready[l])
             def src(k):
                 return inp[k] if k in copied else hi[k]
             cc, o = path.cc[l], path.out[l]
